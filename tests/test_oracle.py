@@ -1,0 +1,100 @@
+"""The CPU oracle against the paper's printed values, closed forms and brute force (no GPU)."""
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_13692_gb300 import instances as I
+from tests import oracle_pins as P
+
+
+@pytest.fixture(scope="module")
+def C():
+    return O.COracle(O.build())
+
+
+@pytest.mark.parametrize("pin", P.ALL_PINS, ids=lambda f: f.__name__)
+def test_pin(C, pin):
+    pin(C)
+
+
+def test_closed_forms_match_printed_table():
+    """Thm 5 closed forms against the Sec. 5.1 table and the Sec. 6.2 values."""
+    for n, free, glob in P.GOLDEN["leave_one_out_table"]["rows"]:
+        assert O.loo_free(n) == free and O.loo_glob(n) == glob
+    for n, free in P.GOLDEN["greedy_on_loo"]["rows"]:
+        assert O.loo_free(n) == free
+    g = P.GOLDEN["leave_one_out_caterpillar"]
+    assert O.loo_glob(g["n"]) == g["cost"]
+    assert O.loo_free(20) == 88
+
+
+def test_global_order_brute_force():
+    """OPT_glob by enumerating chunk orders: Thm 4 (9), Sec. 10.1 (21), Thm 5 (L_n)."""
+    assert O.brute_force_global_order(I.k4_3().weights, I.k4_3().bits) == P.GOLDEN["k4_3"]["opt_glob"]
+    inst = I.open_problem_k4()
+    assert O.brute_force_global_order(inst.weights, inst.bits) == P.GOLDEN["open_problem_k4"]["opt_glob"]
+    for n in range(2, 7):
+        inst = I.leave_one_out(n)
+        assert O.brute_force_global_order(inst.weights, inst.bits) == O.loo_glob(n)
+
+
+def test_trie_cost_of_printed_layout():
+    """Thm 4 proof: the layout abc, abd, cda, cdb has a trie of 8 nodes."""
+    g = P.GOLDEN["k4_3"]
+    ids = {"a": 0, "b": 1, "c": 2, "d": 3}
+    perms = [[ids[c] for c in row] for row in g["layout_example"]]
+    assert O.trie_cost(np.ones(4, dtype=np.int64), perms) == g["layout_example_cost"]
+
+
+def test_thm7_dfs_order_one_request_cache(C):
+    """Thm 7: in the hierarchy's DFS order, a radix cache holding one request's
+    context (LRU leaf eviction) pays exactly the unbounded-cache cost."""
+    rng = np.random.default_rng(97)
+    for t in range(6):
+        inst = I.random_instance(int(rng.integers(3, 11)), 40, (2, 9), seed=int(rng.integers(1 << 30)),
+                                 wmin=1, wmax=20)
+        opt, F, wI, split = C.solve(inst.weights, inst.bits)
+        perms, dfs = O.layout(inst.weights, inst.bits, split)
+        cap = max(sum(int(inst.weights[x]) for x in p) for p in perms)
+        assert O.radix_cache_cost(inst.weights, perms, dfs, cap) == opt
+        # an unbounded cache pays the trie cost in any order
+        assert O.radix_cache_cost(inst.weights, perms, list(range(inst.m))[::-1], 10 ** 9) == opt
+    # with a tiny cache the simulator pays at least the trie cost
+    inst = I.config(1)
+    opt, F, wI, split = C.solve(inst.weights, inst.bits)
+    perms, dfs = O.layout(inst.weights, inst.bits, split)
+    assert O.radix_cache_cost(inst.weights, perms, dfs, 600) >= opt
+
+
+def test_config_instances_shapes():
+    for idx in (1, 2, 3):
+        inst = I.config(idx)
+        c = I.CONFIGS[idx]
+        assert inst.m == c["m"] and inst.n == c["n"]
+        assert inst.bits.shape == (c["m"], (c["n"] + 63) // 64) and inst.bits.dtype == np.uint64
+        assert inst.weights.dtype == np.int64 and inst.weights.min() >= 1
+        reqs = inst.requests()
+        if "k" in c:
+            assert all(len(r) == c["k"] for r in reqs)
+    again = I.config(3)
+    assert np.array_equal(again.bits, I.config(3).bits) and np.array_equal(again.weights, I.config(3).weights)
+    w = I.config(3).weights
+    assert 32 <= w.min() and w.max() <= 512 and 120 < w.mean() < 180
+
+
+def test_pack_roundtrip():
+    reqs = [[0, 63, 64, 129], [], [5]]
+    bits = I.pack_requests(reqs, 130)
+    assert I.unpack_requests(bits, 130) == [sorted(r) for r in reqs]
+
+
+def test_config1_and_config2_full(C):
+    """Config 2 is L_20: OPT = 88 (Thm 5); config 1's layout realises its OPT."""
+    inst = I.config(2)
+    assert C.solve(inst.weights, inst.bits)[0] == O.loo_free(20) == 88
+    inst = I.config(1)
+    opt, F, wI, split = C.solve(inst.weights, inst.bits)
+    perms, dfs = O.layout(inst.weights, inst.bits, split)
+    assert O.trie_cost(inst.weights, perms) == opt
+    assert O.spanning_tree_bound(inst.weights, inst.bits) <= opt <= O.global_order_cost(inst.weights, inst.bits)
