@@ -1,0 +1,161 @@
+/*
+ * mpt.h -- C ABI of the exact Minimum-Prefix-Trie (MPT) solver for GB300 (sm_103a).
+ *
+ * Problem (arxiv 2609.13692, Sec. 2, eq. 1): a universe of n chunks with
+ * positive integer token weights w(x) and m requests R_0..R_{m-1}, each a set
+ * of chunks.  Choose, per request, an order of its chunks so that the trie of
+ * the resulting strings has the least total weight over its non-root nodes.
+ *
+ * Method (Thm 1 and Sec. 3.1): the optimum equals a minimum over binary
+ * hierarchies on the requests, computed exactly by the subset recurrence
+ *     F({i}) = w(R_i),
+ *     F(S)   = min over S = A (+) B of F(A) + F(B) - w(I(S)),
+ * where I(S) is the intersection of R_i over i in S.  OPT = F({0..m-1}).
+ * All work runs in CUDA kernels on the caller's stream; the host only
+ * validates arguments and orders launches.
+ *
+ * Conventions shared by every call:
+ *   - Request i is bit i of every subset mask (request 0 = least significant).
+ *   - Request bitsets: uint64 row-major [m][ceil(n/64)]; bit (x % 64) of word
+ *     (x / 64) in row i is set iff chunk x is in R_i.
+ *   - Chunk ids in every output are the caller's ids 0..n-1.
+ *   - Among optimal splits of S, the reported one is named by its part A that
+ *     holds the lowest request of S, and the smallest such A (as an unsigned
+ *     integer) is chosen; split[S] = A, 0 for singletons and for S = 0.
+ *   - Every call returns a status; on failure no output is written.
+ *   - A context is not thread-safe; distinct contexts are independent.
+ *   - Limits: 1 <= m <= 30, 1 <= n <= 2^31 - 1, every w(x) >= 1, and
+ *     sum_i w(R_i) < 2^62 (MPT_ERR_OVERFLOW otherwise).
+ */
+#ifndef MPT_H
+#define MPT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum mpt_status {
+  MPT_OK = 0,
+  MPT_ERR_INVALID_ARG = 1,         /* null pointer, m < 1, n < 1, w(x) <= 0, a bit set at x >= n */
+  MPT_ERR_TOO_LARGE = 2,           /* m > 30 */
+  MPT_ERR_OVERFLOW = 3,            /* sum_i w(R_i) >= 2^62 */
+  MPT_ERR_OUT_OF_MEMORY = 4,       /* host or device allocation failed */
+  MPT_ERR_WORKSPACE_TOO_SMALL = 5, /* caller workspace below mpt_workspace_bytes() */
+  MPT_ERR_CUDA = 6,                /* a CUDA call failed; mpt_last_error() has its text */
+  MPT_ERR_NOT_SOLVED = 7,          /* results asked for before a successful mpt_solve */
+  MPT_ERR_TIMEOUT = 8,             /* reserved: a bounded device-side wait gave up */
+  MPT_ERR_INTERNAL = 9             /* a device-side consistency check failed */
+} mpt_status;
+
+typedef struct mpt_ctx mpt_ctx;
+
+/* DP kernels mpt_solve may use.  AUTO picks BLOCKED whenever
+ * sum_i w(R_i) < 2^20 (its 32-bit packed keys are then exact), else GENERAL. */
+typedef enum mpt_dp_mode {
+  MPT_DP_AUTO = 0,
+  MPT_DP_BLOCKED = 1, /* shared-memory tiled min-plus; needs sum_i w(R_i) < 2^20 */
+  MPT_DP_GENERAL = 2  /* one subset per thread or warp, int64 gathers from HBM/L2 */
+} mpt_dp_mode;
+
+/* Create a context for one instance (Sec. 2).
+ *   weights:  host int64[n_chunks], w(x) >= 1 for every x.
+ *   req_bits: host uint64[m][ceil(n_chunks/64)], as above; no bit at x >= n.
+ * Both arrays are validated and copied; the caller keeps ownership.
+ * Errors: INVALID_ARG, TOO_LARGE, OVERFLOW, OUT_OF_MEMORY.  *out is written
+ * only on success.  No CUDA call is made. */
+mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* req_bits, int32_t m,
+                      mpt_ctx** out);
+
+/* Bytes of device workspace mpt_solve needs for this context: the input
+ * copies, the intersection-weight table wI int64[2^m], F int64[2^m],
+ * split uint32[2^m], the blocked DP's working tables and the layout buffers. */
+mpt_status mpt_workspace_bytes(const mpt_ctx* ctx, size_t* bytes);
+
+/* Choose the DP kernels (default MPT_DP_AUTO).  BLOCKED is refused with
+ * OVERFLOW when sum_i w(R_i) >= 2^20. */
+mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode);
+
+/* Solve exactly (Sec. 3.1): scatter chunk weights by request set, superset
+ * sums for w(I(S)) of every S, the popcount-layered min-plus recurrence with
+ * its argmin table, then the hierarchy walk for the layout (Thm 1 proof).
+ *   d_workspace: device memory of at least mpt_workspace_bytes(), 256-byte
+ *     aligned, owned by the caller.  Nothing else may write it while this
+ *     context uses it: the instance copied into it by one solve is reused
+ *     (not copied again) by the next solve of the same context with the same
+ *     workspace.  NULL makes the library allocate (and keep) its own.
+ *   stream: a cudaStream_t (NULL = the legacy default stream).  Every copy
+ *     and kernel is enqueued on it; the call synchronises it before return.
+ *   opt_cost: host int64, receives OPT = F({0..m-1}).
+ * Errors: INVALID_ARG, WORKSPACE_TOO_SMALL, OUT_OF_MEMORY, CUDA, INTERNAL. */
+mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream, int64_t* opt_cost);
+
+/* Device views (length 2^m, indexed by subset mask S) of the last solve:
+ *   F[S]     = the recurrence value (F[0] = 0),
+ *   wI[S]    = w(I(S)); wI[0] = weight of the union of all requests,
+ *   split[S] = the reported optimal split (see conventions).
+ * The pointers live in the workspace and stay valid until the next solve or
+ * mpt_destroy.  Any argument may be NULL.  Errors: INVALID_ARG, NOT_SOLVED. */
+mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split);
+
+/* Number of entries mpt_layout writes to perm_chunks: sum_i |R_i|. */
+mpt_status mpt_layout_size(const mpt_ctx* ctx, int64_t* total_chunks);
+
+/* Layout of the last solve (constructive direction of Thm 1): at hierarchy
+ * node B (root = all requests, children split[B] then B \ split[B]) the chunks
+ * of I(B) \ I(parent(B)) are emitted in increasing chunk id; request i's
+ * permutation is the concatenation along its root-to-leaf path.
+ *   perm_offsets: host int64[m+1]; request i is perm_chunks[off[i] .. off[i+1]).
+ *   perm_chunks:  host int64[mpt_layout_size()].
+ *   dfs_order:    host int32[m], the leaves from left to right -- the serving
+ *                 order of Thm 7 (Sec. 8).
+ * Any output may be NULL.  Errors: INVALID_ARG, NOT_SOLVED. */
+mpt_status mpt_layout(const mpt_ctx* ctx, int64_t* perm_offsets, int64_t* perm_chunks, int32_t* dfs_order);
+
+/* Trie cost of a layout (Sec. 2, eq. 1): the total weight of the non-root
+ * nodes of the trie of the m strings, computed by a CUDA kernel.  All
+ * pointers are host memory; perm_offsets has m+1 entries, perm_chunks
+ * perm_offsets[m] entries with ids in [0, n_chunks).  The call allocates a
+ * small device buffer and synchronises the legacy default stream.
+ * Errors: INVALID_ARG, OUT_OF_MEMORY, CUDA. */
+mpt_status mpt_trie_cost(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* perm_offsets,
+                         const int64_t* perm_chunks, int64_t* cost);
+
+/* Per-stage device timings of the last solve, taken with CUDA events on the
+ * solve's stream when profiling is on (mpt_set_profiling). */
+typedef struct mpt_profile {
+  double ms_h2d;        /* input copies */
+  double ms_scatter;    /* N_x and g(T) scatter */
+  double ms_zeta;       /* superset sums -> wI */
+  double ms_dp_pairs;   /* blocked DP: all launches of the pair kernel */
+  double ms_dp_tiles;   /* blocked DP: all launches of the in-tile kernel */
+  double ms_dp_general; /* general DP: all launches */
+  double ms_walk;       /* hierarchy walk -> layout */
+  double ms_d2h;        /* result copies */
+  double splits_pairs;  /* splits evaluated by the pair kernel */
+  double splits_total;  /* (3^m + 1)/2 - 2^m */
+  int64_t launches_pairs;
+  int64_t launches_total; /* kernels launched by the last solve (memsets excluded) */
+  int32_t dp_mode;        /* MPT_DP_BLOCKED or MPT_DP_GENERAL as used */
+  int32_t tile_bits;      /* request bits per shared-memory tile (blocked mode) */
+} mpt_profile;
+
+mpt_status mpt_set_profiling(mpt_ctx* ctx, int32_t on);
+mpt_status mpt_get_profile(const mpt_ctx* ctx, mpt_profile* out);
+
+/* Free the context and any workspace the library allocated.  NULL is a no-op. */
+void mpt_destroy(mpt_ctx* ctx);
+
+/* Static text for a status code. */
+const char* mpt_status_string(mpt_status status);
+
+/* Text of the last CUDA or internal error seen by this context ("" if none). */
+const char* mpt_last_error(const mpt_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MPT_H */

@@ -1,0 +1,425 @@
+// K3 (blocked form): the Sec. 3.1 recurrence
+//     F({i}) = w(R_i),   F(S) = min over S = A (+) B of F(A) + F(B) - w(I(S)),
+// evaluated with shared-memory tiles so that each 4-byte table entry fetched
+// from HBM/L2 serves hundreds of splits.
+//
+// Index layout.  Requests are split into a "tile" part T (requests 0..L-1)
+// and an "inner" part U (requests L..m-1, b = m - L <= 12 of them).  The
+// working tables are stored in rotated order idx(S) = (T << b) | U, so the
+// 2^b subsets sharing one T are contiguous (one 16 KB window per T).
+//
+// Split structure.  A split of S = (T, U) is named by its part A = (Ta, Ua)
+// that holds the lowest request of S.  For T != 0 that request is in T, so
+//   * proper pairs: Ta runs over the subsets of T that hold lowbit(T), Ta != T,
+//     and Ua over ALL subsets of U;  B = (T \ Ta, U \ Ua).  For a fixed Ta this
+//     is a full min-plus subset convolution over the b inner bits of the two
+//     windows F[Ta, .] and F[T \ Ta, .] -- the pair kernel below;
+//   * self pair: Ta = T, Ua a proper subset of U, B = (0, U \ Ua): needs the
+//     tile's own smaller entries, so it runs inside the tile, level by level
+//     in |U| -- the tile kernel below, which also finishes every entry.
+// For T = 0 the tile kernel runs the recurrence on the b inner bits alone.
+// Tiles with |T| = k depend only on tiles with |T| < k: one launch pair per k.
+//
+// Packed keys.  With sum_i w(R_i) < 2^(32-b) every candidate F(A) + F(B) fits
+// in 32 - b bits, so the working tables hold G = F << b and the key of a
+// candidate is
+//     key = Gp[A] + Gc[B] = ((F(A) + F(B)) << b) | (2^b - 1 - U + Ua),
+// Gp = F << b and Gc = (F << b) | (~u & (2^b - 1)) (u = the entry's U part).
+// An unsigned min over keys picks the least value and, among equal values,
+// the least Ua; across proper pairs, taken in increasing Ta with strict
+// improvement, the least Ta; then the self pair (largest Ta = T).  That is the
+// lexicographic order on (value, A) as an integer, since A = Ua * 2^L + Ta.
+#include "mpt_internal.cuh"
+
+namespace mpt {
+namespace {
+
+constexpr int kB = 12;                     // inner bits of the pair kernel
+constexpr int kB2 = 5;                     // inner bits held in registers
+constexpr int kB1 = kB - kB2;              // inner bits that index window rows
+constexpr int kRow = 1 << kB2;             // 32 entries per row
+constexpr int kRowStride = kRow + 4;       // 36 words: consecutive rows start in different 16-byte bank groups
+constexpr int kRows = 1 << kB1;            // 128 rows per window
+constexpr int kWin = kRows * kRowStride;   // words per padded window
+constexpr int kPairThreads = 320;
+constexpr int kPairSmemBytes = 2 * 2 * kWin * (int)sizeof(uint32_t);  // double-buffered X and Y windows
+constexpr int kMinPairsPerItem = 16;
+constexpr int kTileThreads = 512;
+constexpr int kMaxTileBits = 12;
+
+static_assert(kPairSmemBytes >= (1 << kB) * 8, "merge buffer must fit in the window buffers");
+
+// ---------------------------------------------------------------------------
+// Per-thread work of the pair kernel.  The b inner bits are (s1, s2): s1 = the
+// top kB1 bits (window row), s2 = the low kB2 bits (register lane).  Output
+// (s1, s2) collects, for every Ua = (a1, a2) with a1 in s1 and a2 in s2,
+// X[a1][a2] + Y[s1^a1][s2^a2].  A "unit" is one (s1, a1): two rows, 243 adds.
+// A thread owns one s1 (its 32 outputs) and a fixed subset of the a1 in s1:
+// rows with >= 3 bits are split on their lowest set bits into tasks of 8 a1
+// each; rows with < 3 bits are one task.  Packed as s1 | fixed << 8 | free << 16.
+// ---------------------------------------------------------------------------
+struct TaskTable {
+  uint32_t t[kPairThreads];
+  int count;
+};
+
+constexpr int popc_c(uint32_t v) {
+  int c = 0;
+  while (v) {
+    v &= v - 1;
+    ++c;
+  }
+  return c;
+}
+
+constexpr uint32_t deposit_c(uint32_t q, uint32_t mask) {
+  uint32_t out = 0;
+  while (mask) {
+    const uint32_t low = mask & (~mask + 1u);
+    if (q & 1u) out |= low;
+    q >>= 1;
+    mask ^= low;
+  }
+  return out;
+}
+
+constexpr TaskTable make_tasks() {
+  TaskTable tt{};
+  int n = 0;
+  for (uint32_t s1 = 0; s1 < (uint32_t)kRows; ++s1) {
+    const int p = popc_c(s1);
+    if (p < 3) continue;
+    const int q = p - 3;
+    uint32_t lowbits = 0, r = s1;
+    for (int t = 0; t < q; ++t) {
+      const uint32_t lb = r & (~r + 1u);
+      lowbits |= lb;
+      r ^= lb;
+    }
+    const uint32_t freem = s1 ^ lowbits;
+    for (uint32_t v = 0; v < (1u << q); ++v) tt.t[n++] = s1 | (deposit_c(v, lowbits) << 8) | (freem << 16);
+  }
+  for (int p = 2; p >= 0; --p)
+    for (uint32_t s1 = 0; s1 < (uint32_t)kRows; ++s1)
+      if (popc_c(s1) == p) tt.t[n++] = s1 | (s1 << 16);
+  tt.count = n;
+  for (int i = n; i < kPairThreads; ++i) tt.t[i] = 0xFFFFFFFFu;
+  return tt;
+}
+
+constexpr TaskTable kTasksHost = make_tasks();
+static_assert(kTasksHost.count <= kPairThreads, "task table exceeds the block");
+static __constant__ TaskTable c_tasks = make_tasks();
+
+// Row placement inside a padded window: the low 3 row bits are XOR-ed with
+// higher row bits so that rows that differ only above bit 2 still start in
+// different bank groups.
+__device__ __forceinline__ int row_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// Issue the copies of the two windows of one pair into a buffer.
+__device__ __forceinline__ void stage_pair(uint32_t* X, uint32_t* Y, const uint32_t* __restrict__ gx,
+                                           const uint32_t* __restrict__ gy) {
+  for (int c = threadIdx.x; c < 2 * (kRows * kRow / 4); c += kPairThreads) {
+    const int w = c >> (kB - 2);          // 0: X window, 1: Y window
+    const int cc = c & ((1 << (kB - 2)) - 1);
+    const int row = cc >> (kB2 - 2);
+    const int k = cc & ((1 << (kB2 - 2)) - 1);
+    uint32_t* dst = (w ? Y : X) + row_pos((uint32_t)row) * kRowStride + k * 4;
+    const uint32_t* src = (w ? gy : gx) + cc * 4;
+    cp_async16(dst, src);
+  }
+}
+
+__device__ __forceinline__ void load_row(uint32_t (&v)[kRow], const uint32_t* p) {
+  const uint4* q = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+  for (int c = 0; c < kRow / 4; ++c) {
+    const uint4 t = q[c];
+    v[4 * c] = t.x;
+    v[4 * c + 1] = t.y;
+    v[4 * c + 2] = t.z;
+    v[4 * c + 3] = t.w;
+  }
+}
+
+// acc[s2] = min over a2 in s2 of x[a2] + y[s2 ^ a2]  (243 add/min pairs).
+__device__ __forceinline__ void conv_rows(uint32_t (&acc)[kRow], const uint32_t (&x)[kRow], const uint32_t (&y)[kRow]) {
+#pragma unroll
+  for (int s2 = 0; s2 < kRow; ++s2) {
+#pragma unroll
+    for (int a2 = 0; a2 < kRow; ++a2) {
+      if ((a2 & s2) == a2) acc[s2] = min(acc[s2], x[a2] + y[s2 ^ a2]);
+    }
+  }
+}
+
+// Pair kernel for tiles with |T| = kh >= 2.  Block = (tile, range of pairs).
+// Writes, per inner subset U of the tile, the lexicographic minimum of
+// (key, Ta) over its pairs into partial[tile << kB | U] with atomicMin.
+__global__ void __launch_bounds__(kPairThreads, 1)
+k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, unsigned long long* __restrict__ partial,
+           int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item) {
+  extern __shared__ __align__(16) uint32_t smem[];
+  // buffer c holds X at smem + 2c * kWin and Y right after it
+
+  const uint32_t tile = blockIdx.x / items_per_tile;
+  const uint32_t item = blockIdx.x % items_per_tile;
+  const uint32_t T = colex_unrank(tile, kh, L);
+  const uint32_t low = T & (~T + 1u);
+  const uint32_t R = T ^ low;
+  const uint32_t q0 = item * pairs_per_item;
+  const uint32_t q1 = min(q0 + pairs_per_item, pairs_per_tile);
+
+  const uint32_t task = c_tasks.t[threadIdx.x];
+  const bool valid = task != 0xFFFFFFFFu;
+  const uint32_t s1 = task & 0xFFu;
+  const uint32_t fixed = (task >> 8) & 0xFFu;
+  const uint32_t freem = (task >> 16) & 0xFFu;
+
+  uint32_t bk[kRow], bt[kRow];
+#pragma unroll
+  for (int i = 0; i < kRow; ++i) {
+    bk[i] = 0xFFFFFFFFu;
+    bt[i] = 0;
+  }
+
+  uint32_t sub = deposit_bits(q0, R);
+  {
+    const uint32_t Ta = low | sub;
+    stage_pair(smem, smem + kWin, Gp + ((size_t)Ta << kB), Gc + ((size_t)(T ^ Ta) << kB));
+    cp_async_commit();
+  }
+  for (uint32_t q = q0; q < q1; ++q) {
+    const int cur = (int)((q - q0) & 1u);
+    const uint32_t Ta = low | sub;
+    const uint32_t next = (sub - R) & R;
+    if (q + 1 < q1) {
+      const uint32_t Tn = low | next;
+      uint32_t* nb = smem + 2 * (cur ^ 1) * kWin;
+      stage_pair(nb, nb + kWin, Gp + ((size_t)Tn << kB), Gc + ((size_t)(T ^ Tn) << kB));
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    if (valid) {
+      const uint32_t* X = smem + 2 * cur * kWin;
+      const uint32_t* Y = X + kWin;
+      uint32_t acc[kRow];
+#pragma unroll
+      for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
+      uint32_t s = 0;
+      do {
+        const uint32_t a1 = fixed | s;
+        uint32_t x[kRow], y[kRow];
+        load_row(x, X + row_pos(a1) * kRowStride);
+        load_row(y, Y + row_pos(s1 ^ a1) * kRowStride);
+        conv_rows(acc, x, y);
+        s = (s - freem) & freem;
+      } while (s != 0);
+#pragma unroll
+      for (int i = 0; i < kRow; ++i) {
+        const bool better = acc[i] < bk[i];
+        bk[i] = better ? acc[i] : bk[i];
+        bt[i] = better ? Ta : bt[i];
+      }
+    }
+    __syncthreads();
+    sub = next;
+  }
+
+  // Merge the threads that share an s1, then the blocks that share the tile.
+  unsigned long long* merged = reinterpret_cast<unsigned long long*>(smem);
+  for (int i = threadIdx.x; i < (1 << kB); i += kPairThreads) merged[i] = ~0ull;
+  __syncthreads();
+  if (valid) {
+#pragma unroll
+    for (int i = 0; i < kRow; ++i)
+      atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | bt[i]);
+  }
+  __syncthreads();
+  unsigned long long* out = partial + ((size_t)tile << kB);
+  for (int i = threadIdx.x; i < (1 << kB); i += kPairThreads) atomicMin(&out[i], merged[i]);
+}
+
+// Tile kernel: finishes every entry of the tiles with |T| = kh, level by level
+// in |U|, folding in the self pair (kh >= 1) or running the whole recurrence
+// on the inner bits (kh = 0).  One block per tile.
+__global__ void __launch_bounds__(kTileThreads)
+k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned long long* __restrict__ partial,
+          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, int64_t* __restrict__ F, uint32_t* __restrict__ split) {
+  __shared__ uint32_t cur_p[1 << kMaxTileBits];   // this tile, F << b
+  __shared__ uint32_t other_c[1 << kMaxTileBits]; // complement form: this tile (kh = 0) or tile 0 (kh >= 1)
+  __shared__ uint16_t order[1 << kMaxTileBits];   // inner subsets sorted by size, then colex
+
+  const uint32_t tile = blockIdx.x;
+  const uint32_t T = kh == 0 ? 0u : colex_unrank(tile, kh, L);
+  const int size = 1 << b;
+  const uint32_t mask = (uint32_t)size - 1u;
+
+  for (int u = threadIdx.x; u < size; u += kTileThreads) {
+    const int p = __popc(u);
+    uint32_t start = 0;
+    for (int j = 0; j < p; ++j) start += (uint32_t)c_binom.v[b][j];
+    order[start + colex_rank((uint32_t)u)] = (uint16_t)u;
+    if (kh >= 1) other_c[u] = Gc[u];
+  }
+  __syncthreads();
+
+  uint32_t start = 0;
+  for (int p = 0; p <= b; ++p) {
+    const int cnt = (int)c_binom.v[b][p];
+    const int g = p > 3 ? min(p - 3, 5) : 0;  // log2(lanes per output)
+    const int G = 1 << g;
+    const int groups = kTileThreads >> g;
+    for (int base = 0; base < cnt; base += groups) {
+      const int gi = base + (int)(threadIdx.x >> g);
+      const uint32_t r = threadIdx.x & (uint32_t)(G - 1);
+      const bool active = gi < cnt;
+      unsigned long long best = ~0ull;
+      uint32_t U = 0;
+      bool single = false;
+      if (active) {
+        U = order[start + gi];
+        const uint32_t nreq = (uint32_t)p + (uint32_t)kh;
+        single = nreq == 1;
+        if (nreq >= 2 && !(kh >= 1 && U == 0)) {
+          // kh = 0: Ua = lowbit(U) | part, part a proper subset of U \ lowbit(U).
+          // kh >= 1: Ua = part, a proper subset of U (Ta = T).
+          const uint32_t lowU = kh == 0 ? (U & (~U + 1u)) : 0u;
+          const uint32_t emask = U ^ lowU;
+          uint32_t hi = 0, rr = emask;
+          for (int t = 0; t < g; ++t) {
+            const uint32_t top = 1u << (31 - __clz(rr));
+            hi |= top;
+            rr ^= top;
+          }
+          const uint32_t freem = emask ^ hi;
+          const uint32_t fixed = deposit_bits(r, hi);
+          const unsigned long long ta = kh == 0 ? 0ull : (unsigned long long)T;
+          uint32_t s = 0;
+          do {
+            const uint32_t part = fixed | s;
+            if (part != emask) {
+              const uint32_t Ua = lowU | part;
+              const uint32_t key = cur_p[Ua] + other_c[U ^ Ua];
+              const unsigned long long c = ((unsigned long long)key << 32) | ta;
+              best = c < best ? c : best;
+            }
+            s = (s - freem) & freem;
+          } while (s != 0);
+        }
+        if (kh >= 2 && r == 0) {
+          const unsigned long long pv = partial[((size_t)tile << b) | U];
+          best = pv < best ? pv : best;
+        }
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
+        best = o < best ? o : best;
+      }
+      if (active && r == 0) {
+        const size_t S = ((size_t)U << L) | T;
+        int64_t f;
+        uint32_t A;
+        if (S == 0) {
+          f = 0;
+          A = 0;
+        } else if (single) {
+          f = wI[S];
+          A = 0;
+        } else {
+          const uint32_t key = (uint32_t)(best >> 32);
+          const uint32_t Ua = (key & mask) + U - mask;
+          f = (int64_t)(key >> b) - wI[S];
+          A = (Ua << L) | (uint32_t)best;
+        }
+        const uint32_t gp = (uint32_t)f << b;
+        const uint32_t gc = gp | (~U & mask);
+        cur_p[U] = gp;
+        if (kh == 0) other_c[U] = gc;
+        const size_t idx = ((size_t)T << b) | U;
+        Gp[idx] = gp;
+        Gc[idx] = gc;
+        F[S] = f;
+        split[S] = A;
+      }
+    }
+    start += (uint32_t)cnt;
+    __syncthreads();
+  }
+}
+
+}  // namespace
+
+int blocked_tile_bits(int m) { return m < kB ? m : kB; }
+
+int64_t blocked_partial_entries(int m, int b) {
+  const int L = m - b;
+  unsigned long long most = 0;
+  for (int k = 2; k <= L; ++k)
+    if (h_binom.v[L][k] > most) most = h_binom.v[L][k];
+  return (int64_t)(most << b);
+}
+
+int blocked_max_launches(const Shape& s) { return 2 * (s.L + 1); }
+
+cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                              BlockedTiming* timing) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  const int b = s.b, L = s.L;
+  constexpr unsigned long long evals_per_pair = 531441ull;  // 3^12 splits per pair of windows
+  for (int kh = 0; kh <= L; ++kh) {
+    const unsigned long long tiles = h_binom.v[L][kh];
+    if (kh >= 2) {
+      const uint32_t P = (1u << (kh - 1)) - 1u;
+      const unsigned long long target = 152ull * 8;
+      unsigned long long items = (target + tiles - 1) / tiles;
+      const unsigned long long cap = (P + kMinPairsPerItem - 1) / kMinPairsPerItem;
+      if (items > cap) items = cap;
+      if (items < 1) items = 1;
+      const uint32_t ppi = (uint32_t)((P + items - 1) / items);
+      items = (P + ppi - 1) / ppi;
+      cudaError_t e = cudaMemsetAsync(ws.partial, 0xFF, (size_t)(tiles << b) * sizeof(unsigned long long), stream);
+      if (e != cudaSuccess) return e;
+      if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches], stream);
+      k_dp_pairs<<<(unsigned)(tiles * items), kPairThreads, kPairSmemBytes, stream>>>(
+          ws.Gp, ws.Gc, ws.partial, L, kh, P, (uint32_t)items, ppi);
+      if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches + 1], stream);
+      if (timing) {
+        timing->pair_launches++;
+        timing->pair_splits += (double)tiles * (double)P * (double)evals_per_pair;
+      }
+      ++*launches;
+      e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+    }
+    if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches], stream);
+    k_dp_tile<<<(unsigned)tiles, kTileThreads, 0, stream>>>(L, b, kh, ws.wI, kh >= 2 ? ws.partial : nullptr, ws.Gp,
+                                                            ws.Gc, ws.F, ws.split);
+    if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
+    if (timing) timing->tile_launches++;
+    ++*launches;
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace mpt

@@ -1,0 +1,130 @@
+// K1: request-set scatter and K2: superset sums, giving w(I(S)) for every S.
+//
+// Sec. 3 defines S_x = {i : x in R_i}; here it is the m-bit mask N_x.  A chunk
+// x lies in I(S) = intersection of R_i over i in S exactly when S is a subset
+// of N_x, so
+//     w(I(S)) = sum over T superset of S of g(T),   g(T) = sum of w(x) with N_x = T,
+// which is the quantity w(I(B)) of the Sec. 3.1 recurrence.  K1 builds g and
+// the list of chunks that some request uses; K2 is the superset-sum (zeta)
+// transform over the 2^m table, done in shared-memory tiles so that each
+// pass streams the table once with coalesced 128-byte rows.
+#include "mpt_internal.cuh"
+
+namespace mpt {
+namespace {
+
+constexpr int kScatterThreads = 256;
+
+__global__ void __launch_bounds__(kScatterThreads)
+k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m, int64_t words,
+          unsigned long long* __restrict__ g, uint32_t* __restrict__ used_N, int32_t* __restrict__ used_x,
+          int32_t* __restrict__ counters, int64_t slots) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
+    const int64_t word = x >> 6;
+    const int sh = (int)(x & 63);
+    uint32_t N = 0;
+    for (int i = 0; i < m; ++i) N |= (uint32_t)((__ldg(&bits[(int64_t)i * words + word]) >> sh) & 1ull) << i;
+    if (N) {
+      atomicAdd(&g[N], (unsigned long long)w[x]);
+      const int k = atomicAdd(&counters[0], 1);
+      if (k < slots) {
+        used_N[k] = N;
+        used_x[k] = (int32_t)x;
+      } else {
+        atomicOr(&counters[1], kErrWorkspace);
+      }
+    }
+  }
+}
+
+// Superset sums over the low `tb` index bits of each tile of 2^tb entries.
+constexpr int kZetaLowBits = 12;
+constexpr int kZetaThreads = 512;
+
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_low(unsigned long long* __restrict__ g, int tb) {
+  __shared__ unsigned long long t[1 << kZetaLowBits];
+  const int size = 1 << tb;
+  unsigned long long* tile = g + ((size_t)blockIdx.x << tb);
+  for (int i = threadIdx.x; i < size; i += blockDim.x) t[i] = tile[i];
+  const int half = size >> 1;
+  for (int j = 0; j < tb; ++j) {
+    __syncthreads();
+    const int lowmask = (1 << j) - 1;
+    for (int p = threadIdx.x; p < half; p += blockDim.x) {
+      const int i = ((p >> j) << (j + 1)) | (p & lowmask);  // bit j of i is 0
+      t[i] += t[i | (1 << j)];
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < size; i += blockDim.x) tile[i] = t[i];
+}
+
+// Superset sums over index bits [lo, lo + tb): each block owns 16 adjacent
+// columns (bits below lo) and all 2^tb values of those bits, for one value of
+// the bits above; rows of 16 entries are contiguous 128-byte segments.
+constexpr int kZetaCols = 16;
+constexpr int kZetaHighBits = 8;
+
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_high(unsigned long long* __restrict__ g, int lo, int tb) {
+  __shared__ unsigned long long t[(1 << kZetaHighBits) * kZetaCols];
+  const size_t col_groups = ((size_t)1 << lo) / kZetaCols;
+  const size_t cg = blockIdx.x % col_groups;
+  const size_t top = blockIdx.x / col_groups;
+  unsigned long long* base = g + (top << (lo + tb)) + cg * kZetaCols;
+  const int rows = 1 << tb;
+  const int elems = rows * kZetaCols;
+  for (int e = threadIdx.x; e < elems; e += blockDim.x) {
+    const int r = e / kZetaCols, c = e % kZetaCols;
+    t[e] = base[((size_t)r << lo) + c];
+  }
+  const int half = elems >> 1;
+  for (int j = 0; j < tb; ++j) {
+    __syncthreads();
+    const int lowmask = (1 << j) - 1;
+    for (int p = threadIdx.x; p < half; p += blockDim.x) {
+      const int c = p % kZetaCols, q = p / kZetaCols;
+      const int r = ((q >> j) << (j + 1)) | (q & lowmask);  // bit j of r is 0
+      t[r * kZetaCols + c] += t[(r | (1 << j)) * kZetaCols + c];
+    }
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < elems; e += blockDim.x) {
+    const int r = e / kZetaCols, c = e % kZetaCols;
+    base[((size_t)r << lo) + c] = t[e];
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
+  int64_t blocks = (s.n + kScatterThreads - 1) / kScatterThreads;
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  if (blocks < 1) blocks = 1;
+  k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
+      ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned long long*>(ws.wI), ws.used_N, ws.used_x,
+      ws.counters, s.slots);
+  ++*launches;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
+  unsigned long long* g = reinterpret_cast<unsigned long long*>(ws.wI);
+  const int tb = s.m < kZetaLowBits ? s.m : kZetaLowBits;
+  const size_t low_blocks = (size_t)1 << (s.m - tb);
+  k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb);
+  ++*launches;
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  for (int lo = tb; lo < s.m; lo += kZetaHighBits) {
+    const int hb = (s.m - lo) < kZetaHighBits ? (s.m - lo) : kZetaHighBits;
+    const size_t blocks = ((size_t)1 << s.m) / (((size_t)1 << hb) * kZetaCols);
+    k_zeta_high<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, hb);
+    ++*launches;
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace mpt

@@ -1,0 +1,145 @@
+// Internal declarations shared by the CUDA translation units of libmpt.
+// Nothing here is part of the public ABI (include/mpt.h).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace mpt {
+
+// ---------------------------------------------------------------------------
+// Binomial coefficients C(n, k), n, k <= 32, for ranking k-subsets in colex
+// order (the combinatorial number system): the subset {c_1 < .. < c_k} has
+// rank sum_t C(c_t, t).  Every translation unit gets its own constant copy.
+// ---------------------------------------------------------------------------
+struct BinomTable {
+  unsigned long long v[33][33];
+};
+
+constexpr BinomTable make_binom() {
+  BinomTable t{};
+  for (int n = 0; n <= 32; ++n)
+    for (int k = 0; k <= 32; ++k)
+      t.v[n][k] = (k == 0) ? 1ull : (n == 0 ? 0ull : t.v[n - 1][k - 1] + t.v[n - 1][k]);
+  return t;
+}
+
+static __constant__ BinomTable c_binom = make_binom();
+static constexpr BinomTable h_binom = make_binom();
+
+// The idx-th k-subset of {0..n-1} in colex order.
+__device__ __forceinline__ uint32_t colex_unrank(unsigned long long idx, int k, int n) {
+  uint32_t S = 0;
+  for (int pos = n - 1; pos >= 0 && k > 0; --pos) {
+    unsigned long long c = c_binom.v[pos][k];
+    if (idx >= c) {
+      S |= 1u << pos;
+      idx -= c;
+      --k;
+    }
+  }
+  return S;
+}
+
+// Rank of S among the subsets of its size, in colex order.
+__device__ __forceinline__ uint32_t colex_rank(uint32_t S) {
+  uint32_t r = 0;
+  int t = 1;
+  while (S) {
+    int pos = __ffs(S) - 1;
+    r += (uint32_t)c_binom.v[pos][t];
+    ++t;
+    S &= S - 1;
+  }
+  return r;
+}
+
+// Scatter the low bits of q into the set positions of mask (ascending).
+__device__ __forceinline__ uint32_t deposit_bits(uint32_t q, uint32_t mask) {
+  uint32_t out = 0;
+  while (mask && q) {
+    uint32_t low = mask & (~mask + 1u);
+    if (q & 1u) out |= low;
+    q >>= 1;
+    mask ^= low;
+  }
+  return out;
+}
+
+// ---------------------------------------------------------------------------
+// Device-side error flags (bitwise OR into one int in the workspace).
+// ---------------------------------------------------------------------------
+enum DeviceError : int {
+  kErrBadSplit = 1,      // a split entry on the hierarchy is not a proper non-empty subset
+  kErrLayoutCount = 2,   // the layout walk did not place every chunk occurrence
+  kErrWorkspace = 4,     // a kernel saw a size outside what the workspace was carved for
+};
+
+// ---------------------------------------------------------------------------
+// Workspace carve-up (all offsets 256-byte aligned).
+// ---------------------------------------------------------------------------
+struct Workspace {
+  // inputs
+  int64_t* weights;   // [n]
+  uint64_t* bits;     // [m * words]
+  // scatter outputs
+  uint32_t* used_N;   // [slots]  request set N_x of each used chunk
+  int32_t* used_x;    // [slots]  chunk id
+  int32_t* counters;  // [8]      0: number of used chunks, 1: device error flags
+  // tables, natural subset order
+  int64_t* wI;        // [2^m]
+  int64_t* F;         // [2^m]
+  uint32_t* split;    // [2^m]
+  // blocked DP working tables, rotated order (see k_dp_blocked.cu)
+  uint32_t* Gp;       // [2^m]  F << b
+  uint32_t* Gc;       // [2^m]  (F << b) | (~u & (2^b - 1))
+  unsigned long long* partial;  // [max tiles of one layer << b]
+  // layout
+  unsigned long long* keys;  // [slots]
+  int64_t* perm_offsets;     // [m + 1]
+  int64_t* perm_chunks;      // [slots]
+  int32_t* dfs;              // [m]
+  int64_t* opt;              // [1]
+};
+
+struct Shape {
+  int m;
+  int64_t n;
+  int64_t words;
+  int64_t slots;    // sum_i |R_i|
+  bool blocked;     // blocked DP tables present
+  int b;            // tile bits (blocked)
+  int L;            // m - b
+  int64_t partial_entries;
+};
+
+size_t carve_workspace(const Shape& s, char* base, Workspace* ws);
+
+// ---------------------------------------------------------------------------
+// Launchers.  All enqueue on `stream` and return the launch error (if any).
+// ---------------------------------------------------------------------------
+cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+
+cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+
+struct BlockedTiming {
+  cudaEvent_t* pair_ev;  // 2 per pair-kernel launch (start, stop), or nullptr
+  cudaEvent_t* tile_ev;  // 2 per tile-kernel launch, or nullptr
+  int pair_launches;
+  int tile_launches;
+  double pair_splits;
+};
+int blocked_max_launches(const Shape& s);  // upper bound on pair + tile launches
+cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                              BlockedTiming* timing);
+int64_t blocked_partial_entries(int m, int b);
+int blocked_tile_bits(int m);
+
+cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+cudaError_t launch_trie_cost(int m, const int64_t* d_weights, const int64_t* d_offsets, const int64_t* d_chunks,
+                             int64_t* d_cost, cudaStream_t stream);
+
+}  // namespace mpt

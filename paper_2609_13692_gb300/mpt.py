@@ -1,0 +1,287 @@
+"""Thin Python binding of ``include/mpt.h`` (the exact MPT solver on GB300).
+
+Argument marshalling only: every step of a solve runs in the CUDA kernels of
+``libmpt.so``.  PyTorch supplies device memory (the workspace) and the
+current stream.  The functions carry the C names; :func:`solve` strings them
+together for the common case.
+
+The library must have been built (``paper_2609_13692_gb300.build.build()``);
+there is no fallback: loading fails loudly if it is missing.
+"""
+
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+from typing import Optional
+
+import numpy as np
+
+from . import build as _build
+
+MPT_OK = 0
+MPT_DP_AUTO, MPT_DP_BLOCKED, MPT_DP_GENERAL = 0, 1, 2
+_MODES = {"auto": MPT_DP_AUTO, "blocked": MPT_DP_BLOCKED, "general": MPT_DP_GENERAL}
+
+STATUS_NAMES = {
+    0: "MPT_OK",
+    1: "MPT_ERR_INVALID_ARG",
+    2: "MPT_ERR_TOO_LARGE",
+    3: "MPT_ERR_OVERFLOW",
+    4: "MPT_ERR_OUT_OF_MEMORY",
+    5: "MPT_ERR_WORKSPACE_TOO_SMALL",
+    6: "MPT_ERR_CUDA",
+    7: "MPT_ERR_NOT_SOLVED",
+    8: "MPT_ERR_TIMEOUT",
+    9: "MPT_ERR_INTERNAL",
+}
+
+EXPORTED = [
+    "mpt_create", "mpt_workspace_bytes", "mpt_set_dp_mode", "mpt_solve", "mpt_tables", "mpt_layout_size",
+    "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
+    "mpt_last_error",
+]
+
+
+class MPTError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str = ""):
+        self.status = status
+        name = STATUS_NAMES.get(status, str(status))
+        super().__init__(f"{where}: {name}" + (f" ({detail})" if detail else ""))
+
+
+class mpt_profile(ctypes.Structure):
+    _fields_ = [
+        ("ms_h2d", ctypes.c_double),
+        ("ms_scatter", ctypes.c_double),
+        ("ms_zeta", ctypes.c_double),
+        ("ms_dp_pairs", ctypes.c_double),
+        ("ms_dp_tiles", ctypes.c_double),
+        ("ms_dp_general", ctypes.c_double),
+        ("ms_walk", ctypes.c_double),
+        ("ms_d2h", ctypes.c_double),
+        ("splits_pairs", ctypes.c_double),
+        ("splits_total", ctypes.c_double),
+        ("launches_pairs", ctypes.c_int64),
+        ("launches_total", ctypes.c_int64),
+        ("dp_mode", ctypes.c_int32),
+        ("tile_bits", ctypes.c_int32),
+    ]
+
+    def as_dict(self) -> dict:
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
+_LIB = None
+
+
+def library_path() -> str:
+    return str(_build.LIB)
+
+
+def load() -> ctypes.CDLL:
+    """Load libmpt.so (built in-tree); raises if it has not been built."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = _build.LIB
+    if not path.exists():
+        raise RuntimeError(f"{path} is missing: build the CUDA library first "
+                           "(python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(str(path))
+    vp, i64, i32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_size_t
+    i64p = ctypes.POINTER(ctypes.c_int64)
+    u64p = ctypes.POINTER(ctypes.c_uint64)
+    i32p = ctypes.POINTER(ctypes.c_int32)
+    sig = {
+        "mpt_create": ([i64p, i64, u64p, i32, ctypes.POINTER(vp)], ctypes.c_int),
+        "mpt_workspace_bytes": ([vp, ctypes.POINTER(sz)], ctypes.c_int),
+        "mpt_set_dp_mode": ([vp, i32], ctypes.c_int),
+        "mpt_solve": ([vp, vp, sz, vp, i64p], ctypes.c_int),
+        "mpt_tables": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp)], ctypes.c_int),
+        "mpt_layout_size": ([vp, i64p], ctypes.c_int),
+        "mpt_layout": ([vp, i64p, i64p, i32p], ctypes.c_int),
+        "mpt_trie_cost": ([i64p, i64, i32, i64p, i64p, i64p], ctypes.c_int),
+        "mpt_set_profiling": ([vp, i32], ctypes.c_int),
+        "mpt_get_profile": ([vp, ctypes.POINTER(mpt_profile)], ctypes.c_int),
+        "mpt_destroy": ([vp], None),
+        "mpt_status_string": ([ctypes.c_int], ctypes.c_char_p),
+        "mpt_last_error": ([vp], ctypes.c_char_p),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _LIB = lib
+    return lib
+
+
+def _ptr(a: np.ndarray, ct):
+    return a.ctypes.data_as(ctypes.POINTER(ct))
+
+
+def _check(status: int, where: str, ctx=None):
+    if status != MPT_OK:
+        detail = ""
+        if ctx is not None and ctx.handle:
+            detail = load().mpt_last_error(ctx.handle).decode()
+        raise MPTError(status, where, detail)
+
+
+class Context:
+    """Owns one ``mpt_ctx`` (one instance) and, optionally, a torch workspace."""
+
+    def __init__(self, handle: int, m: int, n: int):
+        self.handle = ctypes.c_void_p(handle)
+        self.m = m
+        self.n = n
+        self.workspace = None  # torch uint8 tensor, when the binding allocated it
+
+    def __del__(self):
+        try:
+            mpt_destroy(self)
+        except Exception:
+            pass
+
+
+def mpt_create(weights, bits) -> Context:
+    """Validate and copy an instance (host arrays); see ``mpt_create`` in mpt.h."""
+    lib = load()
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    b = np.ascontiguousarray(bits, dtype=np.uint64)
+    if b.ndim != 2:
+        raise ValueError("bits must be uint64[m, ceil(n/64)]")
+    m, n = int(b.shape[0]), int(w.shape[0])
+    if b.shape[1] != (n + 63) // 64:
+        raise ValueError("bits must have ceil(n/64) words per request")
+    h = ctypes.c_void_p()
+    _check(lib.mpt_create(_ptr(w, ctypes.c_int64), n, _ptr(b, ctypes.c_uint64), m, ctypes.byref(h)), "mpt_create")
+    return Context(h.value, m, n)
+
+
+def mpt_workspace_bytes(ctx: Context) -> int:
+    out = ctypes.c_size_t()
+    _check(load().mpt_workspace_bytes(ctx.handle, ctypes.byref(out)), "mpt_workspace_bytes", ctx)
+    return int(out.value)
+
+
+def mpt_set_dp_mode(ctx: Context, mode: str | int) -> None:
+    code = _MODES[mode] if isinstance(mode, str) else int(mode)
+    _check(load().mpt_set_dp_mode(ctx.handle, code), "mpt_set_dp_mode", ctx)
+
+
+def mpt_set_profiling(ctx: Context, on: bool) -> None:
+    _check(load().mpt_set_profiling(ctx.handle, 1 if on else 0), "mpt_set_profiling", ctx)
+
+
+def mpt_get_profile(ctx: Context) -> dict:
+    p = mpt_profile()
+    _check(load().mpt_get_profile(ctx.handle, ctypes.byref(p)), "mpt_get_profile", ctx)
+    return p.as_dict()
+
+
+def _default_stream_ptr() -> int:
+    import torch
+
+    return int(torch.cuda.current_stream().cuda_stream)
+
+
+def mpt_solve(ctx: Context, workspace=None, stream: Optional[int] = None) -> int:
+    """Run the solve on ``stream`` (default: torch's current stream) using
+    ``workspace`` (a CUDA uint8 tensor of at least mpt_workspace_bytes bytes;
+    default: one the binding allocates with torch and keeps on the context).
+    Returns OPT."""
+    import torch
+
+    need = mpt_workspace_bytes(ctx)
+    if workspace is None:
+        if ctx.workspace is None or ctx.workspace.numel() < need:
+            ctx.workspace = torch.empty(need, dtype=torch.uint8, device="cuda")
+        workspace = ctx.workspace
+    if not (workspace.is_cuda and workspace.dtype == torch.uint8 and workspace.is_contiguous()):
+        raise ValueError("workspace must be a contiguous CUDA uint8 tensor")
+    s = _default_stream_ptr() if stream is None else int(stream)
+    opt = ctypes.c_int64()
+    _check(load().mpt_solve(ctx.handle, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                            ctypes.c_void_p(s), ctypes.byref(opt)), "mpt_solve", ctx)
+    ctx._solved_ws = workspace
+    return int(opt.value)
+
+
+def mpt_tables(ctx: Context):
+    """Device views (torch tensors of length 2^m) of F, wI and split."""
+    import torch
+
+    pF, pW, pS = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+    _check(load().mpt_tables(ctx.handle, ctypes.byref(pF), ctypes.byref(pW), ctypes.byref(pS)), "mpt_tables", ctx)
+    ws = ctx._solved_ws
+    base = ws.data_ptr()
+    N = 1 << ctx.m
+
+    def view(ptr, nbytes, dtype):
+        off = ptr.value - base
+        if off < 0 or off + nbytes > ws.numel():
+            raise RuntimeError("table pointer outside the workspace")
+        return ws[off:off + nbytes].view(dtype)
+
+    return view(pF, 8 * N, torch.int64), view(pW, 8 * N, torch.int64), view(pS, 4 * N, torch.int32)
+
+
+def mpt_layout(ctx: Context):
+    """(perm_offsets int64[m+1], perm_chunks int64[sum |R_i|], dfs_order int32[m])."""
+    lib = load()
+    total = ctypes.c_int64()
+    _check(lib.mpt_layout_size(ctx.handle, ctypes.byref(total)), "mpt_layout_size", ctx)
+    offs = np.zeros(ctx.m + 1, dtype=np.int64)
+    chunks = np.zeros(max(1, total.value), dtype=np.int64)
+    dfs = np.zeros(ctx.m, dtype=np.int32)
+    _check(lib.mpt_layout(ctx.handle, _ptr(offs, ctypes.c_int64), _ptr(chunks, ctypes.c_int64),
+                          _ptr(dfs, ctypes.c_int32)), "mpt_layout", ctx)
+    return offs, chunks[:total.value], dfs
+
+
+def mpt_trie_cost(weights, perm_offsets, perm_chunks) -> int:
+    """Trie cost (eq. 1) of a layout, computed by the library's kernel."""
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    offs = np.ascontiguousarray(perm_offsets, dtype=np.int64)
+    ch = np.ascontiguousarray(perm_chunks, dtype=np.int64)
+    if ch.size == 0:
+        ch = np.zeros(1, dtype=np.int64)
+    m = int(offs.shape[0]) - 1
+    out = ctypes.c_int64()
+    _check(load().mpt_trie_cost(_ptr(w, ctypes.c_int64), int(w.shape[0]), m, _ptr(offs, ctypes.c_int64),
+                                _ptr(ch, ctypes.c_int64), ctypes.byref(out)), "mpt_trie_cost")
+    return int(out.value)
+
+
+def mpt_destroy(ctx: Context) -> None:
+    if ctx.handle and ctx.handle.value:
+        load().mpt_destroy(ctx.handle)
+        ctx.handle = ctypes.c_void_p()
+
+
+@dataclass
+class Result:
+    opt: int
+    perm_offsets: np.ndarray
+    perm_chunks: np.ndarray
+    dfs_order: np.ndarray
+    ctx: Context
+
+    def permutations(self) -> list[list[int]]:
+        o = self.perm_offsets
+        return [self.perm_chunks[o[i]:o[i + 1]].tolist() for i in range(len(o) - 1)]
+
+
+def solve(weights, bits, mode: str = "auto", workspace=None, stream: Optional[int] = None,
+          profile: bool = False) -> Result:
+    """Exact MPT solve of one instance: OPT, per-request permutations and the
+    DFS serving order.  ``result.ctx`` keeps the device tables alive."""
+    ctx = mpt_create(weights, bits)
+    if mode != "auto":
+        mpt_set_dp_mode(ctx, mode)
+    if profile:
+        mpt_set_profiling(ctx, True)
+    opt = mpt_solve(ctx, workspace, stream)
+    offs, chunks, dfs = mpt_layout(ctx)
+    return Result(opt, offs, chunks, dfs, ctx)

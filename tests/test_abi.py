@@ -1,0 +1,97 @@
+"""The C ABI without a GPU: the library loads, exports every declared entry
+point, and its host-side argument checks return the documented statuses."""
+
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2609_13692_gb300 import build as B
+from paper_2609_13692_gb300 import instances as I
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def mpt():
+    B.build()
+    from paper_2609_13692_gb300 import mpt as M
+
+    M.load()
+    return M
+
+
+def declared_functions():
+    names = []
+    for hdr in os.listdir(os.path.join(ROOT, "include")):
+        if hdr.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", hdr)).read()
+            names += re.findall(r"^\s*(?:mpt_status|void|const char\*)\s+(mpt_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(mpt):
+    lib = mpt.load()
+    names = declared_functions()
+    assert "mpt_solve" in names and "mpt_layout" in names and "mpt_trie_cost" in names
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(mpt.EXPORTED) == names
+
+
+def _status(mpt, w, bits, m=None):
+    import ctypes
+
+    lib = mpt.load()
+    w = np.ascontiguousarray(w, dtype=np.int64)
+    bits = np.ascontiguousarray(bits, dtype=np.uint64)
+    h = ctypes.c_void_p()
+    st = lib.mpt_create(w.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), int(w.shape[0]),
+                        bits.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64)),
+                        int(bits.shape[0] if m is None else m), ctypes.byref(h))
+    if st == 0:
+        lib.mpt_destroy(h)
+    return st
+
+
+def test_create_validation(mpt):
+    inst = I.config(1)
+    assert _status(mpt, inst.weights, inst.bits) == 0
+    assert _status(mpt, inst.weights, inst.bits, m=0) == 1
+    bad = inst.weights.copy()
+    bad[3] = 0
+    assert _status(mpt, bad, inst.bits) == 1
+    bits = inst.bits.copy()
+    bits[0, 0] |= np.uint64(1) << np.uint64(50)  # chunk 50 >= n = 48
+    assert _status(mpt, inst.weights, bits) == 1
+    big = I.random_instance(31, 40, 3, seed=1)
+    assert _status(mpt, big.weights, big.bits) == 2
+    huge = I.Instance(np.full(4, 1 << 61, dtype=np.int64), I.pack_requests([[0, 1], [2, 3], [0]], 4))
+    assert _status(mpt, huge.weights, huge.bits) == 3
+
+
+def test_workspace_and_modes(mpt):
+    inst = I.config(2)  # m = 20
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    auto = mpt.mpt_workspace_bytes(ctx)
+    N = 1 << 20
+    assert auto >= N * (8 + 8 + 4 + 4 + 4)  # wI, F, split and the two blocked tables
+    mpt.mpt_set_dp_mode(ctx, "general")
+    assert N * 20 <= mpt.mpt_workspace_bytes(ctx) < auto
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_layout(ctx)
+    assert e.value.status == 7
+    heavy = I.Instance(np.full(20, 60000, dtype=np.int64), inst.bits)  # sum_i w(R_i) >= 2^20
+    ctx2 = mpt.mpt_create(heavy.weights, heavy.bits)
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_set_dp_mode(ctx2, "blocked")
+    assert e.value.status == 3
+    mpt.mpt_destroy(ctx)
+    mpt.mpt_destroy(ctx2)
+
+
+def test_status_strings(mpt):
+    lib = mpt.load()
+    for code in range(10):
+        assert lib.mpt_status_string(code)

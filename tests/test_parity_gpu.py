@@ -1,0 +1,190 @@
+"""CUDA path vs the CPU oracle, through the C ABI.
+
+Integer results must be bit-exact: OPT, every F(S), every w(I(S)), every
+split(S), the per-request permutations and the DFS order.  Where the oracle
+cannot run the whole recurrence (m >= 24), sampled subsets are recomputed by
+the oracle from the GPU's own table of smaller subsets, w(I(S)) is recomputed
+from scratch, and the trie cost of the returned layout must equal OPT.
+"""
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_13692_gb300 import instances as I
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def mpt():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_13692_gb300 import build as B
+
+    B.build()
+    O.build()
+    from paper_2609_13692_gb300 import mpt as M
+
+    M.load()
+    return M
+
+
+def gpu_solve(mpt, inst, mode="auto"):
+    res = mpt.solve(inst.weights, inst.bits, mode=mode, profile=True)
+    F, wI, split = (t.cpu().numpy() for t in mpt.mpt_tables(res.ctx))
+    prof = mpt.mpt_get_profile(res.ctx)
+    return res, F, wI, split.view(np.uint32), prof
+
+
+def assert_full_parity(mpt, inst, mode="auto", expect_mode=None):
+    res, F, wI, split, prof = gpu_solve(mpt, inst, mode)
+    opt, oF, owI, osplit = O.solve(inst.weights, inst.bits)
+    if expect_mode is not None:
+        assert prof["dp_mode"] == expect_mode
+    assert res.opt == opt
+    assert np.array_equal(wI, owI), np.flatnonzero(wI != owI)[:10]
+    assert np.array_equal(F, oF), np.flatnonzero(F != oF)[:10]
+    assert np.array_equal(split, osplit), np.flatnonzero(split != osplit)[:10]
+    perms, dfs = O.layout(inst.weights, inst.bits, osplit)
+    assert res.permutations() == perms
+    assert res.dfs_order.tolist() == dfs
+    assert O.trie_cost(inst.weights, res.permutations()) == opt
+    assert mpt.mpt_trie_cost(inst.weights, res.perm_offsets, res.perm_chunks) == opt
+    return res, prof
+
+
+def test_config1_bit_exact(mpt):
+    """Zipf m = 12, 48 chunks, k = 5 (one in-tile launch)."""
+    assert_full_parity(mpt, I.config(1), expect_mode=1)
+
+
+def test_config2_leave_one_out(mpt):
+    """L_20: OPT = 20*5 - 32 + 20 = 88 (Thm 5); all tables bit-exact."""
+    res, prof = assert_full_parity(mpt, I.config(2), expect_mode=1)
+    assert res.opt == O.loo_free(20) == 88
+
+
+@pytest.mark.parametrize("m", list(range(1, 19)))
+def test_random_sweep_blocked(mpt, m):
+    rng = np.random.default_rng(1000 + m)
+    n = int(rng.integers(1, 300))
+    inst = I.random_instance(m, n, (0, min(n, 14)), seed=int(rng.integers(1 << 30)), wmin=1, wmax=512,
+                             allow_empty=True)
+    assert_full_parity(mpt, inst, "blocked", expect_mode=1)
+
+
+@pytest.mark.parametrize("m", [1, 2, 5, 9, 10, 11, 12, 13, 14, 16])
+def test_random_sweep_general(mpt, m):
+    inst = I.random_instance(m, 64, (1, 12), seed=77 + m, wmin=1, wmax=1000)
+    assert_full_parity(mpt, inst, "general", expect_mode=2)
+
+
+@pytest.mark.parametrize("n", [13, 14, 15, 16, 17, 18])
+def test_leave_one_out_ties(mpt, n):
+    """Unit weights give many optimal splits: the tie rule is exercised everywhere."""
+    res, prof = assert_full_parity(mpt, I.leave_one_out(n), expect_mode=1)
+    assert res.opt == O.loo_free(n)
+
+
+def test_paper_examples(mpt):
+    for inst, opt in ((I.k4_3(), 8), (I.open_problem_k4(), 14), (I.tightness_witness(), 10)):
+        res, prof = assert_full_parity(mpt, inst)
+        assert res.opt == opt
+
+
+def test_edge_cases(mpt):
+    cases = [
+        I.Instance(np.array([5], dtype=np.int64), I.pack_requests([[0]], 1)),                   # m = 1, n = 1
+        I.Instance(np.array([3, 4], dtype=np.int64), I.pack_requests([[], [0, 1], []], 2)),     # empty requests
+        I.Instance(np.arange(1, 9, dtype=np.int64), I.pack_requests([[1, 2, 3]] * 14, 8)),      # identical requests
+        I.Instance(np.arange(1, 17, dtype=np.int64), I.pack_requests([[i] for i in range(16)], 16)),  # disjoint
+        I.Instance(np.ones(200, dtype=np.int64), I.pack_requests([[199]] * 15, 200)),           # last chunk only
+        I.random_instance(15, 3, (0, 3), seed=5, allow_empty=True),                              # tiny universe
+    ]
+    for inst in cases:
+        for mode in ("blocked", "general"):
+            assert_full_parity(mpt, inst, mode)
+
+
+def test_large_weights_use_general(mpt):
+    """sum_i w(R_i) >= 2^20: the packed 32-bit keys would overflow, AUTO picks the int64 kernels."""
+    inst = I.random_instance(14, 50, (3, 12), seed=9, wmin=10 ** 9, wmax=10 ** 12)
+    assert_full_parity(mpt, inst, "auto", expect_mode=2)
+
+
+def test_sum_just_below_blocked_limit(mpt):
+    """Largest weights the blocked kernels accept: sum_i w(R_i) = 2^20 - 1."""
+    m = 15
+    reqs = [[i, (i + 1) % 20, (i + 7) % 20] for i in range(m)]
+    w = np.full(20, 1, dtype=np.int64)
+    total_slots = sum(len(r) for r in reqs)
+    w[:] = (2 ** 20 - 1) // total_slots
+    inst = I.Instance(w, I.pack_requests(reqs, 20))
+    slack = 2 ** 20 - 1 - int(sum(w[x] for r in reqs for x in r))
+    inst.weights[reqs[0][0]] += slack // sum(1 for r in reqs if reqs[0][0] in r)
+    assert sum(int(inst.weights[x]) for r in reqs for x in r) < 2 ** 20
+    assert_full_parity(mpt, inst, "blocked", expect_mode=1)
+
+
+def _sample_subsets(m, rng, uniform=20000, budget_per_layer=2.0e7):
+    """Uniform random subsets plus, per size k, as many random k-subsets as a
+    budget of splits allows (the full set always included)."""
+    full = (1 << m) - 1
+    out = set(int(x) for x in rng.integers(1, full + 1, size=uniform, dtype=np.int64))
+    for k in range(1, m + 1):
+        per = 2.0 ** (k - 1)
+        cnt = int(min(200, max(1, budget_per_layer // per)))
+        for _ in range(cnt):
+            members = rng.choice(m, size=k, replace=False)
+            out.add(int(sum(1 << int(i) for i in members)))
+    out.add(full)
+    return np.array(sorted(out), dtype=np.uint64)
+
+
+def assert_sampled_parity(mpt, inst, seed, uniform=20000):
+    res, F, wI, split, prof = gpu_solve(mpt, inst)
+    m = inst.m
+    full = (1 << m) - 1
+    assert res.opt == F[full]
+    # the layout realises OPT (Thm 1), checked by two independent trie builders
+    assert O.trie_cost(inst.weights, res.permutations()) == res.opt
+    assert mpt.mpt_trie_cost(inst.weights, res.perm_offsets, res.perm_chunks) == res.opt
+    R = O.request_sets(inst.weights, inst.bits)
+    for i, p in enumerate(res.permutations()):
+        assert sorted(p) == sorted(R[i])
+    assert sorted(res.dfs_order.tolist()) == list(range(m))
+    # bounds of Sec. 6.3 and Sec. 3.1
+    assert O.spanning_tree_bound(inst.weights, inst.bits) <= res.opt <= O.global_order_cost(inst.weights, inst.bits)
+    # sampled recomputation
+    rng = np.random.default_rng(seed)
+    subsets = _sample_subsets(m, rng, uniform=uniform)
+    Fr, sr, wr = O.recompute(inst.weights, inst.bits, F, subsets)
+    idx = subsets.astype(np.int64)
+    assert np.array_equal(wr, wI[idx]), idx[np.flatnonzero(wr != wI[idx])[:10]]
+    assert np.array_equal(Fr, F[idx]), idx[np.flatnonzero(Fr != F[idx])[:10]]
+    assert np.array_equal(sr, split[idx]), idx[np.flatnonzero(sr != split[idx])[:10]]
+    return res, prof, len(subsets)
+
+
+def test_config3_m24(mpt):
+    """RAG-shaped m = 24: every w(I(S)) bit-exact; sampled F and split."""
+    inst = I.config(3)
+    res, prof, count = assert_sampled_parity(mpt, inst, seed=24)
+    wI = mpt.mpt_tables(res.ctx)[1].cpu().numpy()
+    assert np.array_equal(wI, O.intersection_weights(inst.weights, inst.bits))
+    assert prof["dp_mode"] == 1 and count > 20000
+
+
+def test_config4_m28(mpt):
+    """RAG-shaped m = 28, k = 20: the benchmark workload, same launch path."""
+    res, prof, count = assert_sampled_parity(mpt, I.config(4), seed=28, uniform=100000)
+    assert prof["dp_mode"] == 1 and count >= 100000
+
+
+def test_config5_m30(mpt):
+    """RAG-shaped m = 30, k = 40, 1M-passage corpus."""
+    res, prof, count = assert_sampled_parity(mpt, I.config(5), seed=30, uniform=20000)
+    assert prof["dp_mode"] == 1
