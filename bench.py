@@ -238,7 +238,7 @@ def run_ours(args):
         B.build()
     mpt.load()
 
-    inst = instances.config(WORKLOAD, seed=replica_seed(rank))
+    inst = instances.config(args.workload, seed=replica_seed(rank))
     m = inst.m
     splits = splits_per_solve(m)
 
@@ -345,10 +345,12 @@ def run_ours(args):
         "dtype": "u32" if dp_mode == "blocked" else "int64",
         "data": "synthetic",
         "solve_time_s": solve_s,
-        "config": {"workload": instances.CONFIG_NAMES[WORKLOAD], "m": m, "n": inst.n, "k": 20, "seed": 0,
+        "config": {"workload": instances.CONFIG_NAMES[args.workload], "m": m, "n": inst.n,
+                   "k": instances.CONFIGS[args.workload].get("k", m - 1), "seed": replica_seed(rank),
                    "splits_per_solve": splits, "dp_mode": dp_mode,
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "l2": "inputs larger than L2: the 2^28-entry tables span 5 GiB (L2 129 MB), no flush",
+                   "l2": f"inputs larger than L2: the 2^{m}-entry tables span {(1 << m) * 28 / 2**30:.2f} GiB "
+                         "(L2 129 MB), no flush",
                    "opt": opts[-1] if opts else None},
         "roofline": roofline,
         "gather_roofline_frac": gather_frac,
@@ -370,6 +372,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--dp-mode", choices=["auto", "blocked", "general"], default="auto")
+    ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5],
+                    help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":

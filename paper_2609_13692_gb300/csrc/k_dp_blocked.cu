@@ -253,9 +253,10 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   for (int i = threadIdx.x; i < (1 << kB); i += kPairThreads) atomicMin(&out[i], merged[i]);
 }
 
-// Tile kernel: finishes every entry of the tiles with |T| = kh, level by level
-// in |U|, folding in the self pair (kh >= 1) or running the whole recurrence
-// on the inner bits (kh = 0).  One block per tile.
+// Generic tile kernel: finishes every entry of the tiles with |T| = kh, level
+// by level in |U|, folding in the self pair (kh >= 1) or running the whole
+// recurrence on the inner bits (kh = 0).  One block per tile.  Used for tile 0
+// (any b <= 12); the tiles with kh >= 1 go to k_dp_tile_rows.
 __global__ void __launch_bounds__(kTileThreads)
 k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned long long* __restrict__ partial,
           uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, int64_t* __restrict__ F, uint32_t* __restrict__ split) {
@@ -361,6 +362,145 @@ k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned l
   }
 }
 
+// Row-blocked tile kernel for |T| = kh >= 1 (inner bits b = kB).  The self
+// pair of output U = (s1, s2) has candidates Ua = (a1, a2) with Ua a proper
+// subset of U, A = (T, Ua) from this tile and B = (0, U \ Ua) from tile 0:
+//   * cross-row: a1 a proper subset of s1, any a2 in s2 -- rows of this tile
+//     finished at an earlier popcount level of s1, combined with whole rows of
+//     tile 0 by the same register convolution as the pair kernel;
+//   * in-row: a1 = s1, a2 a proper subset of s2 -- a 5-bit recurrence inside
+//     the row, in registers, in increasing s2 (every proper subset of s2 is
+//     smaller than s2).
+// Rows are finished level by level in |s1|, so every row read is final.
+constexpr int kRowsThreads = 96;
+constexpr int kRowsSmemBytes = (2 * kWin + 2 * (1 << kB)) * (int)sizeof(uint32_t);
+
+__global__ void __launch_bounds__(kRowsThreads)
+k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned long long* __restrict__ partial,
+               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, int64_t* __restrict__ F,
+               uint32_t* __restrict__ split) {
+  extern __shared__ __align__(16) uint32_t smem[];
+  uint32_t* cur = smem;               // this tile, F << kB, padded rows
+  uint32_t* zc = smem + kWin;         // tile 0, complement form, padded rows
+  uint32_t* bkey = smem + 2 * kWin;   // best key per output so far
+  uint32_t* bsplit = bkey + (1 << kB);  // its Ta; after finishing, the split A
+  constexpr uint32_t kMask = (1u << kB) - 1u;
+
+  const uint32_t tile = blockIdx.x;
+  const uint32_t T = colex_unrank(tile, kh, L);
+  const size_t tbase = (size_t)T << kB;
+
+  for (int c = threadIdx.x; c < (1 << (kB - 2)); c += kRowsThreads) {
+    const int row = c >> (kB2 - 2), k = c & ((1 << (kB2 - 2)) - 1);
+    *reinterpret_cast<uint4*>(zc + row_pos((uint32_t)row) * kRowStride + 4 * k) =
+        *reinterpret_cast<const uint4*>(Gc + 4 * c);
+  }
+  for (int u = threadIdx.x; u < (1 << kB); u += kRowsThreads) {
+    const unsigned long long pv = kh >= 2 ? partial[((size_t)tile << kB) | (uint32_t)u] : ~0ull;
+    bkey[u] = (uint32_t)(pv >> 32);
+    bsplit[u] = (uint32_t)pv;
+  }
+  __syncthreads();
+
+  for (int p1 = 0; p1 <= kB1; ++p1) {
+    const int rows = (int)c_binom.v[kB1][p1];
+    if (p1 >= 1) {
+      // lanes per row chosen so that each lane runs at most 8 row pairs
+      const int g = p1 > 3 ? p1 - 3 : 0;
+      const int G = 1 << g;
+      const int ri = (int)(threadIdx.x >> g);
+      const uint32_t r = threadIdx.x & (uint32_t)(G - 1);
+      const bool active = ri < rows;
+      uint32_t acc[kRow];
+#pragma unroll
+      for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
+      uint32_t s1 = 0;
+      if (active) {
+        s1 = colex_unrank((unsigned long long)ri, p1, kB1);
+        uint32_t hi = 0, rr = s1;
+        for (int t = 0; t < g; ++t) {
+          const uint32_t top = 1u << (31 - __clz(rr));
+          hi |= top;
+          rr ^= top;
+        }
+        const uint32_t freem = s1 ^ hi;
+        const uint32_t fixed = deposit_bits(r, hi);
+        uint32_t sub = 0;
+        do {
+          const uint32_t a1 = fixed | sub;
+          if (a1 != s1) {
+            uint32_t x[kRow], y[kRow];
+            load_row(x, cur + row_pos(a1) * kRowStride);
+            load_row(y, zc + row_pos(s1 ^ a1) * kRowStride);
+            conv_rows(acc, x, y);
+          }
+          sub = (sub - freem) & freem;
+        } while (sub != 0);
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) {
+#pragma unroll
+        for (int i = 0; i < kRow; ++i) acc[i] = min(acc[i], __shfl_xor_sync(0xFFFFFFFFu, acc[i], off));
+      }
+      if (active && r == 0) {
+#pragma unroll
+        for (int i = 0; i < kRow; ++i) {
+          const uint32_t U = (s1 << kB2) | (uint32_t)i;
+          if (acc[i] < bkey[U]) {
+            bkey[U] = acc[i];
+            bsplit[U] = T;
+          }
+        }
+      }
+      __syncthreads();
+    }
+    if ((int)threadIdx.x < rows) {
+      const uint32_t s1 = colex_unrank((unsigned long long)threadIdx.x, p1, kB1);
+      uint32_t z[kRow], c[kRow], wv[kRow];
+      load_row(z, zc + row_pos(0) * kRowStride);
+#pragma unroll
+      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)wI[((size_t)((s1 << kB2) | (uint32_t)i) << L) | T];
+#pragma unroll
+      for (int s2 = 0; s2 < kRow; ++s2) {
+        uint32_t key = 0xFFFFFFFFu;
+#pragma unroll
+        for (int a2 = 0; a2 < kRow; ++a2) {
+          if ((a2 & s2) == a2 && a2 != s2) key = min(key, c[a2] + z[s2 ^ a2]);
+        }
+        const uint32_t U = (s1 << kB2) | (uint32_t)s2;
+        uint32_t bk = bkey[U], bt = bsplit[U];
+        if (key < bk) {
+          bk = key;
+          bt = T;
+        }
+        uint32_t f, A;
+        if (kh == 1 && U == 0) {  // S = T, a single request
+          f = wv[s2];
+          A = 0;
+        } else {
+          const uint32_t Ua = (bk & kMask) + U - kMask;
+          f = (bk >> kB) - wv[s2];
+          A = (Ua << L) | bt;
+        }
+        c[s2] = f << kB;
+        bsplit[U] = A;
+      }
+      uint4* dst = reinterpret_cast<uint4*>(cur + row_pos(s1) * kRowStride);
+#pragma unroll
+      for (int q = 0; q < kRow / 4; ++q) dst[q] = make_uint4(c[4 * q], c[4 * q + 1], c[4 * q + 2], c[4 * q + 3]);
+    }
+    __syncthreads();
+  }
+
+  for (int u = threadIdx.x; u < (1 << kB); u += kRowsThreads) {
+    const uint32_t gp = cur[row_pos((uint32_t)u >> kB2) * kRowStride + (u & (kRow - 1))];
+    Gp[tbase | (uint32_t)u] = gp;
+    Gc[tbase | (uint32_t)u] = gp | (~(uint32_t)u & kMask);
+    const size_t S = ((size_t)u << L) | T;
+    F[S] = (int64_t)(gp >> kB);
+    split[S] = bsplit[u];
+  }
+}
+
 }  // namespace
 
 int blocked_tile_bits(int m) { return m < kB ? m : kB; }
@@ -380,6 +520,8 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
   static bool attr_done = false;
   if (!attr_done) {
     cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_dp_tile_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
@@ -411,8 +553,12 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
       if (e != cudaSuccess) return e;
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches], stream);
-    k_dp_tile<<<(unsigned)tiles, kTileThreads, 0, stream>>>(L, b, kh, ws.wI, kh >= 2 ? ws.partial : nullptr, ws.Gp,
-                                                            ws.Gc, ws.F, ws.split);
+    if (kh == 0) {
+      k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI, nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
+    } else {
+      k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(
+          L, kh, ws.wI, kh >= 2 ? ws.partial : nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
+    }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;
     ++*launches;
