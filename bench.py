@@ -38,9 +38,12 @@ METRIC = "subset-splits evaluated/sec (≈3^m/2 per solve) and exact-MPT solve t
 WORKLOAD = 4
 ORACLE_SAMPLE_REQUESTS = 22  # reference arm: full oracle recurrence on the first 22 requests per step
 CPU_BASELINE_REQUESTS = 23  # cpu_baseline: one run on the first 23 requests (10-30 s of CPU work)
-# int32 lanes per SM x SMs (GB300: 152 SMs of 4 x 32 lanes) x max SM clock
-ALU_PEAK_TOPS = 152 * 128 * 2.070e9 / 1e12
-OPS_PER_SPLIT = 2  # one add and one min per split
+# Integer ALU pipe: 152 SMs x 4 sub-partitions x 16 lanes per clock, at the
+# 2.07 GHz maximum SM clock.  Each split is one 32-bit add and min, which the
+# pair kernel issues as one instruction on that pipe (ncu: its arithmetic runs
+# on the ALU pipe; about 1.3 instructions per split in all).
+ALU_PEAK_TOPS = 152 * 64 * 2.070e9 / 1e12
+OPS_PER_SPLIT = 1
 
 
 def splits_per_solve(m: int) -> int:
@@ -312,7 +315,7 @@ def run_ours(args):
                     "unit": "Tops/s", "frac": achieved / ALU_PEAK_TOPS,
                     "traffic": (tr or {}).get("dram_bytes_per_launch"),
                     "ops_per_split": OPS_PER_SPLIT,
-                    "peak_basis": "152 SMs x 128 int32 lanes x 2.07 GHz (nominal units and max clock)",
+                    "peak_basis": "152 SMs x 64 integer-ALU-pipe lanes x 2.07 GHz (one add-min per split)",
                     "share_of_step": prof_sum["ms_dp_pairs"] / (local_ms if local_ms > 0 else 1)}
     else:
         hbm = float(peaks.get("hbm_gbs", 6800.0))

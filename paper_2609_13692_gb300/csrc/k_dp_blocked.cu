@@ -41,8 +41,12 @@ constexpr int kRow = 1 << kB2;             // 32 entries per row
 constexpr int kRowStride = kRow + 4;       // 36 words: consecutive rows start in different 16-byte bank groups
 constexpr int kRows = 1 << kB1;            // 128 rows per window
 constexpr int kWin = kRows * kRowStride;   // words per padded window
-constexpr int kPairThreads = 320;
-constexpr int kPairSmemBytes = 2 * 2 * kWin * (int)sizeof(uint32_t);  // double-buffered X and Y windows
+constexpr int kPairThreads = 256;         // 8 warps: 2 per SM sub-partition, equal work each
+constexpr int kUnitsPerTask = 8;           // row pairs per register task
+constexpr int kSharedRows = 34;            // rows merged through shared memory every pair
+constexpr int kSharedOut = kSharedRows * kRow;
+constexpr int kSharedOwned = (kSharedOut + kPairThreads - 1) / kPairThreads;
+constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedOut) * (int)sizeof(uint32_t);
 constexpr int kMinPairsPerItem = 16;
 constexpr int kTileThreads = 512;
 constexpr int kMaxTileBits = 12;
@@ -50,20 +54,24 @@ constexpr int kMaxTileBits = 12;
 static_assert(kPairSmemBytes >= (1 << kB) * 8, "merge buffer must fit in the window buffers");
 
 // ---------------------------------------------------------------------------
-// Per-thread work of the pair kernel.  The b inner bits are (s1, s2): s1 = the
-// top kB1 bits (window row), s2 = the low kB2 bits (register lane).  Output
+// Work split of the pair kernel.  The b inner bits are (s1, s2): s1 = the top
+// kB1 bits (window row), s2 = the low kB2 bits (register lane).  Output
 // (s1, s2) collects, for every Ua = (a1, a2) with a1 in s1 and a2 in s2,
-// X[a1][a2] + Y[s1^a1][s2^a2].  A "unit" is one (s1, a1): two rows, 243 adds.
-// A thread owns one s1 (its 32 outputs) and a fixed subset of the a1 in s1:
-// rows with >= 3 bits are split on their lowest set bits into tasks of 8 a1
-// each; rows with < 3 bits are one task.  Packed as s1 | fixed << 8 | free << 16.
+// X[a1][a2] + Y[s1^a1][s2^a2].  A "unit" is one (s1, a1): two rows, 243
+// add-min steps; row s1 has 2^|s1| units, 3^7 = 2187 in all.
+//
+// Register rows: every row with >= 3 bits except the first five with exactly
+// 3 -- 94 rows, 2048 units -- split on their lowest set bits into 256 tasks of
+// exactly 8 units, one per thread.  A thread keeps the 32 outputs of its task
+// in registers across all pairs (running best key and Ta), merged with the
+// other tasks of the row once, at the end.
+// Shared rows: the 29 rows with <= 2 bits and those five -- 34 rows, 139
+// units.  Each unit is one extra unit of some thread (spread evenly over the
+// 8 warps); its 32 minima go to a per-pair shared array with atomicMin, and
+// owner threads fold that array into registers after every pair.
+// So every warp issues 8 units plus at most one extra unit per pair.
 // ---------------------------------------------------------------------------
-struct TaskTable {
-  uint32_t t[kPairThreads];
-  int count;
-};
-
-constexpr int popc_c(uint32_t v) {
+__host__ __device__ constexpr int popc_c(uint32_t v) {
   int c = 0;
   while (v) {
     v &= v - 1;
@@ -83,13 +91,32 @@ constexpr uint32_t deposit_c(uint32_t q, uint32_t mask) {
   return out;
 }
 
-constexpr TaskTable make_tasks() {
-  TaskTable tt{};
-  int n = 0;
+struct PairPlan {
+  uint32_t task[kPairThreads];   // s1 | fixed << 8 | free << 16 (8 units)
+  uint32_t extra[kPairThreads];  // s1 | a1 << 8 | shared-row index << 16, or ~0u
+  uint32_t srow[kSharedRows];    // s1 of each shared row
+  int ntask, nextra, nsrow;
+};
+
+constexpr bool is_shared_row(uint32_t s1) {
+  const int p = popc_c(s1);
+  if (p <= 2) return true;
+  if (p != 3) return false;
+  int rank = 0;  // the first five 3-bit rows in increasing s1 are shared
+  for (uint32_t t = 0; t < s1; ++t)
+    if (popc_c(t) == 3) ++rank;
+  return rank < 5;
+}
+
+constexpr PairPlan make_plan() {
+  PairPlan pl{};
+  int n = 0, nr = 0, ne = 0;
   for (uint32_t s1 = 0; s1 < (uint32_t)kRows; ++s1) {
-    const int p = popc_c(s1);
-    if (p < 3) continue;
-    const int q = p - 3;
+    if (is_shared_row(s1)) {
+      pl.srow[nr++] = s1;
+      continue;
+    }
+    const int q = popc_c(s1) - 3;
     uint32_t lowbits = 0, r = s1;
     for (int t = 0; t < q; ++t) {
       const uint32_t lb = r & (~r + 1u);
@@ -97,19 +124,34 @@ constexpr TaskTable make_tasks() {
       r ^= lb;
     }
     const uint32_t freem = s1 ^ lowbits;
-    for (uint32_t v = 0; v < (1u << q); ++v) tt.t[n++] = s1 | (deposit_c(v, lowbits) << 8) | (freem << 16);
+    for (uint32_t v = 0; v < (1u << q); ++v) pl.task[n++] = s1 | (deposit_c(v, lowbits) << 8) | (freem << 16);
   }
-  for (int p = 2; p >= 0; --p)
-    for (uint32_t s1 = 0; s1 < (uint32_t)kRows; ++s1)
-      if (popc_c(s1) == p) tt.t[n++] = s1 | (s1 << 16);
-  tt.count = n;
-  for (int i = n; i < kPairThreads; ++i) tt.t[i] = 0xFFFFFFFFu;
-  return tt;
+  for (int i = 0; i < kPairThreads; ++i) pl.extra[i] = 0xFFFFFFFFu;
+  for (int ri = 0; ri < nr; ++ri) {
+    const uint32_t s1 = pl.srow[ri];
+    for (uint32_t k = 0; k < (1u << popc_c(s1)); ++k) {
+      const uint32_t a1 = deposit_c(k, s1);
+      const int tid = (ne % 8) * 32 + ne / 8;  // extra unit ne -> warp ne % 8
+      pl.extra[tid] = s1 | (a1 << 8) | ((uint32_t)ri << 16);
+      ++ne;
+    }
+  }
+  pl.ntask = n;
+  pl.nextra = ne;
+  pl.nsrow = nr;
+  return pl;
 }
 
-constexpr TaskTable kTasksHost = make_tasks();
-static_assert(kTasksHost.count <= kPairThreads, "task table exceeds the block");
-static __constant__ TaskTable c_tasks = make_tasks();
+constexpr PairPlan kPlanHost = make_plan();
+static_assert(kPlanHost.ntask == kPairThreads, "register tasks must fill the block");
+static_assert(kPlanHost.nsrow == kSharedRows, "shared row count");
+static_assert(kPlanHost.nextra == 139 && kPlanHost.nextra <= kPairThreads, "extra units");
+static __constant__ PairPlan c_plan = make_plan();
+
+// Word of shared output j = (shared row, lane) in a per-pair minimum array:
+// the lane bits are XOR-ed with the row index so that lanes flushing
+// different rows hit different banks.
+__device__ __forceinline__ uint32_t sw_word(uint32_t j) { return j ^ ((j >> kB2) & (kRow - 1)); }
 
 // Row placement inside a padded window: the low 3 row bits are XOR-ed with
 // higher row bits so that rows that differ only above bit 2 still start in
@@ -170,7 +212,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
 k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, unsigned long long* __restrict__ partial,
            int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item) {
   extern __shared__ __align__(16) uint32_t smem[];
-  // buffer c holds X at smem + 2c * kWin and Y right after it
+  // window buffer c: X at smem + 2c * kWin, Y right after it; then two
+  // per-pair minimum arrays of the shared rows
+  uint32_t* smin = smem + 4 * kWin;
 
   const uint32_t tile = blockIdx.x / items_per_tile;
   const uint32_t item = blockIdx.x % items_per_tile;
@@ -180,17 +224,25 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t q0 = item * pairs_per_item;
   const uint32_t q1 = min(q0 + pairs_per_item, pairs_per_tile);
 
-  const uint32_t task = c_tasks.t[threadIdx.x];
-  const bool valid = task != 0xFFFFFFFFu;
+  const uint32_t task = c_plan.task[threadIdx.x];
   const uint32_t s1 = task & 0xFFu;
   const uint32_t fixed = (task >> 8) & 0xFFu;
   const uint32_t freem = (task >> 16) & 0xFFu;
+  const uint32_t extra = c_plan.extra[threadIdx.x];
+  const bool has_extra = extra != 0xFFFFFFFFu;
+  const uint32_t es1 = extra & 0xFFu, ea1 = (extra >> 8) & 0xFFu, erow = (extra >> 16) & 0xFFu;
 
-  uint32_t bk[kRow], bt[kRow];
+  for (int i = threadIdx.x; i < 2 * kSharedOut; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
+  uint32_t bk[kRow], bt[kRow], sbk[kSharedOwned], sbt[kSharedOwned];
 #pragma unroll
   for (int i = 0; i < kRow; ++i) {
     bk[i] = 0xFFFFFFFFu;
     bt[i] = 0;
+  }
+#pragma unroll
+  for (int j = 0; j < kSharedOwned; ++j) {
+    sbk[j] = 0xFFFFFFFFu;
+    sbt[j] = 0;
   }
 
   uint32_t sub = deposit_bits(q0, R);
@@ -213,40 +265,73 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
       cp_async_wait<0>();
     }
     __syncthreads();
-    if (valid) {
-      const uint32_t* X = smem + 2 * cur * kWin;
-      const uint32_t* Y = X + kWin;
+    const uint32_t* X = smem + 2 * cur * kWin;
+    const uint32_t* Y = X + kWin;
+    uint32_t* sm = smin + cur * kSharedOut;
+    {
       uint32_t acc[kRow];
 #pragma unroll
       for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
-      uint32_t s = 0;
+      uint32_t sa = 0;
       do {
-        const uint32_t a1 = fixed | s;
+        const uint32_t a1 = fixed | sa;
         uint32_t x[kRow], y[kRow];
         load_row(x, X + row_pos(a1) * kRowStride);
         load_row(y, Y + row_pos(s1 ^ a1) * kRowStride);
         conv_rows(acc, x, y);
-        s = (s - freem) & freem;
-      } while (s != 0);
+        sa = (sa - freem) & freem;
+      } while (sa != 0);
 #pragma unroll
       for (int i = 0; i < kRow; ++i) {
         const bool better = acc[i] < bk[i];
         bk[i] = better ? acc[i] : bk[i];
         bt[i] = better ? Ta : bt[i];
       }
+      if (has_extra) {
+#pragma unroll
+        for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
+        uint32_t x[kRow], y[kRow];
+        load_row(x, X + row_pos(ea1) * kRowStride);
+        load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
+        conv_rows(acc, x, y);
+#pragma unroll
+        for (int i = 0; i < kRow; ++i) atomicMin(&sm[sw_word((erow << kB2) | (uint32_t)i)], acc[i]);
+      }
     }
     __syncthreads();
+    // fold this pair's shared-row minima into their owners' running best and
+    // reset the array for the pair after next
+#pragma unroll
+    for (int j = 0; j < kSharedOwned; ++j) {
+      const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
+      if (o < (uint32_t)kSharedOut) {
+        const uint32_t w = sw_word(o);
+        const uint32_t v = sm[w];
+        sm[w] = 0xFFFFFFFFu;
+        if (v < sbk[j]) {
+          sbk[j] = v;
+          sbt[j] = Ta;
+        }
+      }
+    }
     sub = next;
   }
 
-  // Merge the threads that share an s1, then the blocks that share the tile.
+  // Merge the threads that share a row, then the blocks that share the tile.
+  __syncthreads();
   unsigned long long* merged = reinterpret_cast<unsigned long long*>(smem);
   for (int i = threadIdx.x; i < (1 << kB); i += kPairThreads) merged[i] = ~0ull;
   __syncthreads();
-  if (valid) {
 #pragma unroll
-    for (int i = 0; i < kRow; ++i)
-      atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | bt[i]);
+  for (int i = 0; i < kRow; ++i)
+    atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | bt[i]);
+#pragma unroll
+  for (int j = 0; j < kSharedOwned; ++j) {
+    const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
+    if (o < (uint32_t)kSharedOut) {
+      const uint32_t U = (c_plan.srow[o >> kB2] << kB2) | (o & (kRow - 1));
+      atomicMin(&merged[U], ((unsigned long long)sbk[j] << 32) | sbt[j]);
+    }
   }
   __syncthreads();
   unsigned long long* out = partial + ((size_t)tile << kB);
