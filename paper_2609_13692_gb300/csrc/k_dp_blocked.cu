@@ -155,7 +155,8 @@ __device__ __forceinline__ uint32_t sw_word(uint32_t j) { return j ^ ((j >> kB2)
 
 // Row placement inside a padded window: the low 3 row bits are XOR-ed with
 // higher row bits so that rows that differ only above bit 2 still start in
-// different bank groups.
+// different bank groups.  The map is linear over GF(2):
+// row_pos(a ^ b) = row_pos(a) ^ row_pos(b).
 __device__ __forceinline__ int row_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
 
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
@@ -195,12 +196,20 @@ __device__ __forceinline__ void load_row(uint32_t (&v)[kRow], const uint32_t* p)
 }
 
 // acc[s2] = min over a2 in s2 of x[a2] + y[s2 ^ a2]  (243 add/min pairs).
+// The a2-outer order puts independent accumulators next to each other.  With
+// kInit the a2 = 0 term initialises acc instead of being min-ed into it.
+template <bool kInit = false>
 __device__ __forceinline__ void conv_rows(uint32_t (&acc)[kRow], const uint32_t (&x)[kRow], const uint32_t (&y)[kRow]) {
 #pragma unroll
-  for (int s2 = 0; s2 < kRow; ++s2) {
+  for (int a2 = 0; a2 < kRow; ++a2) {
 #pragma unroll
-    for (int a2 = 0; a2 < kRow; ++a2) {
-      if ((a2 & s2) == a2) acc[s2] = min(acc[s2], x[a2] + y[s2 ^ a2]);
+    for (int s2 = 0; s2 < kRow; ++s2) {
+      if ((a2 & s2) == a2) {
+        if (kInit && a2 == 0)
+          acc[s2] = x[0] + y[s2];
+        else
+          acc[s2] = min(acc[s2], x[a2] + y[s2 ^ a2]);
+      }
     }
   }
 }
@@ -227,7 +236,12 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t task = c_plan.task[threadIdx.x];
   const uint32_t s1 = task & 0xFFu;
   const uint32_t fixed = (task >> 8) & 0xFFu;
-  const uint32_t freem = (task >> 16) & 0xFFu;
+  const uint32_t freem = (task >> 16) & 0xFFu;  // exactly 3 bits
+  const uint32_t b0 = freem & (~freem + 1u);
+  const uint32_t b1 = (freem ^ b0) & (~(freem ^ b0) + 1u);
+  const uint32_t b2 = freem ^ b0 ^ b1;
+  const uint32_t pos_fixed = (uint32_t)row_pos(fixed), pos_s1 = (uint32_t)row_pos(s1);
+  const uint32_t pb0 = (uint32_t)row_pos(b0), pb1 = (uint32_t)row_pos(b1), pb2 = (uint32_t)row_pos(b2);
   const uint32_t extra = c_plan.extra[threadIdx.x];
   const bool has_extra = extra != 0xFFFFFFFFu;
   const uint32_t es1 = extra & 0xFFu, ea1 = (extra >> 8) & 0xFFu, erow = (extra >> 16) & 0xFFu;
@@ -269,31 +283,34 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
     const uint32_t* Y = X + kWin;
     uint32_t* sm = smin + cur * kSharedOut;
     {
+      // The 8 units of the task visit a1 = fixed | sub with sub running over the
+      // subsets of its 3 free bits in Gray-code order; row_pos is linear over
+      // GF(2), so each step changes the row position by one XOR.
       uint32_t acc[kRow];
+      uint32_t pa = pos_fixed;
 #pragma unroll
-      for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
-      uint32_t sa = 0;
-      do {
-        const uint32_t a1 = fixed | sa;
+      for (int k = 0; k < 8; ++k) {
+        if (k > 0) pa ^= (k & 1) ? pb0 : ((k & 2) ? pb1 : pb2);
         uint32_t x[kRow], y[kRow];
-        load_row(x, X + row_pos(a1) * kRowStride);
-        load_row(y, Y + row_pos(s1 ^ a1) * kRowStride);
-        conv_rows(acc, x, y);
-        sa = (sa - freem) & freem;
-      } while (sa != 0);
+        load_row(x, X + pa * kRowStride);
+        load_row(y, Y + (pa ^ pos_s1) * kRowStride);
+        if (k == 0)
+          conv_rows<true>(acc, x, y);
+        else
+          conv_rows(acc, x, y);
+      }
 #pragma unroll
       for (int i = 0; i < kRow; ++i) {
-        const bool better = acc[i] < bk[i];
-        bk[i] = better ? acc[i] : bk[i];
-        bt[i] = better ? Ta : bt[i];
+        bool keep;  // true when the running best is <= this pair's minimum
+        const uint32_t m = __vibmin_u32(bk[i], acc[i], &keep);
+        bt[i] = keep ? bt[i] : Ta;
+        bk[i] = m;
       }
       if (has_extra) {
-#pragma unroll
-        for (int i = 0; i < kRow; ++i) acc[i] = 0xFFFFFFFFu;
         uint32_t x[kRow], y[kRow];
         load_row(x, X + row_pos(ea1) * kRowStride);
         load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
-        conv_rows(acc, x, y);
+        conv_rows<true>(acc, x, y);
 #pragma unroll
         for (int i = 0; i < kRow; ++i) atomicMin(&sm[sw_word((erow << kB2) | (uint32_t)i)], acc[i]);
       }
