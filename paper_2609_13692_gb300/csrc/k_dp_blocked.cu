@@ -45,8 +45,10 @@ constexpr int kPairThreads = 256;         // 8 warps: 2 per SM sub-partition, eq
 constexpr int kUnitsPerTask = 8;           // row pairs per register task
 constexpr int kSharedRows = 34;            // rows merged through shared memory every pair
 constexpr int kSharedOut = kSharedRows * kRow;
+constexpr int kSharedStride = kRow + 1;    // words per shared row in the per-pair minimum arrays
+constexpr int kSharedWords = kSharedRows * kSharedStride;
 constexpr int kSharedOwned = (kSharedOut + kPairThreads - 1) / kPairThreads;
-constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedOut) * (int)sizeof(uint32_t);
+constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedWords) * (int)sizeof(uint32_t);
 constexpr int kMinPairsPerItem = 16;
 constexpr int kTileThreads = 512;
 constexpr int kMaxTileBits = 12;
@@ -149,9 +151,9 @@ static_assert(kPlanHost.nextra == 139 && kPlanHost.nextra <= kPairThreads, "extr
 static __constant__ PairPlan c_plan = make_plan();
 
 // Word of shared output j = (shared row, lane) in a per-pair minimum array:
-// the lane bits are XOR-ed with the row index so that lanes flushing
-// different rows hit different banks.
-__device__ __forceinline__ uint32_t sw_word(uint32_t j) { return j ^ ((j >> kB2) & (kRow - 1)); }
+// rows are 33 words apart, so lanes flushing different rows, and owners
+// reading consecutive outputs, hit different banks.
+__device__ __forceinline__ uint32_t sw_word(uint32_t j) { return j + (j >> kB2); }
 
 // Row placement inside a padded window: the low 3 row bits are XOR-ed with
 // higher row bits so that rows that differ only above bit 2 still start in
@@ -169,17 +171,24 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
 }
 
-// Issue the copies of the two windows of one pair into a buffer.
+// Issue the copies of the two windows of one pair into a buffer.  Thread t
+// copies the 16-byte chunks t + kThreads * j: rows (t >> 3) + (kThreads / 8) * j
+// (mod 128) of X (first 1024 chunks) and Y, always column t & 7.  row_pos is
+// linear, so each chunk's row position is one XOR away from row_pos(t >> 3).
+template <int kThreads>
 __device__ __forceinline__ void stage_pair(uint32_t* X, uint32_t* Y, const uint32_t* __restrict__ gx,
                                            const uint32_t* __restrict__ gy) {
-  for (int c = threadIdx.x; c < 2 * (kRows * kRow / 4); c += kPairThreads) {
-    const int w = c >> (kB - 2);          // 0: X window, 1: Y window
-    const int cc = c & ((1 << (kB - 2)) - 1);
-    const int row = cc >> (kB2 - 2);
-    const int k = cc & ((1 << (kB2 - 2)) - 1);
-    uint32_t* dst = (w ? Y : X) + row_pos((uint32_t)row) * kRowStride + k * 4;
-    const uint32_t* src = (w ? gy : gx) + cc * 4;
-    cp_async16(dst, src);
+  constexpr int kChunks = kRows * kRow / 4;  // 1024 per window
+  static_assert(kChunks % kThreads == 0, "whole chunks per thread");
+  const uint32_t t = threadIdx.x;
+  const uint32_t rp0 = (uint32_t)row_pos(t >> 3);
+  const uint32_t col = (t & 7u) * 4u;
+#pragma unroll
+  for (int j = 0; j < kChunks / kThreads; ++j) {
+    const uint32_t rp = rp0 ^ (uint32_t)row_pos((uint32_t)(j * (kThreads / 8)));
+    const uint32_t d = rp * kRowStride + col;
+    cp_async16(X + d, gx + 4 * (t + (uint32_t)(j * kThreads)));
+    cp_async16(Y + d, gy + 4 * (t + (uint32_t)(j * kThreads)));
   }
 }
 
@@ -246,7 +255,7 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const bool has_extra = extra != 0xFFFFFFFFu;
   const uint32_t es1 = extra & 0xFFu, ea1 = (extra >> 8) & 0xFFu, erow = (extra >> 16) & 0xFFu;
 
-  for (int i = threadIdx.x; i < 2 * kSharedOut; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
+  for (int i = threadIdx.x; i < 2 * kSharedWords; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
   uint32_t bk[kRow], bt[kRow], sbk[kSharedOwned], sbt[kSharedOwned];
 #pragma unroll
   for (int i = 0; i < kRow; ++i) {
@@ -262,7 +271,7 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   uint32_t sub = deposit_bits(q0, R);
   {
     const uint32_t Ta = low | sub;
-    stage_pair(smem, smem + kWin, Gp + ((size_t)Ta << kB), Gc + ((size_t)(T ^ Ta) << kB));
+    stage_pair<kPairThreads>(smem, smem + kWin, Gp + ((size_t)Ta << kB), Gc + ((size_t)(T ^ Ta) << kB));
     cp_async_commit();
   }
   for (uint32_t q = q0; q < q1; ++q) {
@@ -272,7 +281,7 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
     if (q + 1 < q1) {
       const uint32_t Tn = low | next;
       uint32_t* nb = smem + 2 * (cur ^ 1) * kWin;
-      stage_pair(nb, nb + kWin, Gp + ((size_t)Tn << kB), Gc + ((size_t)(T ^ Tn) << kB));
+      stage_pair<kPairThreads>(nb, nb + kWin, Gp + ((size_t)Tn << kB), Gc + ((size_t)(T ^ Tn) << kB));
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -281,7 +290,7 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
     __syncthreads();
     const uint32_t* X = smem + 2 * cur * kWin;
     const uint32_t* Y = X + kWin;
-    uint32_t* sm = smin + cur * kSharedOut;
+    uint32_t* sm = smin + cur * kSharedWords;
     {
       // The 8 units of the task visit a1 = fixed | sub with sub running over the
       // subsets of its 3 free bits in Gray-code order; row_pos is linear over
@@ -311,8 +320,9 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
         load_row(x, X + row_pos(ea1) * kRowStride);
         load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
         conv_rows<true>(acc, x, y);
+        uint32_t* row = sm + erow * kSharedStride;
 #pragma unroll
-        for (int i = 0; i < kRow; ++i) atomicMin(&sm[sw_word((erow << kB2) | (uint32_t)i)], acc[i]);
+        for (int i = 0; i < kRow; ++i) atomicMin(&row[i], acc[i]);
       }
     }
     __syncthreads();
