@@ -145,6 +145,31 @@ typedef struct mpt_profile {
 mpt_status mpt_set_profiling(mpt_ctx* ctx, int32_t on);
 mpt_status mpt_get_profile(const mpt_ctx* ctx, mpt_profile* out);
 
+/* Exact solve that allocates nothing, for callers that cannot allocate device
+ * memory: code running in a serving process whose device memory is reserved
+ * up front by its own pool allocator, or code that must not call cudaMalloc /
+ * cudaFree because those calls synchronise the device and stall the work
+ * already running on it.  The paper has no counterpart; it is a deployment
+ * variant of mpt_solve that returns the tables and OPT but no layout.
+ *   d_weights:  device int64[n_chunks];  d_req_bits: device uint64[m][ceil(n/64)]
+ *   d_F, d_wI:  device int64[2^m];       d_split:    device uint32[2^m]
+ *   d_opt:      device int64[1]          (all caller-owned; same meaning as
+ *               mpt_tables and mpt_solve's OPT)
+ *   stream:     a cudaStream_t (NULL = the legacy default stream).
+ * Limits: m <= 20 and sum_i |R_i| <= 65536 (MPT_ERR_TOO_LARGE beyond),
+ * w(x) >= 1 and no bit at x >= n (MPT_ERR_INVALID_ARG), sum_i w(R_i) < 2^62
+ * (MPT_ERR_OVERFLOW).  The scratch -- the blocked recurrence's working tables
+ * and per-layer minima -- is one file-scope device array of 10.7 MiB that
+ * every GPU loading this library holds until the process exits.  The first
+ * call on a device looks up that array's device address, so make it before
+ * any stream capture.  The call synchronises `stream` once, to read the
+ * input check, then enqueues the solve and returns: the outputs are ready
+ * when the stream reaches that point.  Every call shares the one array and
+ * finds the previous call's contents in it; calls whose work overlaps on the
+ * GPU (other streams, other host threads) race and must be serialised. */
+mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chunks, const uint64_t* d_req_bits, int32_t m,
+                             int64_t* d_F, int64_t* d_wI, uint32_t* d_split, int64_t* d_opt, void* stream);
+
 /* Free the context and any workspace the library allocated.  NULL is a no-op. */
 void mpt_destroy(mpt_ctx* ctx);
 

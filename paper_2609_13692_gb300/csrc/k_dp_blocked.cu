@@ -42,7 +42,6 @@ constexpr int kRowStride = kRow + 4;       // 36 words: consecutive rows start i
 constexpr int kRows = 1 << kB1;            // 128 rows per window
 constexpr int kWin = kRows * kRowStride;   // words per padded window
 constexpr int kPairThreads = 256;         // 8 warps: 2 per SM sub-partition, equal work each
-constexpr int kUnitsPerTask = 8;           // row pairs per register task
 constexpr int kSharedRows = 34;            // rows merged through shared memory every pair
 constexpr int kSharedOut = kSharedRows * kRow;
 constexpr int kSharedStride = kRow + 1;    // words per shared row in the per-pair minimum arrays

@@ -39,7 +39,7 @@ STATUS_NAMES = {
 EXPORTED = [
     "mpt_create", "mpt_workspace_bytes", "mpt_set_dp_mode", "mpt_solve", "mpt_tables", "mpt_layout_size",
     "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
-    "mpt_last_error",
+    "mpt_last_error", "mpt_solve_noalloc",
 ]
 
 
@@ -107,6 +107,7 @@ def load() -> ctypes.CDLL:
         "mpt_destroy": ([vp], None),
         "mpt_status_string": ([ctypes.c_int], ctypes.c_char_p),
         "mpt_last_error": ([vp], ctypes.c_char_p),
+        "mpt_solve_noalloc": ([vp, i64, vp, i32, vp, vp, vp, vp, vp], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -258,6 +259,24 @@ def mpt_destroy(ctx: Context) -> None:
     if ctx.handle and ctx.handle.value:
         load().mpt_destroy(ctx.handle)
         ctx.handle = ctypes.c_void_p()
+
+
+def mpt_solve_noalloc(d_weights, d_bits, d_F, d_wI, d_split, d_opt, stream: Optional[int] = None) -> None:
+    """Exact solve into caller-owned device tensors without any allocation by
+    the library (for callers that cannot allocate device memory; see mpt.h).
+    d_weights: CUDA int64[n]; d_bits: CUDA 64-bit [m, ceil(n/64)] (the uint64
+    request bitsets, any 64-bit dtype); d_F, d_wI: CUDA int64[2^m];
+    d_split: CUDA int32[2^m]; d_opt: CUDA int64[1].  Enqueued on ``stream``
+    (default: torch's current stream)."""
+    for t in (d_weights, d_bits, d_F, d_wI, d_split, d_opt):
+        if not (t.is_cuda and t.is_contiguous()):
+            raise ValueError("every argument must be a contiguous CUDA tensor")
+    m, n = int(d_bits.shape[0]), int(d_weights.shape[0])
+    s = _default_stream_ptr() if stream is None else int(stream)
+    _check(load().mpt_solve_noalloc(ctypes.c_void_p(d_weights.data_ptr()), n, ctypes.c_void_p(d_bits.data_ptr()), m,
+                                    ctypes.c_void_p(d_F.data_ptr()), ctypes.c_void_p(d_wI.data_ptr()),
+                                    ctypes.c_void_p(d_split.data_ptr()), ctypes.c_void_p(d_opt.data_ptr()),
+                                    ctypes.c_void_p(s)), "mpt_solve_noalloc")
 
 
 @dataclass
