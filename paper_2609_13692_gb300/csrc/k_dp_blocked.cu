@@ -515,6 +515,15 @@ k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned lon
 
   for (int p1 = 0; p1 <= kB1; ++p1) {
     const int rows = (int)c_binom.v[kB1][p1];
+    // The threads that finish this level's rows fetch their w(I(S)) now, so
+    // that the strided gathers complete while phase A runs.
+    uint32_t wv[kRow];
+    const bool finisher = (int)threadIdx.x < rows;
+    const uint32_t s1f = finisher ? colex_unrank((unsigned long long)threadIdx.x, p1, kB1) : 0u;
+    if (finisher) {
+#pragma unroll
+      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)__ldg(&wI[((size_t)((s1f << kB2) | (uint32_t)i) << L) | T]);
+    }
     if (p1 >= 1) {
       // lanes per row chosen so that each lane runs at most 8 row pairs
       const int g = p1 > 3 ? p1 - 3 : 0;
@@ -564,12 +573,10 @@ k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned lon
       }
       __syncthreads();
     }
-    if ((int)threadIdx.x < rows) {
-      const uint32_t s1 = colex_unrank((unsigned long long)threadIdx.x, p1, kB1);
-      uint32_t z[kRow], c[kRow], wv[kRow];
+    if (finisher) {
+      const uint32_t s1 = s1f;
+      uint32_t z[kRow], c[kRow];
       load_row(z, zc + row_pos(0) * kRowStride);
-#pragma unroll
-      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)wI[((size_t)((s1 << kB2) | (uint32_t)i) << L) | T];
 #pragma unroll
       for (int s2 = 0; s2 < kRow; ++s2) {
         uint32_t key = 0xFFFFFFFFu;
