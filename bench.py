@@ -368,6 +368,79 @@ def run_ours(args):
     print(json.dumps(line), flush=True)
 
 
+def batch_groups(count: int, seed: int, n: int = 100_000, k: int = 8, m_lo: int = 8, m_hi: int = 13):
+    """Request groups shaped like the paper's exact-solve groups (Sec. 7: at
+    most 13 requests, k = 8 retrieved passages): each group draws its requests
+    from one of 64 topical pools of 60 passages (80 %) or a uniform tail."""
+    rng = np.random.default_rng(seed)
+    mu = math.log(150.0) - 0.18
+    weights = np.clip(np.rint(rng.lognormal(mu, 0.6, size=n)), 32, 512).astype(np.int64)
+    pools = rng.choice(n, size=(64, 60), replace=False)
+    groups = []
+    for _ in range(count):
+        m = int(rng.integers(m_lo, m_hi + 1))
+        pool = pools[int(rng.integers(64))]
+        reqs = []
+        for _ in range(m):
+            chosen = set()
+            while len(chosen) < k:
+                chosen.add(int(pool[int(rng.integers(60))]) if rng.random() < 0.8 else int(rng.integers(n)))
+            reqs.append(sorted(chosen))
+        groups.append(reqs)
+    return weights, groups
+
+
+def run_batch(args):
+    """Batched small-instance solves (mpt_batch_*): instances and splits per second."""
+    import torch
+
+    from paper_2609_13692_gb300 import build as B
+    from paper_2609_13692_gb300 import mpt
+
+    torch.cuda.set_device(0)
+    if not B.LIB.exists():
+        B.build()
+    weights, groups = batch_groups(args.batch_size, seed=0)
+    ir, ro, ch = mpt.pack_batch(groups)
+    ms = np.diff(ir)
+    splits = int(sum((3 ** int(m) + 1) // 2 - 2 ** int(m) for m in ms))
+    b = mpt.mpt_batch_create(weights, ir, ro, ch)
+    ws = torch.empty(mpt.mpt_batch_workspace_bytes(b), dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        mpt.mpt_batch_solve(b, ws, stream.cuda_stream)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        mpt.mpt_batch_solve(b, ws, stream.cuda_stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms_step = e0.elapsed_time(e1) / args.steps
+    line = {"mode": "batch", "metric": "exact solves of request groups (m = 8..13, k = 8) per second",
+            "value": len(groups) / (ms_step / 1000.0), "unit": "instances/s", "splits_per_s": splits / (ms_step / 1000.0),
+            "ms_per_step": ms_step, "steps": args.steps, "warmup": args.warmup, "batch": len(groups),
+            "splits_per_step": splits, "note": "timed region includes the per-step input upload and result download"}
+    if not args.no_cpu_baseline:
+        import oracle
+
+        sample = groups[:200]
+        t0 = time.perf_counter()
+        for reqs in sample:
+            oracle.solve(weights, _pack(reqs, weights.shape[0]))
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": len(sample) / dt, "unit": "instances/s", "cores": oracle.max_threads(),
+                                "kind": "oracle", "sample": f"first {len(sample)} groups, one oracle solve each"}
+    print(json.dumps(line), flush=True)
+
+
+def _pack(reqs, n):
+    from paper_2609_13692_gb300 import instances
+
+    return instances.pack_requests(reqs, n)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -378,7 +451,13 @@ def main():
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", choices=["solve", "batch"], default="solve",
+                    help="solve: the m = 28 exact solve (default); batch: many small request groups")
+    ap.add_argument("--batch-size", type=int, default=20000)
     args = ap.parse_args()
+    if args.mode == "batch":
+        run_batch(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -145,6 +145,57 @@ typedef struct mpt_profile {
 mpt_status mpt_set_profiling(mpt_ctx* ctx, int32_t on);
 mpt_status mpt_get_profile(const mpt_ctx* ctx, mpt_profile* out);
 
+/* ---------------------------------------------------------------------------
+ * Batched exact solves of many small instances (the paper's own use of the
+ * recurrence: request groups of at most 13 requests, Sec. 6.2 and Sec. 7).
+ * Every instance shares one chunk universe and weight array; instance b owns
+ * requests inst_requests[b] .. inst_requests[b+1]-1, request r the chunk ids
+ * chunk_ids[req_offsets[r] .. req_offsets[r+1]).  One CUDA block solves one
+ * instance with all of its tables in shared memory; results follow the same
+ * conventions as mpt_solve / mpt_layout for each instance on its own (request
+ * bit i = the instance's i-th request).
+ * ------------------------------------------------------------------------- */
+typedef struct mpt_batch mpt_batch;
+
+/* Validate and copy a batch (host arrays; caller keeps ownership).
+ *   weights: int64[n_chunks] (>= 1); inst_requests: int64[batch+1], starting at
+ *   0; req_offsets: int64[inst_requests[batch]+1], starting at 0;
+ *   chunk_ids: int64[req_offsets[last]] in [0, n_chunks), no repeat inside a
+ *   request.
+ * Limits per instance: 1 <= m <= 13 and at most 2048 chunk occurrences
+ * (MPT_ERR_TOO_LARGE beyond), sum_i w(R_i) < 2^31 (MPT_ERR_OVERFLOW).
+ * Errors: INVALID_ARG, TOO_LARGE, OVERFLOW, OUT_OF_MEMORY.  No CUDA call. */
+mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t batch, const int64_t* inst_requests,
+                            const int64_t* req_offsets, const int64_t* chunk_ids, mpt_batch** out);
+
+/* Device workspace bytes of mpt_batch_solve: input copies, per-instance
+ * F int64 / split uint32 tables (sum over instances of 2^m entries), OPT,
+ * permutations and DFS orders. */
+mpt_status mpt_batch_workspace_bytes(const mpt_batch* b, size_t* bytes);
+
+/* Solve every instance (Sec. 3.1 recurrence and Thm 1 layout per instance).
+ * d_workspace as in mpt_solve (NULL: the library allocates and keeps one);
+ * all work on `stream`, synchronised before return.  Errors: INVALID_ARG,
+ * WORKSPACE_TOO_SMALL, OUT_OF_MEMORY, CUDA, INTERNAL. */
+mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_bytes, void* stream);
+
+/* Results of the last solve, host outputs (any may be NULL):
+ *   opt: int64[batch];
+ *   perm_chunks: int64[req_offsets[last]], each request's chunks in layout
+ *     order, in the request's own slot range of the input CSR;
+ *   dfs_order: int32[inst_requests[batch]], per instance the local request
+ *     indices (0..m-1) from left to right (Thm 7 serving order).
+ * Errors: INVALID_ARG, NOT_SOLVED. */
+mpt_status mpt_batch_results(const mpt_batch* b, int64_t* opt, int64_t* perm_chunks, int32_t* dfs_order);
+
+/* Device tables of the last solve: instance b's F and split (indexed by its
+ * local subset masks) start at table_offsets[b] (host int64[batch+1]).
+ * Valid until the next solve or destroy.  Errors: INVALID_ARG, NOT_SOLVED. */
+mpt_status mpt_batch_tables(const mpt_batch* b, const int64_t** d_F, const uint32_t** d_split,
+                            int64_t* table_offsets);
+
+void mpt_batch_destroy(mpt_batch* b);
+
 /* Exact solve that allocates nothing, for callers that cannot allocate device
  * memory: code running in a serving process whose device memory is reserved
  * up front by its own pool allocator, or code that must not call cudaMalloc /

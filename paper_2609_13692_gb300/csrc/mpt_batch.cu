@@ -1,0 +1,235 @@
+// C ABI of the batched small-instance solver (include/mpt.h, mpt_batch_*):
+// argument checks, workspace carve-up and the one launch of k_batch_solve.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/mpt.h"
+#include "mpt_internal.cuh"
+
+namespace mpt {
+size_t batch_smem_bytes(int max_m, int occ_cap);
+cudaError_t launch_batch(int batch, int max_m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
+                         const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off, int64_t* opt,
+                         int64_t* F, uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status,
+                         cudaStream_t stream);
+}  // namespace mpt
+
+struct mpt_batch {
+  int32_t batch = 0;
+  int64_t n = 0, requests = 0, occurrences = 0, table_entries = 0;
+  int max_m = 0, occ_cap = 1;
+  std::vector<int64_t> w, inst_req, req_off, chunks, tab_off;
+  // results of the last solve
+  bool solved = false;
+  std::vector<int64_t> opt, perm;
+  std::vector<int32_t> dfs, status;
+  const int64_t* d_F = nullptr;
+  const uint32_t* d_split = nullptr;
+  void* own_ws = nullptr;
+  size_t own_bytes = 0;
+};
+
+namespace {
+
+constexpr int kBatchMaxM = 13;
+constexpr int kBatchMaxOcc = 2048;
+
+struct BatchCarve {
+  int64_t *weights, *inst_req, *req_off, *chunks, *tab_off, *opt, *F, *perm;
+  uint32_t* split;
+  int32_t *dfs, *status;
+};
+
+size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> char* {
+    const size_t o = off;
+    off += (bytes + 255) & ~(size_t)255;
+    return base ? base + o : nullptr;
+  };
+  c->weights = reinterpret_cast<int64_t*>(take((size_t)b->n * 8));
+  c->inst_req = reinterpret_cast<int64_t*>(take(((size_t)b->batch + 1) * 8));
+  c->req_off = reinterpret_cast<int64_t*>(take(((size_t)b->requests + 1) * 8));
+  c->chunks = reinterpret_cast<int64_t*>(take((size_t)std::max<int64_t>(b->occurrences, 1) * 8));
+  c->tab_off = reinterpret_cast<int64_t*>(take(((size_t)b->batch + 1) * 8));
+  c->opt = reinterpret_cast<int64_t*>(take((size_t)b->batch * 8));
+  c->F = reinterpret_cast<int64_t*>(take((size_t)b->table_entries * 8));
+  c->split = reinterpret_cast<uint32_t*>(take((size_t)b->table_entries * 4));
+  c->perm = reinterpret_cast<int64_t*>(take((size_t)std::max<int64_t>(b->occurrences, 1) * 8));
+  c->dfs = reinterpret_cast<int32_t*>(take((size_t)b->requests * 4));
+  c->status = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
+  return off;
+}
+
+}  // namespace
+
+extern "C" {
+
+mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t batch, const int64_t* inst_requests,
+                            const int64_t* req_offsets, const int64_t* chunk_ids, mpt_batch** out) {
+  if (!weights || !inst_requests || !req_offsets || !out || n_chunks < 1 || n_chunks > INT32_MAX || batch < 1)
+    return MPT_ERR_INVALID_ARG;
+  if (inst_requests[0] != 0) return MPT_ERR_INVALID_ARG;
+  for (int32_t b = 0; b < batch; ++b) {
+    const int64_t m = inst_requests[b + 1] - inst_requests[b];
+    if (m < 1) return MPT_ERR_INVALID_ARG;
+    if (m > kBatchMaxM) return MPT_ERR_TOO_LARGE;
+  }
+  const int64_t R = inst_requests[batch];
+  if (req_offsets[0] != 0) return MPT_ERR_INVALID_ARG;
+  for (int64_t r = 0; r < R; ++r)
+    if (req_offsets[r + 1] < req_offsets[r]) return MPT_ERR_INVALID_ARG;
+  const int64_t occ_total = req_offsets[R];
+  if (occ_total > 0 && !chunk_ids) return MPT_ERR_INVALID_ARG;
+  for (int64_t x = 0; x < n_chunks; ++x)
+    if (weights[x] <= 0) return MPT_ERR_INVALID_ARG;
+  mpt_batch* c = new (std::nothrow) mpt_batch();
+  if (!c) return MPT_ERR_OUT_OF_MEMORY;
+  try {
+    c->tab_off.resize((size_t)batch + 1);
+    int64_t tab = 0;
+    std::vector<int64_t> ids;
+    for (int32_t b = 0; b < batch; ++b) {
+      const int64_t r0 = inst_requests[b], r1 = inst_requests[b + 1];
+      const int m = (int)(r1 - r0);
+      const int64_t occ = req_offsets[r1] - req_offsets[r0];
+      if (occ > kBatchMaxOcc) {
+        delete c;
+        return MPT_ERR_TOO_LARGE;
+      }
+      int64_t sum = 0;
+      for (int64_t r = r0; r < r1; ++r) {
+        ids.assign(chunk_ids + req_offsets[r], chunk_ids + req_offsets[r + 1]);
+        std::sort(ids.begin(), ids.end());
+        for (size_t j = 0; j < ids.size(); ++j) {
+          if (ids[j] < 0 || ids[j] >= n_chunks || (j > 0 && ids[j] == ids[j - 1])) {
+            delete c;
+            return MPT_ERR_INVALID_ARG;
+          }
+          sum += weights[ids[j]];
+          if (sum >= ((int64_t)1 << 31)) {
+            delete c;
+            return MPT_ERR_OVERFLOW;
+          }
+        }
+      }
+      c->tab_off[(size_t)b] = tab;
+      tab += (int64_t)1 << m;
+      c->max_m = std::max(c->max_m, m);
+      while (c->occ_cap < occ) c->occ_cap <<= 1;
+    }
+    c->tab_off[(size_t)batch] = tab;
+    c->table_entries = tab;
+    c->w.assign(weights, weights + n_chunks);
+    c->inst_req.assign(inst_requests, inst_requests + batch + 1);
+    c->req_off.assign(req_offsets, req_offsets + R + 1);
+    if (occ_total) c->chunks.assign(chunk_ids, chunk_ids + occ_total);
+  } catch (...) {
+    delete c;
+    return MPT_ERR_OUT_OF_MEMORY;
+  }
+  c->batch = batch;
+  c->n = n_chunks;
+  c->requests = R;
+  c->occurrences = occ_total;
+  *out = c;
+  return MPT_OK;
+}
+
+mpt_status mpt_batch_workspace_bytes(const mpt_batch* b, size_t* bytes) {
+  if (!b || !bytes) return MPT_ERR_INVALID_ARG;
+  BatchCarve c{};
+  *bytes = carve(b, nullptr, &c);
+  return MPT_OK;
+}
+
+mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_bytes, void* stream_ptr) {
+  if (!b) return MPT_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
+  b->solved = false;
+  BatchCarve c{};
+  const size_t need = carve(b, nullptr, &c);
+  char* base = nullptr;
+  if (d_workspace) {
+    if (workspace_bytes < need) return MPT_ERR_WORKSPACE_TOO_SMALL;
+    if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return MPT_ERR_INVALID_ARG;
+    base = static_cast<char*>(d_workspace);
+  } else {
+    if (b->own_bytes < need) {
+      if (b->own_ws) cudaFree(b->own_ws);
+      b->own_ws = nullptr;
+      b->own_bytes = 0;
+      if (cudaMalloc(&b->own_ws, need) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+      b->own_bytes = need;
+    }
+    base = static_cast<char*>(b->own_ws);
+  }
+  carve(b, base, &c);
+  const size_t B = (size_t)b->batch;
+  try {
+    b->opt.resize(B);
+    b->status.resize(B);
+    b->perm.resize((size_t)b->occurrences);
+    b->dfs.resize((size_t)b->requests);
+  } catch (...) {
+    return MPT_ERR_OUT_OF_MEMORY;
+  }
+  cudaError_t e = cudaSuccess;
+  auto h2d = [&](void* d, const void* h, size_t bytes) {
+    if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(d, h, bytes, cudaMemcpyHostToDevice, stream);
+  };
+  auto d2h = [&](void* h, const void* d, size_t bytes) {
+    if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(h, d, bytes, cudaMemcpyDeviceToHost, stream);
+  };
+  h2d(c.weights, b->w.data(), (size_t)b->n * 8);
+  h2d(c.inst_req, b->inst_req.data(), (B + 1) * 8);
+  h2d(c.req_off, b->req_off.data(), ((size_t)b->requests + 1) * 8);
+  h2d(c.chunks, b->chunks.data(), (size_t)b->occurrences * 8);
+  h2d(c.tab_off, b->tab_off.data(), (B + 1) * 8);
+  if (e == cudaSuccess)
+    e = mpt::launch_batch(b->batch, b->max_m, b->occ_cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off, c.opt,
+                          c.F, c.split, c.perm, c.dfs, c.status, stream);
+  d2h(b->opt.data(), c.opt, B * 8);
+  d2h(b->status.data(), c.status, B * 4);
+  d2h(b->perm.data(), c.perm, (size_t)b->occurrences * 8);
+  d2h(b->dfs.data(), c.dfs, (size_t)b->requests * 4);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return e == cudaErrorMemoryAllocation ? MPT_ERR_OUT_OF_MEMORY : MPT_ERR_CUDA;
+  for (size_t i = 0; i < B; ++i)
+    if (b->status[i] != 0) return MPT_ERR_INTERNAL;
+  b->d_F = c.F;
+  b->d_split = c.split;
+  b->solved = true;
+  return MPT_OK;
+}
+
+mpt_status mpt_batch_results(const mpt_batch* b, int64_t* opt, int64_t* perm_chunks, int32_t* dfs_order) {
+  if (!b) return MPT_ERR_INVALID_ARG;
+  if (!b->solved) return MPT_ERR_NOT_SOLVED;
+  if (opt) std::memcpy(opt, b->opt.data(), b->opt.size() * 8);
+  if (perm_chunks && !b->perm.empty()) std::memcpy(perm_chunks, b->perm.data(), b->perm.size() * 8);
+  if (dfs_order && !b->dfs.empty()) std::memcpy(dfs_order, b->dfs.data(), b->dfs.size() * 4);
+  return MPT_OK;
+}
+
+mpt_status mpt_batch_tables(const mpt_batch* b, const int64_t** d_F, const uint32_t** d_split,
+                            int64_t* table_offsets) {
+  if (!b) return MPT_ERR_INVALID_ARG;
+  if (!b->solved) return MPT_ERR_NOT_SOLVED;
+  if (d_F) *d_F = b->d_F;
+  if (d_split) *d_split = b->d_split;
+  if (table_offsets) std::memcpy(table_offsets, b->tab_off.data(), b->tab_off.size() * 8);
+  return MPT_OK;
+}
+
+void mpt_batch_destroy(mpt_batch* b) {
+  if (!b) return;
+  if (b->own_ws) cudaFree(b->own_ws);
+  delete b;
+}
+
+}  // extern "C"

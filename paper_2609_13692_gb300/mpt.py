@@ -39,7 +39,8 @@ STATUS_NAMES = {
 EXPORTED = [
     "mpt_create", "mpt_workspace_bytes", "mpt_set_dp_mode", "mpt_solve", "mpt_tables", "mpt_layout_size",
     "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
-    "mpt_last_error", "mpt_solve_noalloc",
+    "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
+    "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy",
 ]
 
 
@@ -108,6 +109,12 @@ def load() -> ctypes.CDLL:
         "mpt_status_string": ([ctypes.c_int], ctypes.c_char_p),
         "mpt_last_error": ([vp], ctypes.c_char_p),
         "mpt_solve_noalloc": ([vp, i64, vp, i32, vp, vp, vp, vp, vp], ctypes.c_int),
+        "mpt_batch_create": ([i64p, i64, i32, i64p, i64p, i64p, ctypes.POINTER(vp)], ctypes.c_int),
+        "mpt_batch_workspace_bytes": ([vp, ctypes.POINTER(sz)], ctypes.c_int),
+        "mpt_batch_solve": ([vp, vp, sz, vp], ctypes.c_int),
+        "mpt_batch_results": ([vp, i64p, i64p, i32p], ctypes.c_int),
+        "mpt_batch_tables": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp), i64p], ctypes.c_int),
+        "mpt_batch_destroy": ([vp], None),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -304,3 +311,124 @@ def solve(weights, bits, mode: str = "auto", workspace=None, stream: Optional[in
     opt = mpt_solve(ctx, workspace, stream)
     offs, chunks, dfs = mpt_layout(ctx)
     return Result(opt, offs, chunks, dfs, ctx)
+
+
+# ---------------------------------------------------------------------------
+# Batched small instances (mpt_batch_*)
+# ---------------------------------------------------------------------------
+
+class Batch:
+    """Owns one ``mpt_batch`` (many instances of at most 13 requests)."""
+
+    def __init__(self, handle: int, batch: int, inst_requests: np.ndarray, req_offsets: np.ndarray):
+        self.handle = ctypes.c_void_p(handle)
+        self.batch = batch
+        self.inst_requests = inst_requests
+        self.req_offsets = req_offsets
+        self.workspace = None
+
+    def __del__(self):
+        try:
+            mpt_batch_destroy(self)
+        except Exception:
+            pass
+
+
+def mpt_batch_create(weights, inst_requests, req_offsets, chunk_ids) -> Batch:
+    lib = load()
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    ir = np.ascontiguousarray(inst_requests, dtype=np.int64)
+    ro = np.ascontiguousarray(req_offsets, dtype=np.int64)
+    ch = np.ascontiguousarray(chunk_ids, dtype=np.int64)
+    if ch.size == 0:
+        ch = np.zeros(1, dtype=np.int64)
+    h = ctypes.c_void_p()
+    _check(lib.mpt_batch_create(_ptr(w, ctypes.c_int64), int(w.shape[0]), int(ir.shape[0]) - 1,
+                                _ptr(ir, ctypes.c_int64), _ptr(ro, ctypes.c_int64), _ptr(ch, ctypes.c_int64),
+                                ctypes.byref(h)), "mpt_batch_create")
+    return Batch(h.value, int(ir.shape[0]) - 1, ir, ro)
+
+
+def mpt_batch_workspace_bytes(b: Batch) -> int:
+    out = ctypes.c_size_t()
+    _check(load().mpt_batch_workspace_bytes(b.handle, ctypes.byref(out)), "mpt_batch_workspace_bytes")
+    return int(out.value)
+
+
+def mpt_batch_solve(b: Batch, workspace=None, stream: Optional[int] = None) -> None:
+    import torch
+
+    need = mpt_batch_workspace_bytes(b)
+    if workspace is None:
+        if b.workspace is None or b.workspace.numel() < need:
+            b.workspace = torch.empty(need, dtype=torch.uint8, device="cuda")
+        workspace = b.workspace
+    s = _default_stream_ptr() if stream is None else int(stream)
+    _check(load().mpt_batch_solve(b.handle, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                  ctypes.c_void_p(s)), "mpt_batch_solve")
+    b._solved_ws = workspace
+
+
+def mpt_batch_results(b: Batch):
+    """(opt int64[batch], perm_chunks int64[occurrences], dfs_order int32[requests])."""
+    opt = np.zeros(b.batch, dtype=np.int64)
+    perm = np.zeros(max(1, int(b.req_offsets[-1])), dtype=np.int64)
+    dfs = np.zeros(max(1, int(b.inst_requests[-1])), dtype=np.int32)
+    _check(load().mpt_batch_results(b.handle, _ptr(opt, ctypes.c_int64), _ptr(perm, ctypes.c_int64),
+                                    _ptr(dfs, ctypes.c_int32)), "mpt_batch_results")
+    return opt, perm[:int(b.req_offsets[-1])], dfs[:int(b.inst_requests[-1])]
+
+
+def mpt_batch_tables(b: Batch):
+    """Device views of all instances' F (int64) and split (int32) tables and
+    the host offsets (instance i's tables start at offsets[i])."""
+    import torch
+
+    pF, pS = ctypes.c_void_p(), ctypes.c_void_p()
+    offs = np.zeros(b.batch + 1, dtype=np.int64)
+    _check(load().mpt_batch_tables(b.handle, ctypes.byref(pF), ctypes.byref(pS), _ptr(offs, ctypes.c_int64)),
+           "mpt_batch_tables")
+    ws = b._solved_ws
+    total = int(offs[-1])
+
+    def view(ptr, nbytes, dtype):
+        off = ptr.value - ws.data_ptr()
+        return ws[off:off + nbytes].view(dtype)
+
+    return view(pF, 8 * total, torch.int64), view(pS, 4 * total, torch.int32), offs
+
+
+def mpt_batch_destroy(b: Batch) -> None:
+    if b.handle and b.handle.value:
+        load().mpt_batch_destroy(b.handle)
+        b.handle = ctypes.c_void_p()
+
+
+def pack_batch(instances):
+    """CSR arrays (inst_requests, req_offsets, chunk_ids) from a list of
+    instances, each a list of requests, each a list of chunk ids."""
+    inst = [0]
+    offs = [0]
+    ids = []
+    for requests in instances:
+        for r in requests:
+            ids.extend(int(x) for x in r)
+            offs.append(len(ids))
+        inst.append(len(offs) - 1)
+    return (np.asarray(inst, dtype=np.int64), np.asarray(offs, dtype=np.int64),
+            np.asarray(ids, dtype=np.int64))
+
+
+def solve_batch(weights, instances, workspace=None, stream: Optional[int] = None):
+    """Exact solves of many small instances.  Returns (opt per instance,
+    per-instance list of per-request chunk orders, per-instance DFS order, batch)."""
+    ir, ro, ch = pack_batch(instances)
+    b = mpt_batch_create(weights, ir, ro, ch)
+    mpt_batch_solve(b, workspace, stream)
+    opt, perm, dfs = mpt_batch_results(b)
+    perms, orders = [], []
+    for i in range(b.batch):
+        r0, r1 = int(ir[i]), int(ir[i + 1])
+        perms.append([perm[ro[r]:ro[r + 1]].tolist() for r in range(r0, r1)])
+        orders.append(dfs[r0:r1].tolist())
+    return opt, perms, orders, b

@@ -95,3 +95,25 @@ def test_status_strings(mpt):
     lib = mpt.load()
     for code in range(10):
         assert lib.mpt_status_string(code)
+
+
+def _batch_status(mpt, weights, instances):
+    try:
+        b = mpt.mpt_batch_create(weights, *mpt.pack_batch(instances))
+        mpt.mpt_batch_destroy(b)
+        return 0
+    except mpt.MPTError as e:
+        return e.status
+
+
+def test_batch_create_validation(mpt):
+    w = np.ones(50, dtype=np.int64)
+    assert _batch_status(mpt, w, [[[1, 2], [3]], [[4]]]) == 0
+    assert _batch_status(mpt, w, [[[i] for i in range(14)]]) == 2           # m > 13
+    assert _batch_status(mpt, w, [[[1, 1]]]) == 1                           # repeated chunk in a request
+    assert _batch_status(mpt, w, [[[50]]]) == 1                             # chunk id >= n
+    assert _batch_status(mpt, w, [[]]) == 1                                 # an instance with no request
+    heavy = np.full(50, 1 << 30, dtype=np.int64)
+    assert _batch_status(mpt, heavy, [[[0, 1]]]) == 3                       # sum of w(R_i) >= 2^31
+    big = [[list(range(0, 2049))]]
+    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), big) == 2      # > 2048 occurrences

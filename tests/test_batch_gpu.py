@@ -1,0 +1,94 @@
+"""Batched small-instance solver (mpt_batch_*) against the oracle, per instance.
+
+Every instance of a batch must match the oracle bit for bit: OPT, every F(S)
+and split(S) of its own 2^m table, every request's chunk order and the DFS
+order.  The batch mixes sizes m = 1..13, empty and repeated requests, and
+RAG-like groups drawn from topical pools (the shape of the paper's request
+groups, Sec. 7).
+"""
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_13692_gb300 import instances as I
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def mpt():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_13692_gb300 import build as B
+
+    B.build()
+    O.build()
+    from paper_2609_13692_gb300 import mpt as M
+
+    M.load()
+    return M
+
+
+def rag_batch(count, n, seed, m_range=(1, 13), k_range=(0, 10), pool_size=40):
+    rng = np.random.default_rng(seed)
+    weights = rng.integers(1, 501, size=n, dtype=np.int64)
+    pools = [rng.choice(n, size=pool_size, replace=False) for _ in range(16)]
+    batch = []
+    for _ in range(count):
+        m = int(rng.integers(m_range[0], m_range[1] + 1))
+        pool = pools[int(rng.integers(len(pools)))]
+        reqs = []
+        for _ in range(m):
+            k = int(rng.integers(k_range[0], k_range[1] + 1))
+            src = pool if rng.random() < 0.8 else np.arange(n)
+            reqs.append(sorted(set(int(x) for x in rng.choice(src, size=k, replace=False))))
+        batch.append(reqs)
+    return weights, batch
+
+
+def check_batch(mpt, weights, batch):
+    opt, perms, orders, b = mpt.solve_batch(weights, batch)
+    F_all, S_all, offs = mpt.mpt_batch_tables(b)
+    F_all = F_all.cpu().numpy()
+    S_all = S_all.cpu().numpy().view(np.uint32)
+    n = int(weights.shape[0])
+    for i, reqs in enumerate(batch):
+        bits = I.pack_requests(reqs, n)
+        o_opt, oF, owI, osplit = O.solve(weights, bits)
+        assert opt[i] == o_opt, (i, opt[i], o_opt)
+        lo, hi = int(offs[i]), int(offs[i + 1])
+        assert np.array_equal(F_all[lo:hi], oF), i
+        assert np.array_equal(S_all[lo:hi], osplit), i
+        o_perms, o_dfs = O.layout(weights, bits, osplit)
+        assert perms[i] == o_perms, i
+        assert orders[i] == o_dfs, i
+
+
+def test_batch_rag_groups(mpt):
+    weights, batch = rag_batch(300, 3000, seed=1)
+    check_batch(mpt, weights, batch)
+
+
+def test_batch_edge_cases(mpt):
+    w = np.arange(1, 21, dtype=np.int64)
+    batch = [
+        [[3]],                                   # m = 1
+        [[], [1, 2], []],                        # empty requests
+        [[1, 2, 3]] * 13,                        # identical requests, m = 13
+        [[i] for i in range(13)],                # disjoint singletons
+        [[x for x in range(13) if x != i] for i in range(13)],  # leave-one-out L_13
+        [[0, 19], [19], [0]],
+    ]
+    check_batch(mpt, w, batch)
+    opt, perms, orders, b = mpt.solve_batch(np.ones(13, dtype=np.int64),
+                                            [[[x for x in range(13) if x != i] for i in range(13)]])
+    assert opt[0] == O.loo_free(13)
+
+
+def test_batch_large_requests(mpt):
+    """Requests of up to 150 chunks (near the 2048-occurrence limit at m = 13)."""
+    weights, batch = rag_batch(40, 20000, seed=2, m_range=(10, 13), k_range=(100, 150), pool_size=400)
+    check_batch(mpt, weights, batch)
