@@ -196,6 +196,32 @@ mpt_status mpt_batch_tables(const mpt_batch* b, const int64_t** d_F, const uint3
 
 void mpt_batch_destroy(mpt_batch* b);
 
+/* Agglomerative common-intersection hierarchy (Sec. 6.2; H_g of Thm 6) and
+ * the spanning-tree lower bound (Sec. 6.3), for request counts far beyond the
+ * exact recurrence.  Every request starts as a cluster with signature R_i;
+ * the two active clusters with the heaviest common signature merge, the
+ * merged signature being that intersection.  A cluster lives in the slot of
+ * its smallest request; ties go to the smallest slot pair (a, b), a < b, and
+ * the merged cluster keeps slot a.  The layout walks the hierarchy top-down
+ * as in the Thm 1 proof (children of a merge: slot a's subtree first).
+ *   weights: host int64[n_chunks] (>= 1); req_offsets: host int64[m+1] from 0;
+ *   chunk_ids: host int64[req_offsets[m]], at most 128 per request, no repeat
+ *   inside a request, each request's weight < 2^32.  1 <= m <= 16384.
+ *   stream: a cudaStream_t (NULL = legacy default), synchronised before return.
+ * Outputs (host, any may be NULL): cost = sum_i w(R_i) - savings (the
+ * hierarchy's Thm 1 cost; the trie of the layout costs at most this),
+ * savings = sum of merge values, lower_bound = sum_i w(R_i) - max spanning
+ * tree of w(R_i cap R_j), merges int32[2(m-1)] (slot pairs a, b in merge
+ * order), merge_values int64[m-1], perm_chunks int64[req_offsets[m]] (each
+ * request's chunks in layout order, in its own CSR range), dfs_order int32[m].
+ * Device memory (m^2 * 4 bytes for the pair weights, plus small buffers) is
+ * allocated and freed by the call.
+ * Errors: INVALID_ARG, TOO_LARGE, OVERFLOW, OUT_OF_MEMORY, CUDA. */
+mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* req_offsets,
+                      const int64_t* chunk_ids, void* stream, int64_t* cost, int64_t* savings,
+                      int64_t* lower_bound, int32_t* merges, int64_t* merge_values, int64_t* perm_chunks,
+                      int32_t* dfs_order);
+
 /* Exact solve that allocates nothing, for callers that cannot allocate device
  * memory: code running in a serving process whose device memory is reserved
  * up front by its own pool allocator, or code that must not call cudaMalloc /

@@ -24,6 +24,9 @@ Everything here follows "Prefix Sharing Is a Sorting Problem" (arxiv
 * ``spanning_tree_bound``: the lower bound of Sec. 6.3.
 * ``radix_cache_cost``: a radix cache with LRU leaf eviction (Sec. 8, Thm 7).
 * ``loo_free`` / ``loo_glob``: the closed forms of Thm 5.
+* ``greedy``: the agglomerative common-intersection hierarchy of Sec. 6.2
+  (Thm 6's H_g), with its layout and savings.
+* ``trie_cost_sorted``: eq. (1) for many strings via lexicographic sorting.
 
 Readings where the paper is silent are stated in ``oracle.c``'s header.
 """
@@ -445,3 +448,95 @@ def loo_free(n: int) -> int:
 def loo_glob(n: int) -> int:
     """Thm 5: OPT_glob(L_n) = (n-1)(n+2)/2."""
     return (n - 1) * (n + 2) // 2
+
+
+def greedy(weights, bits):
+    """Agglomerative common-intersection hierarchy (Sec. 6.2; H_g of Thm 6).
+
+    Every request starts as a cluster whose signature is R_i.  Repeatedly the
+    two active clusters with the heaviest common signature w(I(A) cap I(B))
+    are merged, the merged signature being that intersection.  A cluster is
+    held in the slot of its smallest request; ties go to the smallest slot
+    pair (a, b), a < b (a reading: the paper leaves ties open).  The merged
+    cluster keeps slot a.
+
+    Returns dict(merges=[(a, b, value)], savings, cost = sum_i w(R_i) - savings,
+    perms, dfs): the layout walks the hierarchy top-down as in Thm 1 (at each
+    node the chunks of I(v) minus I(parent(v)), increasing id), children of a
+    merge ordered (slot a, slot b), dfs the leaves from left to right."""
+    R = request_sets(weights, bits)
+    w = np.asarray(weights)
+    m = len(R)
+    wt = lambda s: int(sum(int(w[x]) for x in s))
+    sig = [set(r) for r in R]
+    node = list(range(m))  # current tree node of each slot
+    children = {}
+    node_sig = {i: frozenset(R[i]) for i in range(m)}
+    active = [True] * m
+    merges = []
+    for t in range(m - 1):
+        best = None
+        for a in range(m):
+            if not active[a]:
+                continue
+            for b in range(a + 1, m):
+                if not active[b]:
+                    continue
+                v = wt(sig[a] & sig[b])
+                if best is None or v > best[2]:
+                    best = (a, b, v)
+        a, b, v = best
+        merges.append(best)
+        sig[a] = sig[a] & sig[b]
+        active[b] = False
+        new = m + t
+        children[new] = (node[a], node[b])
+        node_sig[new] = frozenset(sig[a])
+        node[a] = new
+    savings = sum(v for _, _, v in merges)
+    total = sum(wt(r) for r in R)
+    perms: list[list[int]] = [[] for _ in range(m)]
+    dfs: list[int] = []
+
+    def walk(v, parent_sig):
+        emit = sorted(node_sig[v] - parent_sig)
+        leaves = []
+        if v < m:
+            perms[v].extend(emit)
+            dfs.append(v)
+            return [v]
+        left, right = children[v]
+        for i in _leaves(left, children, m) + _leaves(right, children, m):
+            perms[i].extend(emit)
+        walk(left, node_sig[v])
+        walk(right, node_sig[v])
+        return leaves
+
+    if m > 0:
+        walk(node[0] if m > 1 else 0, frozenset())
+    return dict(merges=merges, savings=savings, cost=total - savings, perms=perms, dfs=dfs)
+
+
+def _leaves(v, children, m):
+    if v < m:
+        return [v]
+    l, r = children[v]
+    return _leaves(l, children, m) + _leaves(r, children, m)
+
+
+def trie_cost_sorted(weights, perms) -> int:
+    """Eq. (1) for many strings: sort them lexicographically; each string adds
+    the weight of its suffix after the longest common prefix with its
+    predecessor (each trie node is counted once, at the first string that
+    reaches it in sorted order)."""
+    w = np.asarray(weights)
+    seqs = sorted(tuple(int(x) for x in p) for p in perms)
+    cost = 0
+    prev: tuple = ()
+    for sq in seqs:
+        l = 0
+        while l < len(sq) and l < len(prev) and sq[l] == prev[l]:
+            l += 1
+        cost += int(sum(int(w[x]) for x in sq[l:]))
+        prev = sq
+    return cost

@@ -1,0 +1,422 @@
+// Agglomerative common-intersection hierarchy (Sec. 6.2; H_g of Thm 6) and
+// the spanning-tree lower bound (Sec. 6.3), for request counts far beyond the
+// exact recurrence (m up to 16384).
+//
+// Greedy: every request starts as a cluster with signature R_i; the two active
+// clusters with the heaviest common signature w(I(A) cap I(B)) merge, the
+// merged signature being that intersection.  A cluster lives in the slot of
+// its smallest request; ties go to the smallest slot pair (a, b), a < b, and
+// the merged cluster keeps slot a.  The layout walks the hierarchy as in the
+// Thm 1 proof.  Lower bound: sum_i w(R_i) - MaxSpanningTree(w(R_i cap R_j)).
+//
+// Kernels: k_pair_weights fills W[i][j] = w(R_i cap R_j) (sorted chunk lists,
+// merge-intersection); k_maxst runs Prim on W in one block; k_greedy_merge runs
+// all m - 1 merges in one block, keeping for every active slot its best
+// partner as a 64-bit key (weight, then the smallest slot pair) and rescanning
+// a row only when its best partner was merged; k_greedy_layout climbs each
+// (request, chunk) occurrence to the highest node whose signature still holds
+// the chunk, and ranks each request's chunks by (depth, chunk id).
+#include "../../include/mpt.h"
+#include "mpt_internal.cuh"
+
+#include <algorithm>
+#include <vector>
+
+namespace mpt {
+namespace {
+
+constexpr int kSigMax = 128;       // longest request accepted
+constexpr int kMaxGreedyM = 16384;  // slot ids fit in 14 bits
+constexpr int kGreedyThreads = 1024;
+
+__device__ __forceinline__ uint32_t sig_weight(const int32_t* a, int la, const int32_t* b, int lb,
+                                               const int64_t* __restrict__ w) {
+  uint32_t s = 0;
+  int i = 0, j = 0;
+  while (i < la && j < lb) {
+    const int32_t x = a[i], y = b[j];
+    if (x == y) {
+      s += (uint32_t)w[x];
+      ++i;
+      ++j;
+    } else if (x < y) {
+      ++i;
+    } else {
+      ++j;
+    }
+  }
+  return s;
+}
+
+// key of pair {d, e} with common weight v: larger is better (weight, then the
+// smaller slot pair)
+__device__ __forceinline__ unsigned long long pair_key(uint32_t d, uint32_t e, uint32_t v) {
+  const uint32_t a = min(d, e), b = max(d, e);
+  return ((unsigned long long)v << 28) | (unsigned long long)((1u << 28) - 1u - ((a << 14) | b));
+}
+__device__ __forceinline__ void key_pair(unsigned long long k, uint32_t* a, uint32_t* b) {
+  const uint32_t p = (1u << 28) - 1u - (uint32_t)(k & ((1u << 28) - 1u));
+  *a = p >> 14;
+  *b = p & ((1u << 14) - 1u);
+}
+
+__global__ void k_pair_weights(int m, const int32_t* __restrict__ sig, const int32_t* __restrict__ len,
+                               const int64_t* __restrict__ w, uint32_t* __restrict__ W) {
+  const int i = blockIdx.y;
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < m; j += gridDim.x * blockDim.x) {
+    if (j < i) continue;
+    const uint32_t v = (j == i) ? 0u : sig_weight(sig + (size_t)i * kSigMax, len[i], sig + (size_t)j * kSigMax, len[j], w);
+    W[(size_t)i * m + j] = v;
+    W[(size_t)j * m + i] = v;
+  }
+}
+
+// best partner of every slot: warp per row
+__global__ void k_row_best(int m, const uint32_t* __restrict__ W, unsigned long long* __restrict__ best) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int d = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; d < m; d += warps) {
+    unsigned long long b = 0;
+    for (int e = lane; e < m; e += 32)
+      if (e != d) b = max(b, pair_key((uint32_t)d, (uint32_t)e, W[(size_t)d * m + e]));
+    for (int off = 16; off > 0; off >>= 1) b = max(b, __shfl_xor_sync(0xFFFFFFFFu, b, off));
+    if (lane == 0) best[d] = b;
+  }
+}
+
+__device__ unsigned long long block_max_u64(unsigned long long v, unsigned long long* red) {
+  for (int off = 16; off > 0; off >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, off));
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    v = lane < (int)(blockDim.x >> 5) ? red[lane] : 0ull;
+    for (int off = 16; off > 0; off >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, off));
+    if (lane == 0) red[32] = v;
+  }
+  __syncthreads();
+  const unsigned long long r = red[32];
+  __syncthreads();
+  return r;
+}
+
+// Prim's maximum spanning tree on W (one block).  tree_key[v]: heaviest edge
+// from v into the tree so far.
+__global__ void __launch_bounds__(kGreedyThreads)
+k_maxst(int m, const uint32_t* __restrict__ W, uint32_t* __restrict__ tree_key, uint8_t* __restrict__ in_tree,
+        unsigned long long* __restrict__ out) {
+  __shared__ unsigned long long red[33];
+  for (int v = threadIdx.x; v < m; v += blockDim.x) {
+    tree_key[v] = W[v];  // row 0
+    in_tree[v] = v == 0;
+  }
+  __syncthreads();
+  unsigned long long total = 0;
+  for (int it = 1; it < m; ++it) {
+    unsigned long long cand = 0;
+    for (int v = threadIdx.x; v < m; v += blockDim.x)
+      if (!in_tree[v]) cand = max(cand, ((unsigned long long)tree_key[v] << 20) | (unsigned long long)((1u << 20) - 1u - v));
+    const unsigned long long b = block_max_u64(cand, red);
+    const int v0 = (int)((1u << 20) - 1u - (uint32_t)(b & ((1u << 20) - 1u)));
+    total += b >> 20;
+    if (threadIdx.x == 0) in_tree[v0] = 1;
+    __syncthreads();
+    for (int v = threadIdx.x; v < m; v += blockDim.x)
+      if (!in_tree[v]) tree_key[v] = max(tree_key[v], W[(size_t)v0 * m + v]);
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = total;
+}
+
+__device__ unsigned long long block_row_best(int m, int d, const uint32_t* __restrict__ W,
+                                             const uint8_t* __restrict__ active, unsigned long long* red) {
+  unsigned long long bb = 0;
+  for (int e = threadIdx.x; e < m; e += blockDim.x)
+    if (e != d && active[e]) bb = max(bb, pair_key((uint32_t)d, (uint32_t)e, W[(size_t)d * m + e]));
+  return block_max_u64(bb, red);
+}
+
+// All m - 1 merges (one block).  best[d] is an upper bound on row d's best
+// pair key: pair weights only decrease as clusters merge, so a key stays an
+// upper bound until its row is rescanned.  The largest bound is merged only
+// if it is still exact (both slots active, weight unchanged); otherwise its
+// rows are rescanned and the choice is repeated.  Every rescan makes a row
+// exact, so a step repeats at most m times (kept as a hard cap).
+__global__ void __launch_bounds__(kGreedyThreads)
+k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, int32_t* __restrict__ len,
+               uint32_t* __restrict__ W, unsigned long long* __restrict__ best, uint8_t* __restrict__ active,
+               int32_t* __restrict__ node, int32_t* __restrict__ merges, int64_t* __restrict__ values,
+               int32_t* __restrict__ children, int32_t* __restrict__ node_sig, int32_t* __restrict__ node_len,
+               int32_t* __restrict__ error) {
+  __shared__ unsigned long long red[33];
+  __shared__ int32_t s_new[kSigMax];
+  __shared__ int s_len;
+  for (int d = threadIdx.x; d < m; d += blockDim.x) {
+    active[d] = 1;
+    node[d] = d;
+  }
+  __syncthreads();
+  for (int t = 0; t < m - 1; ++t) {
+    uint32_t a = 0, b = 0, v = 0;
+    int tries = 0;
+    for (;;) {
+      unsigned long long c = 0;
+      for (int d = threadIdx.x; d < m; d += blockDim.x)
+        if (active[d]) c = max(c, best[d]);
+      const unsigned long long top = block_max_u64(c, red);
+      key_pair(top, &a, &b);
+      v = (uint32_t)(top >> 28);
+      if (active[a] && active[b] && W[(size_t)a * m + b] == v) break;
+      if (++tries > m + 1) {
+        if (threadIdx.x == 0) atomicOr(error, 1);
+        break;
+      }
+      if (active[a]) {
+        const unsigned long long r = block_row_best(m, (int)a, W, active, red);
+        if (threadIdx.x == 0) best[a] = r;
+      }
+      if (active[b]) {
+        const unsigned long long r = block_row_best(m, (int)b, W, active, red);
+        if (threadIdx.x == 0) best[b] = r;
+      }
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+      merges[2 * t] = (int32_t)a;
+      merges[2 * t + 1] = (int32_t)b;
+      values[t] = v;
+      children[2 * t] = node[a];
+      children[2 * t + 1] = node[b];
+      const int32_t* sa = sig + (size_t)a * kSigMax;
+      const int32_t* sb = sig + (size_t)b * kSigMax;
+      int i = 0, j = 0, n = 0;
+      while (i < len[a] && j < len[b]) {
+        if (sa[i] == sb[j]) {
+          s_new[n++] = sa[i];
+          ++i;
+          ++j;
+        } else if (sa[i] < sb[j]) {
+          ++i;
+        } else {
+          ++j;
+        }
+      }
+      s_len = n;
+    }
+    __syncthreads();
+    for (int q = threadIdx.x; q < s_len; q += blockDim.x) {
+      sig[(size_t)a * kSigMax + q] = s_new[q];
+      node_sig[(size_t)t * kSigMax + q] = s_new[q];
+    }
+    // new pair weights of the merged slot: zero wherever either old weight was
+    // zero (the merged signature is a subset of both)
+    for (int d = threadIdx.x; d < m; d += blockDim.x) {
+      if (!active[d] || d == (int)a || d == (int)b) continue;
+      const uint32_t wa = W[(size_t)a * m + d], wb = W[(size_t)b * m + d];
+      const uint32_t wv = (wa == 0 || wb == 0 || s_len == 0)
+                              ? 0u
+                              : sig_weight(s_new, s_len, sig + (size_t)d * kSigMax, len[d], w);
+      W[(size_t)a * m + d] = wv;
+      W[(size_t)d * m + a] = wv;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      len[a] = s_len;
+      node_len[t] = s_len;
+      node[a] = m + t;
+      active[b] = 0;
+    }
+    __syncthreads();
+    const unsigned long long r = block_row_best(m, (int)a, W, active, red);
+    if (threadIdx.x == 0) best[a] = r;
+    __syncthreads();
+  }
+}
+
+// Parent and depth of every tree node and the left-to-right leaf order (one thread).
+__global__ void k_greedy_tree(int m, const int32_t* __restrict__ children, int32_t* __restrict__ parent,
+                              int32_t* __restrict__ depth, int32_t* __restrict__ stack, int32_t* __restrict__ dfs) {
+  const int root = m == 1 ? 0 : 2 * m - 2;
+  parent[root] = -1;
+  depth[root] = 0;
+  for (int t = m - 2; t >= 0; --t) {
+    const int v = m + t;
+    for (int c = 0; c < 2; ++c) {
+      const int ch = children[2 * t + c];
+      parent[ch] = v;
+      depth[ch] = depth[v] + 1;
+    }
+  }
+  int sp = 0, nl = 0;
+  stack[sp++] = root;
+  while (sp > 0) {
+    const int v = stack[--sp];
+    if (v < m) {
+      dfs[nl++] = v;
+      continue;
+    }
+    const int t = v - m;
+    stack[sp++] = children[2 * t + 1];  // right after left
+    stack[sp++] = children[2 * t];
+  }
+}
+
+// Emission depth of every (request, chunk) occurrence: climb from the leaf
+// while the parent's signature still holds the chunk.
+__global__ void k_greedy_emit(int m, const int32_t* __restrict__ node_sig, const int32_t* __restrict__ node_len,
+                              const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
+                              const int32_t* __restrict__ parent, const int32_t* __restrict__ depth,
+                              unsigned long long* __restrict__ keys) {
+  const int64_t occ = req_off[m];
+  for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < occ; j += (int64_t)gridDim.x * blockDim.x) {
+    int lo = 0, hi = m - 1;  // request of occurrence j: the last i with req_off[i] <= j
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (req_off[mid] <= j) lo = mid; else hi = mid - 1;
+    }
+    const int32_t x = (int32_t)chunks[j];
+    int v = lo;
+    for (;;) {
+      const int p = parent[v];
+      if (p < 0) break;
+      const int t = p - m;
+      const int32_t* s = node_sig + (size_t)t * kSigMax;
+      const int n = node_len[t];
+      int a = 0, b = n;
+      while (a < b) {
+        const int mid = (a + b) >> 1;
+        if (s[mid] < x) a = mid + 1; else b = mid;
+      }
+      if (a < n && s[a] == x) v = p; else break;
+    }
+    keys[j] = ((unsigned long long)depth[v] << 32) | (unsigned long long)(uint32_t)x;
+  }
+}
+
+// Each request's chunks ranked by (emission depth, chunk id): warp per request.
+__global__ void k_greedy_rank(int m, const int64_t* __restrict__ req_off, const unsigned long long* __restrict__ keys,
+                              int64_t* __restrict__ perm) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < m; i += warps) {
+    const int64_t base = req_off[i];
+    const int len = (int)(req_off[i + 1] - base);
+    for (int q = lane; q < len; q += 32) {
+      const unsigned long long kq = keys[base + q];
+      int rank = 0;
+      for (int r = 0; r < len; ++r) rank += keys[base + r] < kq;
+      perm[base + rank] = (int64_t)(kq & 0xFFFFFFFFull);
+    }
+  }
+}
+
+}  // namespace
+}  // namespace mpt
+
+extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* req_offsets,
+                                 const int64_t* chunk_ids, void* stream_ptr, int64_t* cost, int64_t* savings,
+                                 int64_t* lower_bound, int32_t* merges, int64_t* merge_values, int64_t* perm_chunks,
+                                 int32_t* dfs_order) {
+  using namespace mpt;
+  if (!weights || !req_offsets || n_chunks < 1 || n_chunks > INT32_MAX || m < 1) return MPT_ERR_INVALID_ARG;
+  if (m > kMaxGreedyM) return MPT_ERR_TOO_LARGE;
+  if (req_offsets[0] != 0) return MPT_ERR_INVALID_ARG;
+  const int64_t occ = req_offsets[m];
+  if (occ > 0 && !chunk_ids) return MPT_ERR_INVALID_ARG;
+  for (int64_t x = 0; x < n_chunks; ++x)
+    if (weights[x] <= 0) return MPT_ERR_INVALID_ARG;
+  // sorted, de-duplicated-checked signatures; per-request weight < 2^32
+  std::vector<int32_t> sig((size_t)m * kSigMax, 0), len((size_t)m, 0);
+  int64_t total = 0;
+  for (int i = 0; i < m; ++i) {
+    const int64_t a = req_offsets[i], b = req_offsets[i + 1];
+    if (b < a) return MPT_ERR_INVALID_ARG;
+    if (b - a > kSigMax) return MPT_ERR_TOO_LARGE;
+    std::vector<int64_t> ids(chunk_ids + a, chunk_ids + b);
+    std::sort(ids.begin(), ids.end());
+    int64_t rw = 0;
+    for (size_t q = 0; q < ids.size(); ++q) {
+      if (ids[q] < 0 || ids[q] >= n_chunks || (q > 0 && ids[q] == ids[q - 1])) return MPT_ERR_INVALID_ARG;
+      sig[(size_t)i * kSigMax + q] = (int32_t)ids[q];
+      rw += weights[ids[q]];
+      if (rw >= ((int64_t)1 << 32)) return MPT_ERR_OVERFLOW;
+    }
+    len[(size_t)i] = (int32_t)ids.size();
+    total += rw;
+  }
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
+  // device buffers (this call allocates and frees its own)
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) & ~(size_t)255;
+    return o;
+  };
+  const size_t M = (size_t)m;
+  const size_t o_w = take((size_t)n_chunks * 8), o_sig = take(M * kSigMax * 4), o_len = take(M * 4),
+               o_W = take(M * M * 4), o_best = take(M * 8), o_act = take(M), o_node = take(M * 4),
+               o_re = take(M * 4 + 4), o_mer = take(M * 8), o_val = take(M * 8), o_ch = take(M * 8),
+               o_nsig = take(M * kSigMax * 4), o_nlen = take(M * 4), o_roff = take((M + 1) * 8),
+               o_chunks = take((size_t)std::max<int64_t>(occ, 1) * 8), o_par = take(2 * M * 4),
+               o_dep = take(2 * M * 4), o_stk = take(2 * M * 4), o_keys = take((size_t)std::max<int64_t>(occ, 1) * 8),
+               o_perm = take((size_t)std::max<int64_t>(occ, 1) * 8), o_dfs = take(M * 4), o_tk = take(M * 4),
+               o_int = take(M), o_mst = take(8);
+  char* d = nullptr;
+  if (cudaMalloc(&d, off) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  mpt_status st = MPT_OK;
+  cudaError_t e = cudaSuccess;
+  auto h2d = [&](size_t o, const void* h, size_t bytes) {
+    if (e == cudaSuccess && bytes) e = cudaMemcpyAsync(d + o, h, bytes, cudaMemcpyHostToDevice, stream);
+  };
+  auto d2h = [&](void* h, size_t o, size_t bytes) {
+    if (e == cudaSuccess && bytes && h) e = cudaMemcpyAsync(h, d + o, bytes, cudaMemcpyDeviceToHost, stream);
+  };
+  h2d(o_w, weights, (size_t)n_chunks * 8);
+  h2d(o_sig, sig.data(), sig.size() * 4);
+  h2d(o_len, len.data(), len.size() * 4);
+  h2d(o_roff, req_offsets, (M + 1) * 8);
+  h2d(o_chunks, chunk_ids, (size_t)occ * 8);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d + o_re, 0, 4, stream);
+  auto I64 = [&](size_t o) { return reinterpret_cast<int64_t*>(d + o); };
+  auto I32 = [&](size_t o) { return reinterpret_cast<int32_t*>(d + o); };
+  auto U32 = [&](size_t o) { return reinterpret_cast<uint32_t*>(d + o); };
+  auto U64 = [&](size_t o) { return reinterpret_cast<unsigned long long*>(d + o); };
+  if (e == cudaSuccess) {
+    dim3 grid((unsigned)((m + 255) / 256), (unsigned)m);
+    k_pair_weights<<<grid, 256, 0, stream>>>(m, I32(o_sig), I32(o_len), I64(o_w), U32(o_W));
+    k_maxst<<<1, kGreedyThreads, 0, stream>>>(m, U32(o_W), U32(o_tk), reinterpret_cast<uint8_t*>(d + o_int),
+                                               U64(o_mst));
+    k_row_best<<<(unsigned)((m * 32 + 255) / 256), 256, 0, stream>>>(m, U32(o_W), U64(o_best));
+    k_greedy_merge<<<1, kGreedyThreads, 0, stream>>>(m, I64(o_w), I32(o_sig), I32(o_len), U32(o_W), U64(o_best),
+                                                      reinterpret_cast<uint8_t*>(d + o_act), I32(o_node), I32(o_mer),
+                                                      I64(o_val), I32(o_ch), I32(o_nsig), I32(o_nlen), I32(o_re));
+    k_greedy_tree<<<1, 1, 0, stream>>>(m, I32(o_ch), I32(o_par), I32(o_dep), I32(o_stk), I32(o_dfs));
+    const int64_t eblocks = std::min<int64_t>((std::max<int64_t>(occ, 1) + 255) / 256, 152 * 16);
+    k_greedy_emit<<<(unsigned)eblocks, 256, 0, stream>>>(m, I32(o_nsig), I32(o_nlen), I64(o_roff), I64(o_chunks),
+                                                         I32(o_par), I32(o_dep), U64(o_keys));
+    k_greedy_rank<<<(unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, 152 * 16), 256, 0, stream>>>(
+        m, I64(o_roff), U64(o_keys), I64(o_perm));
+    e = cudaGetLastError();
+  }
+  std::vector<int64_t> vals(M > 1 ? M - 1 : 1, 0);
+  unsigned long long mst = 0;
+  int32_t flag = 0;
+  d2h(&flag, o_re, 4);
+  d2h(vals.data(), o_val, (M - 1) * 8);
+  d2h(&mst, o_mst, 8);
+  d2h(merges, o_mer, (M - 1) * 2 * 4);
+  d2h(perm_chunks, o_perm, (size_t)occ * 8);
+  d2h(dfs_order, o_dfs, M * 4);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) st = MPT_ERR_CUDA;
+  else if (flag != 0) st = MPT_ERR_INTERNAL;
+  cudaFree(d);
+  if (st != MPT_OK) return st;
+  int64_t sav = 0;
+  for (size_t t = 0; t + 1 < M; ++t) sav += vals[t];
+  if (merge_values && M > 1) std::copy(vals.begin(), vals.begin() + (M - 1), merge_values);
+  if (savings) *savings = sav;
+  if (cost) *cost = total - sav;
+  if (lower_bound) *lower_bound = total - (int64_t)mst;
+  return MPT_OK;
+}

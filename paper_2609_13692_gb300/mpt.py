@@ -40,7 +40,7 @@ EXPORTED = [
     "mpt_create", "mpt_workspace_bytes", "mpt_set_dp_mode", "mpt_solve", "mpt_tables", "mpt_layout_size",
     "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
     "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
-    "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy",
+    "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy",
 ]
 
 
@@ -115,6 +115,7 @@ def load() -> ctypes.CDLL:
         "mpt_batch_results": ([vp, i64p, i64p, i32p], ctypes.c_int),
         "mpt_batch_tables": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp), i64p], ctypes.c_int),
         "mpt_batch_destroy": ([vp], None),
+        "mpt_greedy": ([i64p, i64, i32, i64p, i64p, vp, i64p, i64p, i64p, i32p, i64p, i64p, i32p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -432,3 +433,44 @@ def solve_batch(weights, instances, workspace=None, stream: Optional[int] = None
         perms.append([perm[ro[r]:ro[r + 1]].tolist() for r in range(r0, r1)])
         orders.append(dfs[r0:r1].tolist())
     return opt, perms, orders, b
+
+
+# ---------------------------------------------------------------------------
+# Agglomerative greedy and spanning-tree bound (mpt_greedy)
+# ---------------------------------------------------------------------------
+
+@dataclass
+class GreedyResult:
+    cost: int
+    savings: int
+    lower_bound: int
+    merges: np.ndarray        # int32[m-1, 2] slot pairs
+    merge_values: np.ndarray  # int64[m-1]
+    perms: list
+    dfs_order: np.ndarray
+
+
+def mpt_greedy(weights, requests, stream: Optional[int] = None) -> GreedyResult:
+    """Greedy hierarchy + layout + lower bound for ``requests`` (a list of
+    chunk-id lists) over the universe of ``weights``."""
+    lib = load()
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    offs = np.zeros(len(requests) + 1, dtype=np.int64)
+    for i, r in enumerate(requests):
+        offs[i + 1] = offs[i] + len(r)
+    ids = np.ascontiguousarray(np.concatenate([np.asarray(r, dtype=np.int64) for r in requests])
+                               if int(offs[-1]) else np.zeros(1, dtype=np.int64), dtype=np.int64)
+    m = len(requests)
+    cost, sav, lb = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    merges = np.zeros(max(1, 2 * (m - 1)), dtype=np.int32)
+    vals = np.zeros(max(1, m - 1), dtype=np.int64)
+    perm = np.zeros(max(1, int(offs[-1])), dtype=np.int64)
+    dfs = np.zeros(m, dtype=np.int32)
+    s = 0 if stream is None else int(stream)
+    _check(lib.mpt_greedy(_ptr(w, ctypes.c_int64), int(w.shape[0]), m, _ptr(offs, ctypes.c_int64),
+                          _ptr(ids, ctypes.c_int64), ctypes.c_void_p(s), ctypes.byref(cost), ctypes.byref(sav),
+                          ctypes.byref(lb), _ptr(merges, ctypes.c_int32), _ptr(vals, ctypes.c_int64),
+                          _ptr(perm, ctypes.c_int64), _ptr(dfs, ctypes.c_int32)), "mpt_greedy")
+    perms = [perm[offs[i]:offs[i + 1]].tolist() for i in range(m)]
+    return GreedyResult(int(cost.value), int(sav.value), int(lb.value), merges[:2 * (m - 1)].reshape(-1, 2),
+                        vals[:m - 1], perms, dfs)
