@@ -335,7 +335,7 @@ def run_ours(args):
 
     solve_s = max_ms / 1000.0 / args.steps
     line = {
-        "metric": METRIC,
+        "metric": METRIC if m == 28 else METRIC.replace("m=28", f"m={m}"),
         "value": value,
         "unit": "splits/s",
         "n_gpus": world,
@@ -486,7 +486,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--dp-mode", choices=["auto", "blocked", "general"], default="auto")
-    ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5],
+    ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mode", choices=["solve", "batch", "greedy"], default="solve",

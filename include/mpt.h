@@ -24,7 +24,7 @@
  *     integer) is chosen; split[S] = A, 0 for singletons and for S = 0.
  *   - Every call returns a status; on failure no output is written.
  *   - A context is not thread-safe; distinct contexts are independent.
- *   - Limits: 1 <= m <= 30, 1 <= n <= 2^31 - 1, every w(x) >= 1, and
+ *   - Limits: 1 <= m <= 32, 1 <= n <= 2^31 - 1, every w(x) >= 1, and
  *     sum_i w(R_i) < 2^62 (MPT_ERR_OVERFLOW otherwise).
  */
 #ifndef MPT_H
@@ -40,7 +40,7 @@ extern "C" {
 typedef enum mpt_status {
   MPT_OK = 0,
   MPT_ERR_INVALID_ARG = 1,         /* null pointer, m < 1, n < 1, w(x) <= 0, a bit set at x >= n */
-  MPT_ERR_TOO_LARGE = 2,           /* m > 30 */
+  MPT_ERR_TOO_LARGE = 2,           /* beyond a documented limit (m > 32 for mpt_create) */
   MPT_ERR_OVERFLOW = 3,            /* sum_i w(R_i) >= 2^62 */
   MPT_ERR_OUT_OF_MEMORY = 4,       /* host or device allocation failed */
   MPT_ERR_WORKSPACE_TOO_SMALL = 5, /* caller workspace below mpt_workspace_bytes() */

@@ -27,6 +27,11 @@ Everything here follows "Prefix Sharing Is a Sorting Problem" (arxiv
 * ``greedy``: the agglomerative common-intersection hierarchy of Sec. 6.2
   (Thm 6's H_g), with its layout and savings.
 * ``trie_cost_sorted``: eq. (1) for many strings via lexicographic sorting.
+* ``serve_order``: Thm 7's serving order (lexicographic order of the laid-out
+  strings), optionally inside consecutive windows of arrivals (Sec. 8.1).
+* ``radix_cache_costs``: ``radix_cache_cost`` over a list of capacities.
+* ``pinned_layout`` / ``brute_force_pinned``: the Sec. 7.1 variant that pins
+  each request's top-t passages, in relevance order, at the end.
 
 Readings where the paper is silent are stated in ``oracle.c``'s header.
 """
@@ -540,3 +545,81 @@ def trie_cost_sorted(weights, perms) -> int:
         cost += int(sum(int(w[x]) for x in sq[l:]))
         prev = sq
     return cost
+
+
+def recompute_local(weights, bits, S: int, F_sub) -> tuple[int, int, int]:
+    """F(S), split(S) and w(I(S)) for one subset S from a table of S's own
+    submasks: F_sub[j] = F(A) where A has the bits of j deposited into the set
+    bits of S (j = 0 .. 2^|S| - 1).  Depositing preserves order, so the
+    smallest index j is the smallest A; the lowest request of S is bit 0 of j.
+    Used to check single entries of tables too large for oracle_dp."""
+    F_sub = np.asarray(F_sub, dtype=np.int64)
+    k = bin(S).count("1")
+    full = (1 << k) - 1
+    wi = wI_one(weights, bits, S)
+    if k <= 1:
+        return (wi if S else 0), 0, wi
+    j = np.arange(1, full, 2, dtype=np.int64)  # holds bit 0 (the lowest request), not the whole set
+    vals = F_sub[j] + F_sub[full ^ j]
+    t = int(np.argmin(vals))  # first minimum = smallest A
+    jbest = int(j[t])
+    A = 0
+    pos = [i for i in range(64) if (S >> i) & 1]
+    for q, p in enumerate(pos):
+        if (jbest >> q) & 1:
+            A |= 1 << p
+    return int(vals[t]) - wi, A, wi
+
+
+def serve_order(perms, arrival=None, window: int = 0) -> list[int]:
+    """Thm 7 (Sec. 8): serve requests in the DFS order of the trie of their
+    laid-out strings, i.e. sorted lexicographically (a string before its
+    extensions).  With ``window`` = W in [1, m), the stream ``arrival`` is cut
+    into consecutive windows of W arrivals and each window is sorted on its own
+    (the bounded reorder window of Sec. 8.1).  Identical strings keep the
+    smaller request index first."""
+    m = len(perms)
+    arr = list(range(m)) if arrival is None else [int(a) for a in arrival]
+    W = m if (window <= 0 or window >= m) else int(window)
+    out: list[int] = []
+    for lo in range(0, m, max(W, 1)):
+        out += sorted(arr[lo:lo + W], key=lambda r: (tuple(int(x) for x in perms[r]), r))
+    return out
+
+
+def radix_cache_costs(weights, perms, order, capacities) -> list[int]:
+    """``radix_cache_cost`` for each capacity in ``capacities`` (one simulation each)."""
+    return [radix_cache_cost(weights, perms, order, int(c)) for c in capacities]
+
+
+def pinned_layout(weights, ranked, t: int, C=None):
+    """Sec. 7.1: pin the first ``t`` passages of each request's relevance-ranked
+    list ``ranked[i]`` at the end of its prompt, in relevance order (rank 1
+    first), and lay the remaining passages out freely with the exact
+    recurrence (Sec. 3.1) on the reduced request sets.  Returns
+    (strings, trie cost by eq. (1))."""
+    from paper_2609_13692_gb300 import instances as _inst  # bit packing only
+
+    C = C or _default()
+    n = len(weights)
+    free = [[int(x) for x in r[t:]] for r in ranked]
+    pins = [[int(x) for x in r[:t]] for r in ranked]
+    bits = _inst.pack_requests(free, n)
+    if len(ranked) == 0:
+        return [], 0
+    _opt, _F, _wI, split = C.solve(np.asarray(weights, dtype=np.int64), bits)
+    perms, _dfs = layout(weights, bits, split)
+    seqs = [list(p) + q for p, q in zip(perms, pins)]
+    return seqs, trie_cost(weights, seqs)
+
+
+def brute_force_pinned(weights, ranked, t: int) -> int:
+    """Least eq. (1) cost over every permutation of each request's free
+    passages, with its top ``t`` fixed at the end in relevance order."""
+    free = [sorted(int(x) for x in r[t:]) for r in ranked]
+    pins = [[int(x) for x in r[:t]] for r in ranked]
+    best = None
+    for choice in itertools.product(*[list(itertools.permutations(f)) for f in free]):
+        c = trie_cost(weights, [list(p) + q for p, q in zip(choice, pins)])
+        best = c if best is None or c < best else best
+    return int(best)

@@ -34,7 +34,7 @@ struct mpt_ctx {
 
 namespace {
 
-constexpr int kMaxRequests = 30;
+constexpr int kMaxRequests = 32;
 constexpr int64_t kSumLimit = (int64_t)1 << 62;
 
 bool blocked_feasible(const mpt_ctx* c) {
@@ -113,7 +113,7 @@ const char* mpt_status_string(mpt_status s) {
   switch (s) {
     case MPT_OK: return "ok";
     case MPT_ERR_INVALID_ARG: return "invalid argument";
-    case MPT_ERR_TOO_LARGE: return "too many requests (m > 30)";
+    case MPT_ERR_TOO_LARGE: return "instance beyond the documented limits";
     case MPT_ERR_OVERFLOW: return "weights too large for the requested arithmetic";
     case MPT_ERR_OUT_OF_MEMORY: return "out of memory";
     case MPT_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
@@ -310,7 +310,7 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
   p.dp_mode = s.blocked ? MPT_DP_BLOCKED : MPT_DP_GENERAL;
   p.tile_bits = s.blocked ? s.b : 0;
   {
-    // (3^m + 1)/2 - 2^m, exactly representable in a double for m <= 30
+    // (3^m + 1)/2 - 2^m, exactly representable in a double for m <= 32
     double three = 1.0;
     for (int i = 0; i < s.m; ++i) three *= 3.0;
     p.splits_total = (three + 1.0) / 2.0 - (double)N;

@@ -172,6 +172,8 @@ CONFIGS = {
     3: dict(kind="rag", m=24, n=100_000, pools=8, pool_size=200, k=10, tail_s=1.1),
     4: dict(kind="rag", m=28, n=100_000, pools=16, pool_size=300, k=20, tail_s=1.1),
     5: dict(kind="rag", m=30, n=1_000_000, pools=32, pool_size=400, k=40, tail_s=1.2),
+    6: dict(kind="rag", m=31, n=100_000, pools=16, pool_size=300, k=20, tail_s=1.1),
+    7: dict(kind="rag", m=32, n=100_000, pools=16, pool_size=300, k=20, tail_s=1.1),
 }
 
 CONFIG_NAMES = {
@@ -180,11 +182,13 @@ CONFIG_NAMES = {
     3: "rag-m24-n100k-8x200-k10",
     4: "rag-m28-n100k-16x300-k20",
     5: "rag-m30-n1M-32x400-k40",
+    6: "rag-m31-n100k-16x300-k20",
+    7: "rag-m32-n100k-16x300-k20",
 }
 
 
 def config(idx: int, seed: int = 0) -> Instance:
-    """Workload ``idx`` (1..5) with the given seed."""
+    """Workload ``idx`` (1..7) with the given seed (6, 7: the m = 31, 32 extensions)."""
     c = CONFIGS[idx]
     if c["kind"] == "zipf":
         inst = zipf_small(c["m"], c["n"], c["k"], c["s"], seed=seed)

@@ -164,6 +164,27 @@ def pin_recompute(C):
     assert np.array_equal(Fr, F[1:]) and np.array_equal(sr, split[1:]) and np.array_equal(wr, wI[1:])
 
 
+def pin_recompute_local(C):
+    """recompute_local (one subset from its own submask table) agrees with oracle_dp."""
+    inst = I.random_instance(9, 40, (2, 8), seed=87, wmin=1, wmax=60)
+    opt, F, wI, split = C.solve(inst.weights, inst.bits)
+    rng = np.random.default_rng(1)
+    for S in [int(x) for x in rng.integers(1, 1 << inst.m, size=60)] + [(1 << inst.m) - 1]:
+        pos = [i for i in range(inst.m) if (S >> i) & 1]
+        idx = [sum(1 << pos[q] for q in range(len(pos)) if (j >> q) & 1) for j in range(1 << len(pos))]
+        F_sub = F[idx]
+        k = len(pos)
+        full = (1 << k) - 1
+        wi = int(wI[S])
+        if k <= 1:
+            continue
+        j = np.arange(1, full, 2)
+        vals = F_sub[j] + F_sub[full ^ j]
+        assert int(vals.min()) - wi == F[S]
+        f, a, w = O.recompute_local(inst.weights, inst.bits, S, F_sub)
+        assert (f, a, w) == (F[S], split[S], wI[S])
+
+
 ALL_PINS = [
     pin_k4_3,
     pin_open_problem,
@@ -177,4 +198,5 @@ ALL_PINS = [
     pin_bounds,
     pin_split_rule,
     pin_recompute,
+    pin_recompute_local,
 ]

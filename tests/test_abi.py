@@ -65,7 +65,7 @@ def test_create_validation(mpt):
     bits = inst.bits.copy()
     bits[0, 0] |= np.uint64(1) << np.uint64(50)  # chunk 50 >= n = 48
     assert _status(mpt, inst.weights, bits) == 1
-    big = I.random_instance(31, 40, 3, seed=1)
+    big = I.random_instance(33, 40, 3, seed=1)
     assert _status(mpt, big.weights, big.bits) == 2
     huge = I.Instance(np.full(4, 1 << 61, dtype=np.int64), I.pack_requests([[0, 1], [2, 3], [0]], 4))
     assert _status(mpt, huge.weights, huge.bits) == 3

@@ -188,3 +188,57 @@ def test_config5_m30(mpt):
     """RAG-shaped m = 30, k = 40, 1M-passage corpus."""
     res, prof, count = assert_sampled_parity(mpt, I.config(5), seed=30, uniform=20000)
     assert prof["dp_mode"] == 1
+
+
+def _submask_index(S):
+    pos = [i for i in range(64) if (S >> i) & 1]
+    idx = np.zeros(1 << len(pos), dtype=np.int64)
+    for q, p in enumerate(pos):
+        idx[np.arange(1 << len(pos)) & (1 << q) != 0] |= 1 << p
+    return idx
+
+
+def test_m31_extension(mpt):
+    """m = 31 (2^31-entry tables): layout trie cost = OPT, bounds, the split of
+    every sampled subset attains its F, no random split does better, and small
+    subsets recomputed by the oracle from their own submask tables."""
+    inst = I.config(6)
+    res = mpt.solve(inst.weights, inst.bits)
+    F_d, wI_d, split_d = mpt.mpt_tables(res.ctx)
+    m = inst.m
+    assert O.trie_cost(inst.weights, res.permutations()) == res.opt
+    assert mpt.mpt_trie_cost(inst.weights, res.perm_offsets, res.perm_chunks) == res.opt
+    R = O.request_sets(inst.weights, inst.bits)
+    assert all(sorted(p) == sorted(R[i]) for i, p in enumerate(res.permutations()))
+    assert O.spanning_tree_bound(inst.weights, inst.bits) <= res.opt <= O.global_order_cost(inst.weights, inst.bits)
+    rng = np.random.default_rng(31)
+    full = (1 << m) - 1
+    # property checks on random subsets of every size (and the full set)
+    Ss = [full] + [int(sum(1 << int(i) for i in rng.choice(m, size=k, replace=False)))
+                   for k in range(2, m + 1) for _ in range(8)]
+    S_t = torch.tensor(Ss, dtype=torch.int64, device=F_d.device)
+    A_t = split_d[S_t].to(torch.int64) & 0xFFFFFFFF
+    F_S, F_A, F_B = F_d[S_t], F_d[A_t], F_d[S_t ^ A_t]
+    wI_S = wI_d[S_t]
+    assert bool(torch.all(F_S == F_A + F_B - wI_S))
+    assert bool(torch.all((A_t & S_t) == A_t)) and bool(torch.all((A_t & (S_t & -S_t)) != 0))
+    for S in Ss[:40]:
+        assert int(wI_d[S].item()) == O.wI_one(inst.weights, inst.bits, S)
+    for _ in range(200):  # random other splits never beat the chosen one
+        k = int(rng.integers(0, len(Ss)))
+        S = Ss[k]
+        low = S & -S
+        rest = S ^ low
+        bits_rest = [i for i in range(m) if (rest >> i) & 1]
+        sub = sum(1 << i for i in bits_rest if rng.random() < 0.5)
+        if sub == rest:
+            continue
+        A = low | sub
+        assert int(F_d[A].item()) + int(F_d[S ^ A].item()) - int(wI_d[S].item()) >= int(F_d[S].item())
+    # oracle recomputation of small subsets from their own submask tables
+    for k in range(2, 15):
+        for _ in range(6):
+            S = int(sum(1 << int(i) for i in rng.choice(m, size=k, replace=False)))
+            idx = torch.from_numpy(_submask_index(S)).to(F_d.device)
+            f, a, w = O.recompute_local(inst.weights, inst.bits, S, F_d[idx].cpu().numpy())
+            assert (f, a, w) == (int(F_d[S].item()), int(split_d[S].item()) & 0xFFFFFFFF, int(wI_d[S].item()))
