@@ -473,6 +473,68 @@ def run_greedy(args):
     print(json.dumps(line), flush=True)
 
 
+def run_cache(args):
+    """Finite-cache study (Sec. 8) on the NFCorpus-shaped stream: prefill cost
+    at many capacities per call, in arrival order, inside reorder windows and
+    in Thm 7's order, for the production (relevance-order), greedy and pinned
+    layouts."""
+    import torch
+
+    from paper_2609_13692_gb300 import build as B
+    from paper_2609_13692_gb300 import instances
+    from paper_2609_13692_gb300 import mpt
+
+    torch.cuda.set_device(0)
+    if not B.LIB.exists():
+        B.build()
+    weights, ranked = instances.stream("nfcorpus-shaped", seed=0)
+    n, m = len(weights), len(ranked)
+    one = float(np.mean([sum(int(weights[x]) for x in q) for q in ranked]))
+    mult = [0.25, 0.5, 0.75, 0.9, 1, 4, 16, 64, 256, 1024]
+    caps = [int(round(f * one)) for f in mult]
+    layouts = {"production": [list(r) for r in ranked], "greedy": mpt.mpt_greedy(weights, ranked).perms}
+    for t in (1, 2, 3):
+        layouts[f"pin_top{t}"] = mpt.mpt_layout_pinned(weights, ranked, t, "greedy").strings
+    total = int(sum(int(weights[x]) for q in ranked for x in q))
+    arrival = list(range(m))
+    g = layouts["greedy"]
+    for _ in range(args.warmup):
+        mpt.mpt_cache_costs(weights, g, caps, arrival)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        mpt.mpt_cache_costs(weights, g, caps, arrival)
+    dt = (time.perf_counter() - t0) / args.steps
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        thm7 = mpt.mpt_serve_order(n, g)
+    dt_order = (time.perf_counter() - t0) / args.steps
+
+    table = {}
+    for name, strings in layouts.items():
+        unb = None
+        row = {}
+        for label, order in (("arrival", arrival), ("thm7", mpt.mpt_serve_order(n, strings).tolist())):
+            costs, unb = mpt.mpt_cache_costs(weights, strings, caps, order)
+            row[label] = {f"{f}x": int(c) for f, c in zip(mult, costs)}
+        row["unbounded"] = unb
+        row["saving_vs_no_sharing"] = 1 - unb / total
+        table[name] = row
+    windows = {}
+    for W in (1, 128, 512, 2048, m):
+        order = mpt.mpt_serve_order(n, g, arrival, W).tolist()
+        costs, unb = mpt.mpt_cache_costs(weights, g, caps[4:], order)
+        windows["all" if W == m else str(W)] = {f"{f}x": round(c / unb - 1, 4) for f, c in zip(mult[4:], costs)}
+    line = {"mode": "cache", "metric": "finite radix cache, prefill cost at 10 capacities per call",
+            "value": dt, "unit": "s", "higher_is_better": False, "steps": args.steps,
+            "workload": f"nfcorpus-shaped stream: m = {m} requests, k = 8, one request = {one:.0f} tokens",
+            "accesses": int(sum(len(q) for q in g)), "serve_order_s": dt_order,
+            "capacities_in_requests": mult, "no_sharing_cost": total, "layouts": table,
+            "window_excess_over_unbounded_greedy": windows,
+            "note": "host arrays in and out, device buffers allocated inside each call"}
+    print(json.dumps(line), flush=True)
+
+
 def _pack(reqs, n):
     from paper_2609_13692_gb300 import instances
 
@@ -489,9 +551,10 @@ def main():
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--mode", choices=["solve", "batch", "greedy"], default="solve",
+    ap.add_argument("--mode", choices=["solve", "batch", "greedy", "cache"], default="solve",
                     help="solve: the m = 28 exact solve (default); batch: many small request groups; "
-                         "greedy: agglomerative hierarchy on a trace-sized request set")
+                         "greedy: agglomerative hierarchy on a trace-sized request set; "
+                         "cache: finite-cache study on a request stream")
     ap.add_argument("--batch-size", type=int, default=20000)
     ap.add_argument("--greedy-m", type=int, default=3000)
     args = ap.parse_args()
@@ -500,6 +563,9 @@ def main():
         return
     if args.mode == "greedy":
         run_greedy(args)
+        return
+    if args.mode == "cache":
+        run_cache(args)
         return
     if args.impl == "reference":
         run_reference(args)

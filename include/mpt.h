@@ -115,11 +115,15 @@ mpt_status mpt_layout_size(const mpt_ctx* ctx, int64_t* total_chunks);
 mpt_status mpt_layout(const mpt_ctx* ctx, int64_t* perm_offsets, int64_t* perm_chunks, int32_t* dfs_order);
 
 /* Trie cost of a layout (Sec. 2, eq. 1): the total weight of the non-root
- * nodes of the trie of the m strings, computed by a CUDA kernel.  All
- * pointers are host memory; perm_offsets has m+1 entries, perm_chunks
- * perm_offsets[m] entries with ids in [0, n_chunks).  The call allocates a
- * small device buffer and synchronises the legacy default stream.
- * Errors: INVALID_ARG, OUT_OF_MEMORY, CUDA. */
+ * nodes of the trie of the m strings, computed on the GPU.  All pointers are
+ * host memory; perm_offsets has m+1 entries, perm_chunks perm_offsets[m]
+ * entries with ids in [0, n_chunks).  Up to 32 strings one block compares
+ * every pair; beyond that the strings are sorted lexicographically and each
+ * adds the weight of its suffix after the common prefix with its predecessor.
+ * Limits: m <= 2^22 strings, perm_offsets[m] <= 2^27, each string <= 4096
+ * chunks (MPT_ERR_TOO_LARGE).  The call allocates and frees a device buffer
+ * and synchronises the legacy default stream.
+ * Errors: INVALID_ARG, TOO_LARGE, OUT_OF_MEMORY, CUDA. */
 mpt_status mpt_trie_cost(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* perm_offsets,
                          const int64_t* perm_chunks, int64_t* cost);
 
@@ -221,6 +225,69 @@ mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32_t m, const
                       const int64_t* chunk_ids, void* stream, int64_t* cost, int64_t* savings,
                       int64_t* lower_bound, int32_t* merges, int64_t* merge_values, int64_t* perm_chunks,
                       int32_t* dfs_order);
+
+/* ---------------------------------------------------------------------------
+ * Serving order and finite cache (Sec. 8, Thm 7)
+ *
+ * Strings are laid-out requests, given as a host CSR: string i is
+ * seq_chunks[seq_offsets[i] .. seq_offsets[i+1]) (chunk ids in [0, n_chunks);
+ * seq_offsets[0] = 0).  Limits: 1 <= m <= 2^22 strings, seq_offsets[m] <=
+ * 2^27 chunk occurrences, each string <= 4096 chunks (MPT_ERR_TOO_LARGE).
+ * Each call allocates and frees its device buffers, runs on `stream` (a
+ * cudaStream_t, NULL = legacy default) and synchronises it before returning.
+ * ------------------------------------------------------------------------- */
+
+/* Thm 7's serving order: the strings sorted lexicographically (a string
+ * before its extensions; identical strings by increasing index), which is the
+ * DFS order of their trie.  With 0 < window < m, the stream `arrival` (a
+ * permutation of 0..m-1, NULL = 0, 1, .., m-1) is cut into consecutive
+ * windows of `window` arrivals and each window is sorted on its own -- the
+ * bounded reorder window of Sec. 8.1; window = 0 or >= m sorts everything.
+ *   order: host int32[m], the request served at each position.
+ * Errors: INVALID_ARG, TOO_LARGE, OUT_OF_MEMORY, CUDA. */
+mpt_status mpt_serve_order(int64_t n_chunks, int32_t m, const int64_t* seq_offsets, const int64_t* seq_chunks,
+                           const int32_t* arrival, int32_t window, void* stream, int32_t* order);
+
+/* Prefill cost under a finite radix (prefix) cache, for several capacities at
+ * once (Sec. 8).  Requests are served in `order` (host int32[m], a
+ * permutation; NULL = 0, 1, .., m-1).  The cache holds trie nodes (one chunk
+ * each, weight w(chunk)); a cached node implies its ancestors are cached.
+ * Serving a request computes, and pays for, every chunk of its string past
+ * the longest cached prefix, then inserts them; when the cached weight exceeds
+ * the capacity, least recently used leaves that are not on the current
+ * request's path are evicted (a request touches every node of its path), and
+ * chunks that still find no room are computed without being cached.
+ *   weights: host int64[n_chunks] (>= 1); capacities: host int64[n_caps]
+ *   (>= 0, n_caps <= 1024);
+ *   costs: host int64[n_caps], the total prefill weight at each capacity;
+ *   unbounded: host int64[1] (may be NULL), the cost with no eviction = the
+ *   trie weight of eq. (1).
+ * Thm 7: in the order of mpt_serve_order, any capacity >= max_i w(string i)
+ * pays exactly `unbounded`.  Errors: INVALID_ARG, TOO_LARGE, OVERFLOW (total
+ * string weight >= 2^62), OUT_OF_MEMORY, CUDA, INTERNAL. */
+mpt_status mpt_cache_costs(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* seq_offsets,
+                           const int64_t* seq_chunks, const int32_t* order, const int64_t* capacities,
+                           int32_t n_caps, void* stream, int64_t* costs, int64_t* unbounded);
+
+/* Quality-preserving variant of the layout (Sec. 7.1): each request's t most
+ * relevant passages are pinned at the end of its prompt, in relevance order
+ * (rank 1 first), and only the rest is laid out: by the exact recurrence
+ * (method MPT_PIN_EXACT, m <= 32) or by the agglomerative hierarchy
+ * (MPT_PIN_GREEDY, the limits of mpt_greedy) on the reduced request sets.
+ *   ranked_offsets / ranked_chunks: host CSR, request i's passages in
+ *   relevance order (most relevant first), no repeats inside a request;
+ *   t >= 0 (a request with at most t passages is pinned whole);
+ *   perm_chunks: host int64[ranked_offsets[m]] (may be NULL), each request's
+ *   laid-out string in its own CSR range;
+ *   serve_order: host int32[m] (may be NULL), Thm 7's order of those strings;
+ *   cost: host int64[1] (may be NULL), their trie weight (eq. 1).
+ * Errors: those of mpt_create / mpt_solve or mpt_greedy, plus INVALID_ARG and
+ * TOO_LARGE. */
+#define MPT_PIN_EXACT 0
+#define MPT_PIN_GREEDY 1
+mpt_status mpt_layout_pinned(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* ranked_offsets,
+                             const int64_t* ranked_chunks, int32_t t, int32_t method, void* stream,
+                             int64_t* perm_chunks, int32_t* serve_order, int64_t* cost);
 
 /* Exact solve that allocates nothing, for callers that cannot allocate device
  * memory: code running in a serving process whose device memory is reserved

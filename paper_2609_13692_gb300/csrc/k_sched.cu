@@ -851,4 +851,74 @@ mpt_status mpt_cache_costs(const int64_t* weights, int64_t n_chunks, int32_t m, 
   return MPT_OK;
 }
 
+mpt_status mpt_layout_pinned(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* ranked_offsets,
+                             const int64_t* ranked_chunks, int32_t t, int32_t method, void* stream,
+                             int64_t* perm_chunks, int32_t* serve_order, int64_t* cost) {
+  using namespace mpt;
+  if (!weights || !ranked_offsets || n_chunks < 1 || n_chunks >= INT32_MAX || m < 1 || t < 0) return MPT_ERR_INVALID_ARG;
+  if (method != MPT_PIN_EXACT && method != MPT_PIN_GREEDY) return MPT_ERR_INVALID_ARG;
+  if (method == MPT_PIN_EXACT && m > 32) return MPT_ERR_TOO_LARGE;
+  if (ranked_offsets[0] != 0) return MPT_ERR_INVALID_ARG;
+  const int64_t total = ranked_offsets[m];
+  if (total > 0 && !ranked_chunks) return MPT_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < m; ++i)
+    if (ranked_offsets[i + 1] < ranked_offsets[i]) return MPT_ERR_INVALID_ARG;
+  for (int64_t p = 0; p < total; ++p)
+    if (ranked_chunks[p] < 0 || ranked_chunks[p] >= n_chunks) return MPT_ERR_INVALID_ARG;
+  // free part of request i: its ranked list after the first t entries
+  std::vector<int64_t> foff((size_t)m + 1, 0), fchunks, seq((size_t)(total > 0 ? total : 1));
+  for (int32_t i = 0; i < m; ++i) {
+    const int64_t a = ranked_offsets[i], b = ranked_offsets[i + 1];
+    const int64_t pin = b - a < t ? b - a : t;
+    for (int64_t p = a + pin; p < b; ++p) fchunks.push_back(ranked_chunks[p]);
+    foff[(size_t)i + 1] = (int64_t)fchunks.size();
+  }
+  std::vector<int64_t> fperm(fchunks.size() > 0 ? fchunks.size() : 1);
+  mpt_status ms;
+  if (method == MPT_PIN_EXACT) {
+    const int64_t words = (n_chunks + 63) / 64;
+    std::vector<uint64_t> bits((size_t)m * (size_t)words, 0);
+    for (int32_t i = 0; i < m; ++i)
+      for (int64_t p = foff[(size_t)i]; p < foff[(size_t)i + 1]; ++p) {
+        const int64_t x = fchunks[(size_t)p];
+        uint64_t& wd = bits[(size_t)i * (size_t)words + (size_t)(x >> 6)];
+        if (wd >> (x & 63) & 1ull) return MPT_ERR_INVALID_ARG;  // repeated chunk
+        wd |= 1ull << (x & 63);
+      }
+    mpt_ctx* ctx = nullptr;
+    if ((ms = mpt_create(weights, n_chunks, bits.data(), m, &ctx)) != MPT_OK) return ms;
+    int64_t opt = 0;
+    std::vector<int64_t> poff((size_t)m + 1);
+    ms = mpt_solve(ctx, nullptr, 0, stream, &opt);
+    if (ms == MPT_OK) ms = mpt_layout(ctx, poff.data(), fperm.data(), nullptr);
+    mpt_destroy(ctx);
+    if (ms != MPT_OK) return ms;
+    // mpt_layout's request ranges coincide with the free CSR (same sizes)
+    for (int32_t i = 0; i <= m; ++i)
+      if (poff[(size_t)i] != foff[(size_t)i]) return MPT_ERR_INTERNAL;
+  } else {
+    ms = mpt_greedy(weights, n_chunks, m, foff.data(), fchunks.empty() ? nullptr : fchunks.data(), stream, nullptr,
+                    nullptr, nullptr, nullptr, nullptr, fperm.data(), nullptr);
+    if (ms != MPT_OK) return ms;
+  }
+  // strings: free layout, then the pinned passages in relevance order
+  for (int32_t i = 0; i < m; ++i) {
+    const int64_t a = ranked_offsets[i], b = ranked_offsets[i + 1];
+    const int64_t pin = b - a < t ? b - a : t;
+    int64_t o = a;
+    for (int64_t p = foff[(size_t)i]; p < foff[(size_t)i + 1]; ++p) seq[(size_t)o++] = fperm[(size_t)p];
+    for (int64_t p = a; p < a + pin; ++p) seq[(size_t)o++] = ranked_chunks[p];
+  }
+  if (perm_chunks && total > 0) std::memcpy(perm_chunks, seq.data(), (size_t)total * 8);
+  if (serve_order) {
+    ms = mpt_serve_order(n_chunks, m, ranked_offsets, seq.data(), nullptr, 0, stream, serve_order);
+    if (ms != MPT_OK) return ms;
+  }
+  if (cost) {
+    ms = trie_cost_lex(weights, n_chunks, m, ranked_offsets, seq.data(), reinterpret_cast<cudaStream_t>(stream), cost);
+    if (ms != MPT_OK) return ms;
+  }
+  return MPT_OK;
+}
+
 }  // extern "C"

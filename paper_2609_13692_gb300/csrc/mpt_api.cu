@@ -361,7 +361,8 @@ mpt_status mpt_layout(const mpt_ctx* ctx, int64_t* perm_offsets, int64_t* perm_c
 
 mpt_status mpt_trie_cost(const int64_t* weights, int64_t n_chunks, int32_t m, const int64_t* perm_offsets,
                          const int64_t* perm_chunks, int64_t* cost) {
-  if (!weights || !perm_offsets || !cost || n_chunks < 1 || m < 1 || m > 32) return MPT_ERR_INVALID_ARG;
+  if (!weights || !perm_offsets || !cost || n_chunks < 1 || m < 1) return MPT_ERR_INVALID_ARG;
+  if (m > 32) return mpt::trie_cost_lex(weights, n_chunks, m, perm_offsets, perm_chunks, 0, cost);
   if (perm_offsets[0] != 0) return MPT_ERR_INVALID_ARG;
   for (int i = 0; i < m; ++i)
     if (perm_offsets[i + 1] < perm_offsets[i]) return MPT_ERR_INVALID_ARG;

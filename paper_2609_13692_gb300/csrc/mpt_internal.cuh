@@ -7,6 +7,8 @@
 
 #include <cuda_runtime.h>
 
+#include "../../include/mpt.h"
+
 namespace mpt {
 
 // ---------------------------------------------------------------------------
@@ -139,6 +141,9 @@ int64_t blocked_partial_entries(int m, int b);
 int blocked_tile_bits(int m);
 
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+// eq. (1) for any number of strings by lexicographic sorting (k_sched.cu)
+mpt_status trie_cost_lex(const int64_t* weights, int64_t n_chunks, int64_t m, const int64_t* offsets,
+                         const int64_t* chunks, cudaStream_t st, int64_t* cost);
 cudaError_t launch_trie_cost(int m, const int64_t* d_weights, const int64_t* d_offsets, const int64_t* d_chunks,
                              int64_t* d_cost, cudaStream_t stream);
 

@@ -34,6 +34,9 @@ __all__ = [
     "zipf_small",
     "leave_one_out",
     "rag_pools",
+    "rag_ranked",
+    "stream",
+    "STREAMS",
     "config",
     "CONFIGS",
     "random_instance",
@@ -127,19 +130,9 @@ def leave_one_out(n: int) -> Instance:
     return Instance(weights, pack_requests(reqs, n), f"leave-one-out n={n}")
 
 
-def rag_pools(m: int, n: int, pools: int, pool_size: int, k: int, tail_s: float, seed: int = 0,
-              p_pool: float = 0.8, w_mean: float = 150.0, w_sigma: float = 0.6, wmin: int = 32,
-              wmax: int = 512) -> Instance:
-    """RAG-shaped retrieval groups.
-
-    The corpus has ``n`` passages.  ``pools`` disjoint topical pools of
-    ``pool_size`` passages are drawn from it; a global tail ranks every passage
-    (random permutation) under finite Zipf(``tail_s``).  Request i picks a pool
-    uniformly; each of its ``k`` slots comes from that pool (uniformly) with
-    probability ``p_pool``, else from the tail; duplicates are redrawn.
-    Passage weights are lognormal with mean ``w_mean`` (mu = ln(mean) - sigma^2/2),
-    rounded and clipped to [wmin, wmax].
-    """
+def _rag_draw(m: int, n: int, pools: int, pool_size: int, k: int, tail_s: float, seed: int, p_pool: float,
+              w_mean: float, w_sigma: float, wmin: int, wmax: int):
+    """Weights and per-request passage lists, in draw order (see rag_pools)."""
     rng = np.random.default_rng(seed)
     mu = math.log(w_mean) - w_sigma * w_sigma / 2.0
     weights = np.clip(np.rint(rng.lognormal(mu, w_sigma, size=n)), wmin, wmax).astype(np.int64)
@@ -161,8 +154,51 @@ def rag_pools(m: int, n: int, pools: int, pool_size: int, k: int, tail_s: float,
             return draw_tail()
 
         reqs.append(_draw_distinct(rng, k, draw_one))
+    return weights, reqs
+
+
+def rag_pools(m: int, n: int, pools: int, pool_size: int, k: int, tail_s: float, seed: int = 0,
+              p_pool: float = 0.8, w_mean: float = 150.0, w_sigma: float = 0.6, wmin: int = 32,
+              wmax: int = 512) -> Instance:
+    """RAG-shaped retrieval groups.
+
+    The corpus has ``n`` passages.  ``pools`` disjoint topical pools of
+    ``pool_size`` passages are drawn from it; a global tail ranks every passage
+    (random permutation) under finite Zipf(``tail_s``).  Request i picks a pool
+    uniformly; each of its ``k`` slots comes from that pool (uniformly) with
+    probability ``p_pool``, else from the tail; duplicates are redrawn.
+    Passage weights are lognormal with mean ``w_mean`` (mu = ln(mean) - sigma^2/2),
+    rounded and clipped to [wmin, wmax].
+    """
+    weights, reqs = _rag_draw(m, n, pools, pool_size, k, tail_s, seed, p_pool, w_mean, w_sigma, wmin, wmax)
     return Instance(weights, pack_requests(reqs, n),
                     f"rag m={m} n={n} pools={pools}x{pool_size} k={k} tail_s={tail_s} seed={seed}")
+
+
+def rag_ranked(m: int, n: int, pools: int, pool_size: int, k: int, tail_s: float, seed: int = 0,
+               p_pool: float = 0.8, w_mean: float = 150.0, w_sigma: float = 0.6, wmin: int = 32,
+               wmax: int = 512):
+    """The requests of rag_pools as relevance-ranked lists (rank = draw order),
+    in arrival order: (weights int64[n], list of m chunk-id lists)."""
+    return _rag_draw(m, n, pools, pool_size, k, tail_s, seed, p_pool, w_mean, w_sigma, wmin, wmax)
+
+
+# Request streams of the finite-cache study (Sec. 8): NFCorpus- and
+# SciFact-shaped (k = 8 passages per query; about 6,000 tokens per request,
+# i.e. passages of about 750 tokens), in arrival order.
+STREAMS = {
+    "nfcorpus-shaped": dict(m=2921, n=3633, pools=64, pool_size=40, k=8, tail_s=1.0, w_mean=750.0, wmin=64,
+                            wmax=4096),
+    "scifact-shaped": dict(m=1109, n=5183, pools=32, pool_size=60, k=8, tail_s=1.0, w_mean=750.0, wmin=64,
+                           wmax=4096),
+}
+
+
+def stream(name: str, seed: int = 0):
+    """(weights, ranked requests in arrival order) of a Sec. 8 stream."""
+    c = dict(STREAMS[name])
+    return rag_ranked(c.pop("m"), c.pop("n"), c.pop("pools"), c.pop("pool_size"), c.pop("k"), c.pop("tail_s"),
+                      seed=seed, **c)
 
 
 # The five workloads of the exact-solver benchmark, indexed 1..5.

@@ -40,7 +40,8 @@ EXPORTED = [
     "mpt_create", "mpt_workspace_bytes", "mpt_set_dp_mode", "mpt_solve", "mpt_tables", "mpt_layout_size",
     "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
     "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
-    "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy",
+    "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
+    "mpt_cache_costs", "mpt_layout_pinned",
 ]
 
 
@@ -116,6 +117,9 @@ def load() -> ctypes.CDLL:
         "mpt_batch_tables": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp), i64p], ctypes.c_int),
         "mpt_batch_destroy": ([vp], None),
         "mpt_greedy": ([i64p, i64, i32, i64p, i64p, vp, i64p, i64p, i64p, i32p, i64p, i64p, i32p], ctypes.c_int),
+        "mpt_serve_order": ([i64, i32, i64p, i64p, i32p, i32, vp, i32p], ctypes.c_int),
+        "mpt_cache_costs": ([i64p, i64, i32, i64p, i64p, i32p, i64p, i32, vp, i64p, i64p], ctypes.c_int),
+        "mpt_layout_pinned": ([i64p, i64, i32, i64p, i64p, i32, i32, vp, i64p, i32p, i64p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -474,3 +478,84 @@ def mpt_greedy(weights, requests, stream: Optional[int] = None) -> GreedyResult:
     perms = [perm[offs[i]:offs[i + 1]].tolist() for i in range(m)]
     return GreedyResult(int(cost.value), int(sav.value), int(lb.value), merges[:2 * (m - 1)].reshape(-1, 2),
                         vals[:m - 1], perms, dfs)
+
+
+def _csr(strings):
+    """(offsets, ids) int64 arrays of a list of chunk-id lists; ids has >= 1 entry."""
+    offs = np.zeros(len(strings) + 1, dtype=np.int64)
+    for i, r in enumerate(strings):
+        offs[i + 1] = offs[i] + len(r)
+    ids = (np.concatenate([np.asarray(r, dtype=np.int64) for r in strings])
+           if int(offs[-1]) else np.zeros(1, dtype=np.int64))
+    return offs, np.ascontiguousarray(ids, dtype=np.int64)
+
+
+def mpt_serve_order(n_chunks: int, strings, arrival=None, window: int = 0,
+                    stream: Optional[int] = None) -> np.ndarray:
+    """Thm 7's serving order of ``strings`` (lists of chunk ids), optionally
+    sorted only inside consecutive windows of ``window`` arrivals of ``arrival``."""
+    lib = load()
+    offs, ids = _csr(strings)
+    m = len(strings)
+    arr = None if arrival is None else np.ascontiguousarray(arrival, dtype=np.int32)
+    out = np.zeros(max(m, 1), dtype=np.int32)
+    s = 0 if stream is None else int(stream)
+    _check(lib.mpt_serve_order(int(n_chunks), m, _ptr(offs, ctypes.c_int64), _ptr(ids, ctypes.c_int64),
+                               None if arr is None else _ptr(arr, ctypes.c_int32), int(window), ctypes.c_void_p(s),
+                               _ptr(out, ctypes.c_int32)), "mpt_serve_order")
+    return out[:m]
+
+
+def mpt_cache_costs(weights, strings, capacities, order=None, stream: Optional[int] = None):
+    """Prefill cost of serving ``strings`` in ``order`` through a radix cache
+    with LRU leaf eviction, at every capacity in ``capacities``.  Returns
+    (costs int64[len(capacities)], unbounded-cache cost)."""
+    lib = load()
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    offs, ids = _csr(strings)
+    m = len(strings)
+    caps = np.ascontiguousarray(capacities, dtype=np.int64)
+    if caps.size == 0:
+        caps = np.zeros(1, dtype=np.int64)
+        n_caps = 0
+    else:
+        n_caps = int(caps.size)
+    ordv = None if order is None else np.ascontiguousarray(order, dtype=np.int32)
+    costs = np.zeros(max(n_caps, 1), dtype=np.int64)
+    unb = ctypes.c_int64()
+    s = 0 if stream is None else int(stream)
+    _check(lib.mpt_cache_costs(_ptr(w, ctypes.c_int64), int(w.shape[0]), m, _ptr(offs, ctypes.c_int64),
+                               _ptr(ids, ctypes.c_int64), None if ordv is None else _ptr(ordv, ctypes.c_int32),
+                               _ptr(caps, ctypes.c_int64), n_caps, ctypes.c_void_p(s), _ptr(costs, ctypes.c_int64),
+                               ctypes.byref(unb)), "mpt_cache_costs")
+    return costs[:n_caps], int(unb.value)
+
+
+PIN_METHODS = {"exact": 0, "greedy": 1}
+
+
+@dataclass
+class PinnedResult:
+    strings: list  # per request: free layout, then the pinned passages
+    serve_order: np.ndarray
+    cost: int
+
+
+def mpt_layout_pinned(weights, ranked, t: int, method: str = "exact",
+                      stream: Optional[int] = None) -> PinnedResult:
+    """Sec. 7.1 layout: each request's first ``t`` passages of ``ranked[i]``
+    (relevance order) pinned at the end, the rest laid out by ``method``."""
+    lib = load()
+    w = np.ascontiguousarray(weights, dtype=np.int64)
+    offs, ids = _csr(ranked)
+    m = len(ranked)
+    perm = np.zeros(max(1, int(offs[-1])), dtype=np.int64)
+    order = np.zeros(max(m, 1), dtype=np.int32)
+    cost = ctypes.c_int64()
+    s = 0 if stream is None else int(stream)
+    _check(lib.mpt_layout_pinned(_ptr(w, ctypes.c_int64), int(w.shape[0]), m, _ptr(offs, ctypes.c_int64),
+                                 _ptr(ids, ctypes.c_int64), int(t), PIN_METHODS[method], ctypes.c_void_p(s),
+                                 _ptr(perm, ctypes.c_int64), _ptr(order, ctypes.c_int32), ctypes.byref(cost)),
+           "mpt_layout_pinned")
+    strings = [perm[offs[i]:offs[i + 1]].tolist() for i in range(m)]
+    return PinnedResult(strings, order[:m], int(cost.value))

@@ -117,3 +117,63 @@ def test_batch_create_validation(mpt):
     assert _batch_status(mpt, heavy, [[[0, 1]]]) == 3                       # sum of w(R_i) >= 2^31
     big = [[list(range(0, 2049))]]
     assert _batch_status(mpt, np.ones(3000, dtype=np.int64), big) == 2      # > 2048 occurrences
+
+
+def test_schedule_and_cache_validation(mpt):
+    """Argument checks of mpt_serve_order / mpt_cache_costs / mpt_layout_pinned
+    happen on the host, before any CUDA call."""
+    import ctypes
+
+    lib = mpt.load()
+    i64p, i32p = ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int32)
+
+    def p64(a):
+        return np.ascontiguousarray(a, dtype=np.int64).ctypes.data_as(i64p)
+
+    w = np.ones(5, dtype=np.int64)
+    offs = np.array([0, 2, 3], dtype=np.int64)
+    ch = np.array([0, 1, 4], dtype=np.int64)
+    out = np.zeros(2, dtype=np.int32)
+    o32 = out.ctypes.data_as(i32p)
+
+    def order_status(n, m, offs, ch, arrival=None, window=0):
+        arr = None if arrival is None else np.ascontiguousarray(arrival, dtype=np.int32).ctypes.data_as(i32p)
+        return lib.mpt_serve_order(n, m, p64(offs), p64(ch), arr, window, None, o32)
+
+    assert order_status(5, 0, offs, ch) == 1                          # m < 1
+    assert order_status(5, 2, np.array([1, 2, 3]), ch) == 1            # offsets not from 0
+    assert order_status(5, 2, np.array([0, 3, 2]), ch) == 1            # decreasing offsets
+    assert order_status(4, 2, offs, ch) == 1                          # chunk id >= n
+    assert order_status(5, 2, offs, ch, arrival=[0, 0]) == 1          # arrival not a permutation
+    assert order_status(5, 2, offs, ch, window=-1) == 1               # negative window
+    long_offs = np.array([0, 4097], dtype=np.int64)
+    assert order_status(5000, 1, long_offs, np.arange(4097)) == 2     # string longer than 4096
+
+    caps = np.array([0, 3], dtype=np.int64)
+    costs = np.zeros(2, dtype=np.int64)
+
+    def cache_status(w, caps, n_caps, order=None):
+        o = None if order is None else np.ascontiguousarray(order, dtype=np.int32).ctypes.data_as(i32p)
+        return lib.mpt_cache_costs(p64(w), int(len(w)), 2, p64(offs), p64(ch), o, p64(caps), n_caps, None,
+                                   costs.ctypes.data_as(i64p), None)
+
+    assert cache_status(w, caps, -1) == 1                              # negative count
+    assert cache_status(w, caps, 1025) == 1                            # more than 1024 capacities
+    assert cache_status(w, np.array([-1, 3]), 2) == 1                  # negative capacity
+    assert cache_status(np.array([1, 1, 0, 1, 1]), caps, 2) == 1       # weight 0
+    assert cache_status(w, caps, 2, order=[1, 1]) == 1                 # order not a permutation
+    big = np.full(5, 1 << 61, dtype=np.int64)
+    assert cache_status(big, caps, 2) == 3                             # total weight >= 2^62
+
+    perm = np.zeros(3, dtype=np.int64)
+
+    def pinned_status(m, offs, ch, t, method):
+        return lib.mpt_layout_pinned(p64(w), 5, m, p64(offs), p64(ch), t, method, None,
+                                     perm.ctypes.data_as(i64p), None, None)
+
+    assert pinned_status(2, offs, ch, -1, 0) == 1                      # t < 0
+    assert pinned_status(2, offs, ch, 1, 7) == 1                       # unknown method
+    assert pinned_status(2, offs, np.array([0, 1, 9]), 1, 0) == 1      # chunk id >= n
+    assert pinned_status(2, offs, np.array([0, 0, 4]), 0, 0) == 1      # repeated chunk in a request
+    o33 = np.arange(34, dtype=np.int64) % 3
+    assert pinned_status(33, np.arange(34, dtype=np.int64), o33, 0, 0) == 2  # exact method beyond 32
