@@ -92,6 +92,35 @@ mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode);
  * Errors: INVALID_ARG, WORKSPACE_TOO_SMALL, OUT_OF_MEMORY, CUDA, INTERNAL. */
 mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream, int64_t* opt_cost);
 
+/* Staged solve: the same computation as mpt_solve in resumable pieces, for
+ * long solves (m = 31..32 runs for tens of seconds) that must yield the GPU,
+ * report progress or survive a restart.  The recurrence runs in steps that
+ * each depend only on earlier ones (Sec. 3.1 layers: one step per tile layer
+ * |T| = 0 .. m - b of the blocked kernels, or the singletons and one step per
+ * subset size of the general kernels); mpt_solve_steps gives their number.
+ *   mpt_solve_begin:  input copies, K1, K2 and step 0;
+ *   mpt_solve_layers: the next `count` steps (fewer at the end); *next_step
+ *                     (may be NULL) receives the index of the next step;
+ *   mpt_solve_end:    after the last step: the layout walk and OPT, as
+ *                     mpt_solve (then mpt_tables / mpt_layout apply).
+ * Every call enqueues its work on `stream` and returns (mpt_solve_end
+ * synchronises it).  Between calls the workspace holds the whole state: once
+ * the stream is idle, a copy of its mpt_workspace_bytes() bytes is a
+ * checkpoint.  To resume, copy it back into a workspace (any 256-byte-aligned
+ * device buffer of that size) and call mpt_solve_resume with the step the
+ * checkpoint had reached, on a context created from the same instance with
+ * the same DP mode.  All three step calls must name the same workspace
+ * (NULL: the context's own, for begin, layers and end only).
+ * Errors: INVALID_ARG (wrong workspace, step out of range), NOT_SOLVED (no
+ * staged solve begun, or steps left before mpt_solve_end), and those of
+ * mpt_solve. */
+mpt_status mpt_solve_steps(const mpt_ctx* ctx, int32_t* steps);
+mpt_status mpt_solve_begin(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream);
+mpt_status mpt_solve_layers(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream, int32_t count,
+                            int32_t* next_step);
+mpt_status mpt_solve_end(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream, int64_t* opt_cost);
+mpt_status mpt_solve_resume(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, int32_t next_step);
+
 /* Device views (length 2^m, indexed by subset mask S) of the last solve:
  *   F[S]     = the recurrence value (F[0] = 0),
  *   wI[S]    = w(I(S)); wI[0] = weight of the union of all requests,

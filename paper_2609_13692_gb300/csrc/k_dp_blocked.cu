@@ -634,7 +634,7 @@ int64_t blocked_partial_entries(int m, int b) {
 int blocked_max_launches(const Shape& s) { return 2 * (s.L + 1); }
 
 cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
-                              BlockedTiming* timing) {
+                              BlockedTiming* timing, int step_begin, int step_end) {
   static bool attr_done = false;
   if (!attr_done) {
     cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
@@ -645,7 +645,8 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
   }
   const int b = s.b, L = s.L;
   constexpr unsigned long long evals_per_pair = 531441ull;  // 3^12 splits per pair of windows
-  for (int kh = 0; kh <= L; ++kh) {
+  if (step_end < 0 || step_end > L + 1) step_end = L + 1;
+  for (int kh = step_begin < 0 ? 0 : step_begin; kh < step_end; ++kh) {
     const unsigned long long tiles = h_binom.v[L][kh];
     if (kh >= 2) {
       const uint32_t P = (1u << (kh - 1)) - 1u;

@@ -106,12 +106,21 @@ k_dp_layer_warp(int m, int k, unsigned long long count, const int64_t* __restric
 
 }  // namespace
 
-cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
-  k_dp_init<<<1, 32, 0, stream>>>(s.m, ws.wI, ws.F, ws.split);
-  ++*launches;
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
-  for (int k = 2; k <= s.m; ++k) {
+int dp_steps(const Shape& s) { return s.blocked ? s.L + 1 : s.m; }
+
+cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                              int step_begin, int step_end) {
+  if (step_end < 0 || step_end > s.m) step_end = s.m;
+  cudaError_t err = cudaSuccess;
+  if (step_begin <= 0 && step_end > 0) {
+    k_dp_init<<<1, 32, 0, stream>>>(s.m, ws.wI, ws.F, ws.split);
+    ++*launches;
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+  }
+  // step j >= 1 is the layer of (j + 1)-request subsets
+  const int k_begin = step_begin < 1 ? 2 : step_begin + 1;
+  for (int k = k_begin; k <= step_end; ++k) {
     const unsigned long long count = h_binom.v[s.m][k];
     if (k <= kThreadMaxLayer) {
       const unsigned long long blocks = (count + kThreads - 1) / kThreads;

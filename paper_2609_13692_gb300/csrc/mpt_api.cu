@@ -30,6 +30,8 @@ struct mpt_ctx {
   std::vector<cudaEvent_t> events;
   mpt::Workspace ws{};  // carve-up of the last successful solve
   char* resident = nullptr;  // workspace whose input copies hold this context's instance
+  int32_t staged_next = -1;  // staged solve: next step of the recurrence (-1: none begun)
+  char* staged_base = nullptr;  // staged solve: its workspace
 };
 
 namespace {
@@ -180,6 +182,7 @@ mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode) {
   ctx->mode = mode;
   refresh_shape(ctx);
   ctx->solved = false;
+  ctx->staged_next = -1;
   ctx->resident = nullptr;  // the carve-up may move the input copies
   return MPT_OK;
 }
@@ -203,21 +206,17 @@ static float elapsed(cudaEvent_t a, cudaEvent_t b) {
   return ms;
 }
 
-mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream_ptr, int64_t* opt_cost) {
-  mpt_ctx* c = ctx;
-  if (!c || !opt_cost) return MPT_ERR_INVALID_ARG;
-  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
-  const mpt::Shape& s = c->shape;
-  c->solved = false;
-  c->err.clear();
+namespace {
 
-  mpt::Workspace ws{};
-  const size_t need = mpt::carve_workspace(s, nullptr, &ws);
-  char* base = nullptr;
+// Resolve the workspace of a solve (the caller's, or one the context owns)
+// and carve it.
+mpt_status bind_workspace(mpt_ctx* c, void* d_workspace, size_t workspace_bytes, mpt::Workspace* ws, char** base) {
+  const mpt::Shape& s = c->shape;
+  const size_t need = mpt::carve_workspace(s, nullptr, ws);
   if (d_workspace) {
     if (workspace_bytes < need) return MPT_ERR_WORKSPACE_TOO_SMALL;
     if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return MPT_ERR_INVALID_ARG;
-    base = static_cast<char*>(d_workspace);
+    *base = static_cast<char*>(d_workspace);
   } else {
     if (c->own_bytes < need) {
       if (c->own_ws) cudaFree(c->own_ws);
@@ -227,26 +226,19 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
       MPT_CK(cudaMalloc(&c->own_ws, need), "cudaMalloc(workspace)");
       c->own_bytes = need;
     }
-    base = static_cast<char*>(c->own_ws);
+    *base = static_cast<char*>(c->own_ws);
   }
-  mpt::carve_workspace(s, base, &ws);
+  mpt::carve_workspace(s, *base, ws);
+  return MPT_OK;
+}
 
-  // events: 7 stage marks + 2 per blocked-DP launch
-  const int dp_launches = mpt::blocked_max_launches(s);
-  const size_t n_events = 7 + 4 * (size_t)dp_launches;
-  if (c->profiling && c->events.size() < n_events) {
-    while (c->events.size() < n_events) {
-      cudaEvent_t e;
-      MPT_CK(cudaEventCreate(&e), "cudaEventCreate");
-      c->events.push_back(e);
-    }
-  }
-  cudaEvent_t* ev = c->profiling ? c->events.data() : nullptr;
+// Input copies (unless this workspace already holds them), K1 and K2.
+mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStream_t stream, int* launches,
+                     cudaEvent_t* ev) {
+  const mpt::Shape& s = c->shape;
   auto mark = [&](int i) {
     if (ev) cudaEventRecord(ev[i], stream);
   };
-
-  int launches = 0;
   const size_t N = (size_t)1 << s.m;
   mark(0);
   if (c->resident != base) {
@@ -257,22 +249,34 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
   MPT_CK(cudaMemsetAsync(ws.counters, 0, 8 * 4, stream), "memset counters");
   MPT_CK(cudaMemsetAsync(ws.wI, 0, N * 8, stream), "memset g");
   mark(1);
-  MPT_CK(mpt::launch_scatter(s, ws, stream, &launches), "scatter kernel");
+  MPT_CK(mpt::launch_scatter(s, ws, stream, launches), "scatter kernel");
   mark(2);
-  MPT_CK(mpt::launch_zeta(s, ws, stream, &launches), "zeta kernels");
+  MPT_CK(mpt::launch_zeta(s, ws, stream, launches), "zeta kernels");
   mark(3);
-  mpt::BlockedTiming timing{};
-  if (s.blocked) {
-    timing.pair_ev = ev ? ev + 7 : nullptr;
-    timing.tile_ev = ev ? ev + 7 + 2 * dp_launches : nullptr;
-    MPT_CK(mpt::launch_dp_blocked(s, ws, stream, &launches, &timing), "blocked DP kernels");
-  } else {
-    MPT_CK(mpt::launch_dp_general(s, ws, stream, &launches), "general DP kernels");
-  }
-  mark(4);
-  MPT_CK(mpt::launch_walk(s, ws, stream, &launches), "walk kernel");
-  mark(5);
+  return MPT_OK;
+}
 
+// Steps [begin, end) of the recurrence.
+mpt_status run_steps(mpt_ctx* c, const mpt::Workspace& ws, cudaStream_t stream, int* launches,
+                     mpt::BlockedTiming* timing, int begin, int end) {
+  const mpt::Shape& s = c->shape;
+  if (s.blocked) {
+    MPT_CK(mpt::launch_dp_blocked(s, ws, stream, launches, timing, begin, end), "blocked DP kernels");
+  } else {
+    MPT_CK(mpt::launch_dp_general(s, ws, stream, launches, begin, end), "general DP kernels");
+  }
+  return MPT_OK;
+}
+
+// The walk, the copies of its results and the consistency flags.
+mpt_status run_back(mpt_ctx* c, const mpt::Workspace& ws, cudaStream_t stream, int* launches, cudaEvent_t* ev,
+                    int64_t* opt_out) {
+  const mpt::Shape& s = c->shape;
+  auto mark = [&](int i) {
+    if (ev) cudaEventRecord(ev[i], stream);
+  };
+  MPT_CK(mpt::launch_walk(s, ws, stream, launches), "walk kernel");
+  mark(5);
   int32_t counters[8];
   int64_t opt = 0;
   const size_t slots = (size_t)s.slots;
@@ -293,13 +297,56 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
   MPT_CK(cudaMemcpyAsync(c->h_dfs.data(), ws.dfs, (size_t)s.m * 4, cudaMemcpyDeviceToHost, stream), "copy dfs");
   mark(6);
   MPT_CK(cudaStreamSynchronize(stream), "solve");
-
   if (counters[1] != 0) {
     char buf[128];
     std::snprintf(buf, sizeof(buf), "device consistency flags 0x%x", counters[1]);
     c->err = buf;
     return MPT_ERR_INTERNAL;
   }
+  *opt_out = opt;
+  return MPT_OK;
+}
+
+}  // namespace
+
+mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream_ptr, int64_t* opt_cost) {
+  mpt_ctx* c = ctx;
+  if (!c || !opt_cost) return MPT_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
+  const mpt::Shape& s = c->shape;
+  c->solved = false;
+  c->staged_next = -1;
+  c->err.clear();
+
+  mpt::Workspace ws{};
+  char* base = nullptr;
+  mpt_status st = bind_workspace(c, d_workspace, workspace_bytes, &ws, &base);
+  if (st != MPT_OK) return st;
+
+  // events: 7 stage marks + 2 per blocked-DP launch
+  const int dp_launches = mpt::blocked_max_launches(s);
+  const size_t n_events = 7 + 4 * (size_t)dp_launches;
+  if (c->profiling && c->events.size() < n_events) {
+    while (c->events.size() < n_events) {
+      cudaEvent_t e;
+      MPT_CK(cudaEventCreate(&e), "cudaEventCreate");
+      c->events.push_back(e);
+    }
+  }
+  cudaEvent_t* ev = c->profiling ? c->events.data() : nullptr;
+
+  int launches = 0;
+  const size_t N = (size_t)1 << s.m;
+  if ((st = run_front(c, ws, base, stream, &launches, ev)) != MPT_OK) return st;
+  mpt::BlockedTiming timing{};
+  if (s.blocked) {
+    timing.pair_ev = ev ? ev + 7 : nullptr;
+    timing.tile_ev = ev ? ev + 7 + 2 * dp_launches : nullptr;
+  }
+  if ((st = run_steps(c, ws, stream, &launches, &timing, 0, -1)) != MPT_OK) return st;
+  if (ev) cudaEventRecord(ev[4], stream);
+  int64_t opt = 0;
+  if ((st = run_back(c, ws, stream, &launches, ev, &opt)) != MPT_OK) return st;
   c->ws = ws;
   c->opt = opt;
   c->resident = base;
@@ -330,6 +377,89 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
     p.ms_walk = elapsed(ev[4], ev[5]);
     p.ms_d2h = elapsed(ev[5], ev[6]);
   }
+  c->solved = true;
+  *opt_cost = opt;
+  return MPT_OK;
+}
+
+mpt_status mpt_solve_steps(const mpt_ctx* ctx, int32_t* steps) {
+  if (!ctx || !steps) return MPT_ERR_INVALID_ARG;
+  *steps = mpt::dp_steps(ctx->shape);
+  return MPT_OK;
+}
+
+mpt_status mpt_solve_begin(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream_ptr) {
+  mpt_ctx* c = ctx;
+  if (!c) return MPT_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
+  c->solved = false;
+  c->staged_next = -1;
+  c->err.clear();
+  mpt::Workspace ws{};
+  char* base = nullptr;
+  mpt_status st = bind_workspace(c, d_workspace, workspace_bytes, &ws, &base);
+  if (st != MPT_OK) return st;
+  int launches = 0;
+  if ((st = run_front(c, ws, base, stream, &launches, nullptr)) != MPT_OK) return st;
+  if ((st = run_steps(c, ws, stream, &launches, nullptr, 0, 1)) != MPT_OK) return st;
+  c->resident = base;
+  c->staged_base = base;
+  c->staged_next = 1;
+  return MPT_OK;
+}
+
+mpt_status mpt_solve_resume(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, int32_t next_step) {
+  mpt_ctx* c = ctx;
+  if (!c || !d_workspace) return MPT_ERR_INVALID_ARG;
+  if (next_step < 1 || next_step > mpt::dp_steps(c->shape)) return MPT_ERR_INVALID_ARG;
+  mpt::Workspace ws{};
+  char* base = nullptr;
+  mpt_status st = bind_workspace(c, d_workspace, workspace_bytes, &ws, &base);
+  if (st != MPT_OK) return st;
+  c->solved = false;
+  c->resident = base;  // a checkpoint carries the input copies with it
+  c->staged_base = base;
+  c->staged_next = next_step;
+  return MPT_OK;
+}
+
+mpt_status mpt_solve_layers(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream_ptr, int32_t count,
+                            int32_t* next_step) {
+  mpt_ctx* c = ctx;
+  if (!c || count < 0) return MPT_ERR_INVALID_ARG;
+  if (c->staged_next < 0) return MPT_ERR_NOT_SOLVED;
+  mpt::Workspace ws{};
+  char* base = nullptr;
+  mpt_status st = bind_workspace(c, d_workspace, workspace_bytes, &ws, &base);
+  if (st != MPT_OK) return st;
+  if (base != c->staged_base) return MPT_ERR_INVALID_ARG;
+  const int total = mpt::dp_steps(c->shape);
+  const int end = c->staged_next + count < total ? c->staged_next + count : total;
+  int launches = 0;
+  if ((st = run_steps(c, ws, reinterpret_cast<cudaStream_t>(stream_ptr), &launches, nullptr, c->staged_next, end)) !=
+      MPT_OK)
+    return st;
+  c->staged_next = end;
+  if (next_step) *next_step = end;
+  return MPT_OK;
+}
+
+mpt_status mpt_solve_end(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, void* stream_ptr, int64_t* opt_cost) {
+  mpt_ctx* c = ctx;
+  if (!c || !opt_cost) return MPT_ERR_INVALID_ARG;
+  if (c->staged_next < 0 || c->staged_next != mpt::dp_steps(c->shape)) return MPT_ERR_NOT_SOLVED;
+  mpt::Workspace ws{};
+  char* base = nullptr;
+  mpt_status st = bind_workspace(c, d_workspace, workspace_bytes, &ws, &base);
+  if (st != MPT_OK) return st;
+  if (base != c->staged_base) return MPT_ERR_INVALID_ARG;
+  int launches = 0;
+  int64_t opt = 0;
+  if ((st = run_back(c, ws, reinterpret_cast<cudaStream_t>(stream_ptr), &launches, nullptr, &opt)) != MPT_OK) return st;
+  c->ws = ws;
+  c->opt = opt;
+  c->staged_next = -1;
+  std::memset(&c->prof, 0, sizeof(c->prof));
   c->solved = true;
   *opt_cost = opt;
   return MPT_OK;

@@ -125,7 +125,13 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws);
 cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
 cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
 
-cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+// The recurrence runs in steps that depend only on earlier steps: the blocked
+// path has one step per tile layer |T| = 0..L, the general path one for the
+// singletons and one per popcount layer 2..m.  Launchers run steps
+// [step_begin, step_end) (step_end < 0: to the last).
+int dp_steps(const Shape& s);
+cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                              int step_begin = 0, int step_end = -1);
 
 struct BlockedTiming {
   cudaEvent_t* pair_ev;  // 2 per pair-kernel launch (start, stop), or nullptr
@@ -136,7 +142,7 @@ struct BlockedTiming {
 };
 int blocked_max_launches(const Shape& s);  // upper bound on pair + tile launches
 cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
-                              BlockedTiming* timing);
+                              BlockedTiming* timing, int step_begin = 0, int step_end = -1);
 int64_t blocked_partial_entries(int m, int b);
 int blocked_tile_bits(int m);
 

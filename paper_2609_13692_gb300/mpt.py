@@ -41,7 +41,8 @@ EXPORTED = [
     "mpt_layout", "mpt_trie_cost", "mpt_set_profiling", "mpt_get_profile", "mpt_destroy", "mpt_status_string",
     "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
     "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
-    "mpt_cache_costs", "mpt_layout_pinned",
+    "mpt_cache_costs", "mpt_layout_pinned", "mpt_solve_steps", "mpt_solve_begin", "mpt_solve_layers",
+    "mpt_solve_end", "mpt_solve_resume",
 ]
 
 
@@ -120,6 +121,11 @@ def load() -> ctypes.CDLL:
         "mpt_serve_order": ([i64, i32, i64p, i64p, i32p, i32, vp, i32p], ctypes.c_int),
         "mpt_cache_costs": ([i64p, i64, i32, i64p, i64p, i32p, i64p, i32, vp, i64p, i64p], ctypes.c_int),
         "mpt_layout_pinned": ([i64p, i64, i32, i64p, i64p, i32, i32, vp, i64p, i32p, i64p], ctypes.c_int),
+        "mpt_solve_steps": ([vp, i32p], ctypes.c_int),
+        "mpt_solve_begin": ([vp, vp, sz, vp], ctypes.c_int),
+        "mpt_solve_layers": ([vp, vp, sz, vp, i32, i32p], ctypes.c_int),
+        "mpt_solve_end": ([vp, vp, sz, vp, i64p], ctypes.c_int),
+        "mpt_solve_resume": ([vp, vp, sz, i32], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -219,6 +225,60 @@ def mpt_solve(ctx: Context, workspace=None, stream: Optional[int] = None) -> int
                             ctypes.c_void_p(s), ctypes.byref(opt)), "mpt_solve", ctx)
     ctx._solved_ws = workspace
     return int(opt.value)
+
+
+def _workspace_for(ctx: Context, workspace):
+    import torch
+
+    need = mpt_workspace_bytes(ctx)
+    if workspace is None:
+        if ctx.workspace is None or ctx.workspace.numel() < need:
+            ctx.workspace = torch.empty(need, dtype=torch.uint8, device="cuda")
+        workspace = ctx.workspace
+    if not (workspace.is_cuda and workspace.dtype == torch.uint8 and workspace.is_contiguous()):
+        raise ValueError("workspace must be a contiguous CUDA uint8 tensor")
+    return workspace
+
+
+def mpt_solve_steps(ctx: Context) -> int:
+    """Number of steps of the recurrence (see mpt_solve_begin)."""
+    n = ctypes.c_int32()
+    _check(load().mpt_solve_steps(ctx.handle, ctypes.byref(n)), "mpt_solve_steps", ctx)
+    return int(n.value)
+
+
+def mpt_solve_begin(ctx: Context, workspace=None, stream: Optional[int] = None):
+    """Start a staged solve; returns the workspace tensor it runs in."""
+    ws = _workspace_for(ctx, workspace)
+    s = _default_stream_ptr() if stream is None else int(stream)
+    _check(load().mpt_solve_begin(ctx.handle, ctypes.c_void_p(ws.data_ptr()), ws.numel(), ctypes.c_void_p(s)),
+           "mpt_solve_begin", ctx)
+    return ws
+
+
+def mpt_solve_layers(ctx: Context, workspace, count: int, stream: Optional[int] = None) -> int:
+    """Run the next ``count`` steps in ``workspace``; returns the next step."""
+    s = _default_stream_ptr() if stream is None else int(stream)
+    nxt = ctypes.c_int32()
+    _check(load().mpt_solve_layers(ctx.handle, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                   ctypes.c_void_p(s), int(count), ctypes.byref(nxt)), "mpt_solve_layers", ctx)
+    return int(nxt.value)
+
+
+def mpt_solve_end(ctx: Context, workspace, stream: Optional[int] = None) -> int:
+    """Finish a staged solve (layout walk); returns OPT."""
+    s = _default_stream_ptr() if stream is None else int(stream)
+    opt = ctypes.c_int64()
+    _check(load().mpt_solve_end(ctx.handle, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                ctypes.c_void_p(s), ctypes.byref(opt)), "mpt_solve_end", ctx)
+    ctx._solved_ws = workspace
+    return int(opt.value)
+
+
+def mpt_solve_resume(ctx: Context, workspace, next_step: int) -> None:
+    """Continue a staged solve from a checkpoint restored into ``workspace``."""
+    _check(load().mpt_solve_resume(ctx.handle, ctypes.c_void_p(workspace.data_ptr()), workspace.numel(),
+                                   int(next_step)), "mpt_solve_resume", ctx)
 
 
 def mpt_tables(ctx: Context):

@@ -177,3 +177,24 @@ def test_schedule_and_cache_validation(mpt):
     assert pinned_status(2, offs, np.array([0, 0, 4]), 0, 0) == 1      # repeated chunk in a request
     o33 = np.arange(34, dtype=np.int64) % 3
     assert pinned_status(33, np.arange(34, dtype=np.int64), o33, 0, 0) == 2  # exact method beyond 32
+
+
+def test_staged_solve_host_checks(mpt):
+    """Step counts and the state checks of the staged solve need no GPU."""
+    import ctypes
+
+    lib = mpt.load()
+    inst = I.random_instance(14, 40, 3, seed=2)
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    n = ctypes.c_int32()
+    assert lib.mpt_solve_steps(ctx.handle, ctypes.byref(n)) == 0 and n.value == 3  # tile layers 0..2
+    mpt.mpt_set_dp_mode(ctx, "general")
+    assert lib.mpt_solve_steps(ctx.handle, ctypes.byref(n)) == 0 and n.value == 14  # singletons + sizes 2..14
+    opt = ctypes.c_int64()
+    assert lib.mpt_solve_layers(ctx.handle, None, 0, None, 1, None) == 7  # nothing begun
+    assert lib.mpt_solve_end(ctx.handle, None, 0, None, ctypes.byref(opt)) == 7
+    fake = ctypes.c_void_p(1 << 20)
+    assert lib.mpt_solve_resume(ctx.handle, fake, 1 << 30, 0) == 1  # step 0 is not resumable
+    assert lib.mpt_solve_resume(ctx.handle, fake, 1 << 30, 15) == 1  # past the last step
+    assert lib.mpt_solve_resume(ctx.handle, None, 1 << 30, 1) == 1  # needs a workspace
+    mpt.mpt_destroy(ctx)
