@@ -248,6 +248,8 @@ def run_ours(args):
     ctx = mpt.mpt_create(inst.weights, inst.bits)
     if args.dp_mode != "auto":
         mpt.mpt_set_dp_mode(ctx, args.dp_mode)
+    if args.tables != "int64":
+        mpt.mpt_set_tables(ctx, args.tables)
     mpt.mpt_set_profiling(ctx, True)
     ws = torch.empty(mpt.mpt_workspace_bytes(ctx), dtype=torch.uint8, device=device)
     stream = torch.cuda.current_stream()
@@ -293,6 +295,8 @@ def run_ours(args):
         c2 = mpt.mpt_create(inst.weights, inst.bits)
         if args.dp_mode != "auto":
             mpt.mpt_set_dp_mode(c2, args.dp_mode)
+        if args.tables != "int64":
+            mpt.mpt_set_tables(c2, args.tables)
         mpt.mpt_solve(c2, ws, stream.cuda_stream)
         offs, chunks, dfs = mpt.mpt_layout(c2)
         mpt.mpt_destroy(c2)
@@ -350,10 +354,11 @@ def run_ours(args):
         "solve_time_s": solve_s,
         "config": {"workload": instances.CONFIG_NAMES[args.workload], "m": m, "n": inst.n,
                    "k": instances.CONFIGS[args.workload].get("k", m - 1), "seed": replica_seed(rank),
-                   "splits_per_solve": splits, "dp_mode": dp_mode,
+                   "splits_per_solve": splits, "dp_mode": dp_mode, "tables": args.tables,
+                   "workspace_gib": round(ws.numel() / 2**30, 2),
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "l2": f"inputs larger than L2: the 2^{m}-entry tables span {(1 << m) * 28 / 2**30:.2f} GiB "
-                         "(L2 129 MB), no flush",
+                   "l2": f"inputs larger than L2: the 2^{m}-entry tables span "
+                         f"{(1 << m) * (16 if args.tables == 'lean' else 28) / 2**30:.2f} GiB (L2 129 MB), no flush",
                    "opt": opts[-1] if opts else None},
         "roofline": roofline,
         "gather_roofline_frac": gather_frac,
@@ -551,6 +556,8 @@ def main():
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tables", choices=["int64", "lean"], default="int64",
+                    help="table layout of the exact solve (lean: one int32 table, F over w(I))")
     ap.add_argument("--mode", choices=["solve", "batch", "greedy", "cache"], default="solve",
                     help="solve: the m = 28 exact solve (default); batch: many small request groups; "
                          "greedy: agglomerative hierarchy on a trace-sized request set; "

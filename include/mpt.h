@@ -109,7 +109,7 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
  * checkpoint.  To resume, copy it back into a workspace (any 256-byte-aligned
  * device buffer of that size) and call mpt_solve_resume with the step the
  * checkpoint had reached, on a context created from the same instance with
- * the same DP mode.  All three step calls must name the same workspace
+ * the same DP mode and table layout.  All three step calls must name the same workspace
  * (NULL: the context's own, for begin, layers and end only).
  * Errors: INVALID_ARG (wrong workspace, step out of range), NOT_SOLVED (no
  * staged solve begun, or steps left before mpt_solve_end), and those of
@@ -126,8 +126,28 @@ mpt_status mpt_solve_resume(mpt_ctx* ctx, void* d_workspace, size_t workspace_by
  *   wI[S]    = w(I(S)); wI[0] = weight of the union of all requests,
  *   split[S] = the reported optimal split (see conventions).
  * The pointers live in the workspace and stay valid until the next solve or
- * mpt_destroy.  Any argument may be NULL.  Errors: INVALID_ARG, NOT_SOLVED. */
+ * mpt_destroy.  Any argument may be NULL.  Errors: INVALID_ARG (also when
+ * the context uses MPT_TABLES_LEAN: see mpt_tables32), NOT_SOLVED. */
 mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split);
+
+/* Table layout of the solve (Sec. 3.1 tables; N3 "leaner" form).
+ *   MPT_TABLES_INT64 (default): w(I(S)) and F(S) in separate int64[2^m]
+ *     tables (mpt_tables);
+ *   MPT_TABLES_LEAN: one int32[2^m] table that holds w(I(S)) after K2 and
+ *     F(S) once the recurrence has finished S (each entry is overwritten in
+ *     place by the thread that finishes it), read with mpt_tables32; w(I(S))
+ *     is then no longer available.  Allowed when sum_i w(R_i) < 2^31
+ *     (MPT_ERR_OVERFLOW otherwise), which bounds every w(I(S)) and F(S).
+ *     The blocked path's workspace falls from 28 to 16 bytes per subset
+ *     (m = 32: 64 GiB instead of 112 GiB).
+ * Changing the layout discards the last solve.  Errors: INVALID_ARG, OVERFLOW. */
+#define MPT_TABLES_INT64 0
+#define MPT_TABLES_LEAN 1
+mpt_status mpt_set_tables(mpt_ctx* ctx, int32_t kind);
+
+/* Device views of the lean tables of the last solve: F int32[2^m] and split
+ * uint32[2^m] (as in mpt_tables).  Errors: INVALID_ARG (not lean), NOT_SOLVED. */
+mpt_status mpt_tables32(const mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split);
 
 /* Number of entries mpt_layout writes to perm_chunks: sum_i |R_i|. */
 mpt_status mpt_layout_size(const mpt_ctx* ctx, int64_t* total_chunks);

@@ -368,9 +368,20 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
 // by level in |U|, folding in the self pair (kh >= 1) or running the whole
 // recurrence on the inner bits (kh = 0).  One block per tile.  Used for tile 0
 // (any b <= 12); the tiles with kh >= 1 go to k_dp_tile_rows.
+// Tab: int64 tables, or the int32 lean table (wI and F the same array: every
+// entry's w(I(S)) is read before its F(S) is written, by the same block).
+template <typename Tab>
+__device__ __forceinline__ int64_t load_wI(const Tab* p) {
+  if constexpr (sizeof(Tab) == 8)
+    return __ldg(p);
+  else
+    return (int64_t)*p;  // lean: the same array is written by this kernel
+}
+
+template <typename Tab>
 __global__ void __launch_bounds__(kTileThreads)
-k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned long long* __restrict__ partial,
-          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, int64_t* __restrict__ F, uint32_t* __restrict__ split) {
+k_dp_tile(int L, int b, int kh, const Tab* wI, const unsigned long long* __restrict__ partial,
+          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, Tab* F, uint32_t* __restrict__ split) {
   __shared__ uint32_t cur_p[1 << kMaxTileBits];   // this tile, F << b
   __shared__ uint32_t other_c[1 << kMaxTileBits]; // complement form: this tile (kh = 0) or tile 0 (kh >= 1)
   __shared__ uint16_t order[1 << kMaxTileBits];   // inner subsets sorted by size, then colex
@@ -449,12 +460,12 @@ k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned l
           f = 0;
           A = 0;
         } else if (single) {
-          f = wI[S];
+          f = load_wI(wI + S);
           A = 0;
         } else {
           const uint32_t key = (uint32_t)(best >> 32);
           const uint32_t Ua = (key & mask) + U - mask;
-          f = (int64_t)(key >> b) - wI[S];
+          f = (int64_t)(key >> b) - load_wI(wI + S);
           A = (Ua << L) | (uint32_t)best;
         }
         const uint32_t gp = (uint32_t)f << b;
@@ -464,7 +475,7 @@ k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned l
         const size_t idx = ((size_t)T << b) | U;
         Gp[idx] = gp;
         Gc[idx] = gc;
-        F[S] = f;
+        F[S] = (Tab)f;
         split[S] = A;
       }
     }
@@ -486,10 +497,10 @@ k_dp_tile(int L, int b, int kh, const int64_t* __restrict__ wI, const unsigned l
 constexpr int kRowsThreads = 96;
 constexpr int kRowsSmemBytes = (2 * kWin + 2 * (1 << kB)) * (int)sizeof(uint32_t);
 
+template <typename Tab>
 __global__ void __launch_bounds__(kRowsThreads)
-k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned long long* __restrict__ partial,
-               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, int64_t* __restrict__ F,
-               uint32_t* __restrict__ split) {
+k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restrict__ partial,
+               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, Tab* F, uint32_t* __restrict__ split) {
   extern __shared__ __align__(16) uint32_t smem[];
   uint32_t* cur = smem;               // this tile, F << kB, padded rows
   uint32_t* zc = smem + kWin;         // tile 0, complement form, padded rows
@@ -522,7 +533,7 @@ k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned lon
     const uint32_t s1f = finisher ? colex_unrank((unsigned long long)threadIdx.x, p1, kB1) : 0u;
     if (finisher) {
 #pragma unroll
-      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)__ldg(&wI[((size_t)((s1f << kB2) | (uint32_t)i) << L) | T]);
+      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)load_wI(wI + (((size_t)((s1f << kB2) | (uint32_t)i) << L) | T));
     }
     if (p1 >= 1) {
       // lanes per row chosen so that each lane runs at most 8 row pairs
@@ -614,7 +625,7 @@ k_dp_tile_rows(int L, int kh, const int64_t* __restrict__ wI, const unsigned lon
     Gp[tbase | (uint32_t)u] = gp;
     Gc[tbase | (uint32_t)u] = gp | (~(uint32_t)u & kMask);
     const size_t S = ((size_t)u << L) | T;
-    F[S] = (int64_t)(gp >> kB);
+    F[S] = (Tab)(gp >> kB);
     split[S] = bsplit[u];
   }
 }
@@ -639,7 +650,9 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
   if (!attr_done) {
     cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_dp_tile_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
@@ -673,10 +686,18 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches], stream);
     if (kh == 0) {
-      k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI, nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
+      if (s.lean)
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.fw, nullptr, ws.Gp, ws.Gc, ws.fw, ws.split);
+      else
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI, nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
     } else {
-      k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(
-          L, kh, ws.wI, kh >= 2 ? ws.partial : nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
+      const unsigned long long* part = kh >= 2 ? ws.partial : nullptr;
+      if (s.lean)
+        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.fw, part, ws.Gp, ws.Gc,
+                                                                                  ws.fw, ws.split);
+      else
+        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.wI, part, ws.Gp, ws.Gc,
+                                                                                  ws.F, ws.split);
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;

@@ -8,7 +8,10 @@
 // every split (16 bytes per split), so it is bound by random gathers.  It is
 // exact for any weights below the int64 limit and is used when the blocked
 // kernels' 32-bit packed keys could overflow (sum_i w(R_i) >= 2^20), or on
-// request.
+// request.  T is the table type: int64 (separate w(I) and F tables), or int32
+// for the lean table, where wI and F are the same array -- the thread that
+// finishes S reads w(I(S)) and writes F(S) over it, and F is read only at
+// finished subsets of lower layers.
 #include <climits>
 
 #include "mpt_internal.cuh"
@@ -19,7 +22,8 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kThreadMaxLayer = 9;  // layers up to 9 requests: one subset per thread
 
-__global__ void k_dp_init(int m, const int64_t* __restrict__ wI, int64_t* __restrict__ F, uint32_t* __restrict__ split) {
+template <typename T>
+__global__ void k_dp_init(int m, const T* wI, T* F, uint32_t* __restrict__ split) {
   const int i = threadIdx.x;
   if (i == 0) {
     F[0] = 0;
@@ -32,15 +36,15 @@ __global__ void k_dp_init(int m, const int64_t* __restrict__ wI, int64_t* __rest
   }
 }
 
+template <typename T>
 __device__ __forceinline__ void scan_splits(uint32_t S, uint32_t low, uint32_t fixed, uint32_t free_bits,
-                                            uint32_t rest, const int64_t* __restrict__ F, int64_t& best,
-                                            uint32_t& arg) {
+                                            uint32_t rest, const T* F, int64_t& best, uint32_t& arg) {
   uint32_t sub = 0;
   do {
     const uint32_t part = fixed | sub;
     if (part != rest) {
       const uint32_t A = low | part;
-      const int64_t c = F[A] + F[S ^ A];
+      const int64_t c = (int64_t)F[A] + (int64_t)F[S ^ A];
       if (c < best) {
         best = c;
         arg = A;
@@ -50,9 +54,9 @@ __device__ __forceinline__ void scan_splits(uint32_t S, uint32_t low, uint32_t f
   } while (sub != 0);
 }
 
+template <typename T>
 __global__ void __launch_bounds__(kThreads)
-k_dp_layer_thread(int m, int k, unsigned long long count, const int64_t* __restrict__ wI, int64_t* __restrict__ F,
-                  uint32_t* __restrict__ split) {
+k_dp_layer_thread(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split) {
   const unsigned long long idx = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= count) return;
   const uint32_t S = colex_unrank(idx, k, m);
@@ -61,16 +65,16 @@ k_dp_layer_thread(int m, int k, unsigned long long count, const int64_t* __restr
   int64_t best = LLONG_MAX;
   uint32_t arg = 0;
   scan_splits(S, low, 0u, rest, rest, F, best, arg);
-  F[S] = best - wI[S];
+  F[S] = (T)(best - (int64_t)wI[S]);
   split[S] = arg;
 }
 
 // One warp per subset: lane r takes the parts whose top five bits (within S
 // minus its lowest request) spell r; the lanes' results are merged
 // lexicographically on (value, A).
+template <typename T>
 __global__ void __launch_bounds__(kThreads)
-k_dp_layer_warp(int m, int k, unsigned long long count, const int64_t* __restrict__ wI, int64_t* __restrict__ F,
-                uint32_t* __restrict__ split) {
+k_dp_layer_warp(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split) {
   const int lane = threadIdx.x & 31;
   const unsigned long long warps = (unsigned long long)gridDim.x * (blockDim.x >> 5);
   for (unsigned long long w = (unsigned long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); w < count;
@@ -98,22 +102,19 @@ k_dp_layer_warp(int m, int k, unsigned long long count, const int64_t* __restric
       }
     }
     if (lane == 0) {
-      F[S] = best - wI[S];
+      F[S] = (T)(best - (int64_t)wI[S]);
       split[S] = arg;
     }
   }
 }
 
-}  // namespace
-
-int dp_steps(const Shape& s) { return s.blocked ? s.L + 1 : s.m; }
-
-cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
-                              int step_begin, int step_end) {
+template <typename T>
+cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, cudaStream_t stream, int* launches,
+                       int step_begin, int step_end) {
   if (step_end < 0 || step_end > s.m) step_end = s.m;
   cudaError_t err = cudaSuccess;
   if (step_begin <= 0 && step_end > 0) {
-    k_dp_init<<<1, 32, 0, stream>>>(s.m, ws.wI, ws.F, ws.split);
+    k_dp_init<<<1, 32, 0, stream>>>(s.m, wI, F, split);
     ++*launches;
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
@@ -124,18 +125,27 @@ cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t 
     const unsigned long long count = h_binom.v[s.m][k];
     if (k <= kThreadMaxLayer) {
       const unsigned long long blocks = (count + kThreads - 1) / kThreads;
-      k_dp_layer_thread<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, ws.wI, ws.F,
-                                                                   ws.split);
+      k_dp_layer_thread<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split);
     } else {
       unsigned long long blocks = (count + (kThreads / 32) - 1) / (kThreads / 32);
       if (blocks > 152ull * 16) blocks = 152ull * 16;
-      k_dp_layer_warp<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, ws.wI, ws.F, ws.split);
+      k_dp_layer_warp<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split);
     }
     ++*launches;
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
   }
   return cudaSuccess;
+}
+
+}  // namespace
+
+int dp_steps(const Shape& s) { return s.blocked ? s.L + 1 : s.m; }
+
+cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                              int step_begin, int step_end) {
+  if (s.lean) return dp_general<int32_t>(s, ws.fw, ws.fw, ws.split, stream, launches, step_begin, step_end);
+  return dp_general<int64_t>(s, ws.wI, ws.F, ws.split, stream, launches, step_begin, step_end);
 }
 
 }  // namespace mpt

@@ -1,4 +1,5 @@
-// K1: request-set scatter and K2: superset sums, giving w(I(S)) for every S.
+// K1: request-set scatter and K2: superset sums, giving w(I(S)) for every S
+// (uint64 sums, or uint32 in the lean table when sum_i w(R_i) < 2^31).
 //
 // Sec. 3 defines S_x = {i : x in R_i}; here it is the m-bit mask N_x.  A chunk
 // x lies in I(S) = intersection of R_i over i in S exactly when S is a subset
@@ -15,9 +16,11 @@ namespace {
 
 constexpr int kScatterThreads = 256;
 
+// g is uint64 (int64 tables) or uint32 (lean tables, sum_i w(R_i) < 2^31).
+template <typename G>
 __global__ void __launch_bounds__(kScatterThreads)
 k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m, int64_t words,
-          unsigned long long* __restrict__ g, uint32_t* __restrict__ used_N, int32_t* __restrict__ used_x,
+          G* __restrict__ g, uint32_t* __restrict__ used_N, int32_t* __restrict__ used_x,
           int32_t* __restrict__ counters, int64_t slots) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
@@ -26,7 +29,7 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
     uint32_t N = 0;
     for (int i = 0; i < m; ++i) N |= (uint32_t)((__ldg(&bits[(int64_t)i * words + word]) >> sh) & 1ull) << i;
     if (N) {
-      atomicAdd(&g[N], (unsigned long long)w[x]);
+      atomicAdd(&g[N], (G)w[x]);
       const int k = atomicAdd(&counters[0], 1);
       if (k < slots) {
         used_N[k] = N;
@@ -42,10 +45,11 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
 constexpr int kZetaLowBits = 12;
 constexpr int kZetaThreads = 512;
 
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_low(unsigned long long* __restrict__ g, int tb) {
-  __shared__ unsigned long long t[1 << kZetaLowBits];
+template <typename G>
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_low(G* __restrict__ g, int tb) {
+  __shared__ G t[1 << kZetaLowBits];
   const int size = 1 << tb;
-  unsigned long long* tile = g + ((size_t)blockIdx.x << tb);
+  G* tile = g + ((size_t)blockIdx.x << tb);
   for (int i = threadIdx.x; i < size; i += blockDim.x) t[i] = tile[i];
   const int half = size >> 1;
   for (int j = 0; j < tb; ++j) {
@@ -66,12 +70,13 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_low(unsigned long long* _
 constexpr int kZetaCols = 16;
 constexpr int kZetaHighBits = 8;
 
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_high(unsigned long long* __restrict__ g, int lo, int tb) {
-  __shared__ unsigned long long t[(1 << kZetaHighBits) * kZetaCols];
+template <typename G>
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_high(G* __restrict__ g, int lo, int tb) {
+  __shared__ G t[(1 << kZetaHighBits) * kZetaCols];
   const size_t col_groups = ((size_t)1 << lo) / kZetaCols;
   const size_t cg = blockIdx.x % col_groups;
   const size_t top = blockIdx.x / col_groups;
-  unsigned long long* base = g + (top << (lo + tb)) + cg * kZetaCols;
+  G* base = g + (top << (lo + tb)) + cg * kZetaCols;
   const int rows = 1 << tb;
   const int elems = rows * kZetaCols;
   for (int e = threadIdx.x; e < elems; e += blockDim.x) {
@@ -101,15 +106,20 @@ cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t str
   int64_t blocks = (s.n + kScatterThreads - 1) / kScatterThreads;
   if (blocks > 152 * 16) blocks = 152 * 16;
   if (blocks < 1) blocks = 1;
-  k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
-      ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned long long*>(ws.wI), ws.used_N, ws.used_x,
-      ws.counters, s.slots);
+  if (s.lean)
+    k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
+        ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned int*>(ws.fw), ws.used_N, ws.used_x,
+        ws.counters, s.slots);
+  else
+    k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
+        ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned long long*>(ws.wI), ws.used_N, ws.used_x,
+        ws.counters, s.slots);
   ++*launches;
   return cudaGetLastError();
 }
 
-cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
-  unsigned long long* g = reinterpret_cast<unsigned long long*>(ws.wI);
+template <typename G>
+static cudaError_t zeta(const Shape& s, G* g, cudaStream_t stream, int* launches) {
   const int tb = s.m < kZetaLowBits ? s.m : kZetaLowBits;
   const size_t low_blocks = (size_t)1 << (s.m - tb);
   k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb);
@@ -125,6 +135,11 @@ cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream
     if (err != cudaSuccess) return err;
   }
   return cudaSuccess;
+}
+
+cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
+  if (s.lean) return zeta(s, reinterpret_cast<unsigned int*>(ws.fw), stream, launches);
+  return zeta(s, reinterpret_cast<unsigned long long*>(ws.wI), stream, launches);
 }
 
 }  // namespace mpt

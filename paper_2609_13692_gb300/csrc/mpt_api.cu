@@ -18,6 +18,7 @@ struct mpt_ctx {
   std::vector<uint64_t> bits;
   int64_t sum_w = 0;  // sum_i w(R_i)
   int32_t mode = MPT_DP_AUTO;
+  int32_t tables = MPT_TABLES_INT64;
   void* own_ws = nullptr;
   size_t own_bytes = 0;
   bool solved = false;
@@ -52,6 +53,7 @@ bool use_blocked(const mpt_ctx* c) {
 void refresh_shape(mpt_ctx* c) {
   mpt::Shape& s = c->shape;
   s.blocked = use_blocked(c);
+  s.lean = c->tables == MPT_TABLES_LEAN;
   s.b = mpt::blocked_tile_bits(s.m);
   s.L = s.m - s.b;
   s.partial_entries = s.blocked ? mpt::blocked_partial_entries(s.m, s.b) : 0;
@@ -88,8 +90,14 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws) {
   ws->used_N = reinterpret_cast<uint32_t*>(take(slots * 4));
   ws->used_x = reinterpret_cast<int32_t*>(take(slots * 4));
   ws->counters = reinterpret_cast<int32_t*>(take(8 * 4));
-  ws->wI = reinterpret_cast<int64_t*>(take(N * 8));
-  ws->F = reinterpret_cast<int64_t*>(take(N * 8));
+  if (s.lean) {
+    ws->fw = reinterpret_cast<int32_t*>(take(N * 4));
+    ws->wI = ws->F = nullptr;
+  } else {
+    ws->wI = reinterpret_cast<int64_t*>(take(N * 8));
+    ws->F = reinterpret_cast<int64_t*>(take(N * 8));
+    ws->fw = nullptr;
+  }
   ws->split = reinterpret_cast<uint32_t*>(take(N * 4));
   if (s.blocked) {
     ws->Gp = reinterpret_cast<uint32_t*>(take(N * 4));
@@ -187,6 +195,17 @@ mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode) {
   return MPT_OK;
 }
 
+mpt_status mpt_set_tables(mpt_ctx* ctx, int32_t kind) {
+  if (!ctx || (kind != MPT_TABLES_INT64 && kind != MPT_TABLES_LEAN)) return MPT_ERR_INVALID_ARG;
+  if (kind == MPT_TABLES_LEAN && ctx->sum_w >= ((int64_t)1 << 31)) return MPT_ERR_OVERFLOW;
+  ctx->tables = kind;
+  refresh_shape(ctx);
+  ctx->solved = false;
+  ctx->staged_next = -1;
+  ctx->resident = nullptr;  // the carve-up moves
+  return MPT_OK;
+}
+
 mpt_status mpt_set_profiling(mpt_ctx* ctx, int32_t on) {
   if (!ctx) return MPT_ERR_INVALID_ARG;
   ctx->profiling = on != 0;
@@ -247,7 +266,10 @@ mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStrea
     MPT_CK(cudaMemcpyAsync(ws.bits, c->bits.data(), c->bits.size() * 8, cudaMemcpyHostToDevice, stream), "copy bits");
   }
   MPT_CK(cudaMemsetAsync(ws.counters, 0, 8 * 4, stream), "memset counters");
-  MPT_CK(cudaMemsetAsync(ws.wI, 0, N * 8, stream), "memset g");
+  if (s.lean)
+    MPT_CK(cudaMemsetAsync(ws.fw, 0, N * 4, stream), "memset g");
+  else
+    MPT_CK(cudaMemsetAsync(ws.wI, 0, N * 8, stream), "memset g");
   mark(1);
   MPT_CK(mpt::launch_scatter(s, ws, stream, launches), "scatter kernel");
   mark(2);
@@ -466,10 +488,18 @@ mpt_status mpt_solve_end(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes
 }
 
 mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split) {
-  if (!ctx) return MPT_ERR_INVALID_ARG;
+  if (!ctx || ctx->tables != MPT_TABLES_INT64) return MPT_ERR_INVALID_ARG;
   if (!ctx->solved) return MPT_ERR_NOT_SOLVED;
   if (d_F) *d_F = ctx->ws.F;
   if (d_wI) *d_wI = ctx->ws.wI;
+  if (d_split) *d_split = ctx->ws.split;
+  return MPT_OK;
+}
+
+mpt_status mpt_tables32(const mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split) {
+  if (!ctx || ctx->tables != MPT_TABLES_LEAN) return MPT_ERR_INVALID_ARG;
+  if (!ctx->solved) return MPT_ERR_NOT_SOLVED;
+  if (d_F) *d_F = ctx->ws.fw;
   if (d_split) *d_split = ctx->ws.split;
   return MPT_OK;
 }

@@ -90,9 +90,11 @@ struct Workspace {
   uint32_t* used_N;   // [slots]  request set N_x of each used chunk
   int32_t* used_x;    // [slots]  chunk id
   int32_t* counters;  // [8]      0: number of used chunks, 1: device error flags
-  // tables, natural subset order
-  int64_t* wI;        // [2^m]
-  int64_t* F;         // [2^m]
+  // tables, natural subset order (int64 tables: wI and F; lean: fw alone,
+  // w(I(S)) until the recurrence writes F(S) over it)
+  int64_t* wI;        // [2^m] or nullptr
+  int64_t* F;         // [2^m] or nullptr
+  int32_t* fw;        // [2^m] (lean) or nullptr
   uint32_t* split;    // [2^m]
   // blocked DP working tables, rotated order (see k_dp_blocked.cu)
   uint32_t* Gp;       // [2^m]  F << b
@@ -112,6 +114,7 @@ struct Shape {
   int64_t words;
   int64_t slots;    // sum_i |R_i|
   bool blocked;     // blocked DP tables present
+  bool lean;        // one int32 table for w(I(S)) then F(S)
   int b;            // tile bits (blocked)
   int L;            // m - b
   int64_t partial_entries;

@@ -42,7 +42,7 @@ EXPORTED = [
     "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
     "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
     "mpt_cache_costs", "mpt_layout_pinned", "mpt_solve_steps", "mpt_solve_begin", "mpt_solve_layers",
-    "mpt_solve_end", "mpt_solve_resume",
+    "mpt_solve_end", "mpt_solve_resume", "mpt_set_tables", "mpt_tables32",
 ]
 
 
@@ -126,6 +126,8 @@ def load() -> ctypes.CDLL:
         "mpt_solve_layers": ([vp, vp, sz, vp, i32, i32p], ctypes.c_int),
         "mpt_solve_end": ([vp, vp, sz, vp, i64p], ctypes.c_int),
         "mpt_solve_resume": ([vp, vp, sz, i32], ctypes.c_int),
+        "mpt_set_tables": ([vp, i32], ctypes.c_int),
+        "mpt_tables32": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp)], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -300,6 +302,34 @@ def mpt_tables(ctx: Context):
     return view(pF, 8 * N, torch.int64), view(pW, 8 * N, torch.int64), view(pS, 4 * N, torch.int32)
 
 
+TABLES = {"int64": 0, "lean": 1}
+
+
+def mpt_set_tables(ctx: Context, kind: str | int) -> None:
+    """Table layout: "int64" (default) or "lean" (one int32 table, F over w(I))."""
+    k = TABLES[kind] if isinstance(kind, str) else int(kind)
+    _check(load().mpt_set_tables(ctx.handle, k), "mpt_set_tables", ctx)
+
+
+def mpt_tables32(ctx: Context):
+    """Device views (torch tensors of length 2^m) of the lean F (int32) and split."""
+    import torch
+
+    pF, pS = ctypes.c_void_p(), ctypes.c_void_p()
+    _check(load().mpt_tables32(ctx.handle, ctypes.byref(pF), ctypes.byref(pS)), "mpt_tables32", ctx)
+    ws = ctx._solved_ws
+    base = ws.data_ptr()
+    N = 1 << ctx.m
+
+    def view(ptr, nbytes, dtype):
+        off = ptr.value - base
+        if off < 0 or off + nbytes > ws.numel():
+            raise RuntimeError("table pointer outside the workspace")
+        return ws[off:off + nbytes].view(dtype)
+
+    return view(pF, 4 * N, torch.int32), view(pS, 4 * N, torch.int32)
+
+
 def mpt_layout(ctx: Context):
     """(perm_offsets int64[m+1], perm_chunks int64[sum |R_i|], dfs_order int32[m])."""
     lib = load()
@@ -365,12 +395,14 @@ class Result:
 
 
 def solve(weights, bits, mode: str = "auto", workspace=None, stream: Optional[int] = None,
-          profile: bool = False) -> Result:
+          profile: bool = False, tables: str = "int64") -> Result:
     """Exact MPT solve of one instance: OPT, per-request permutations and the
     DFS serving order.  ``result.ctx`` keeps the device tables alive."""
     ctx = mpt_create(weights, bits)
     if mode != "auto":
         mpt_set_dp_mode(ctx, mode)
+    if tables != "int64":
+        mpt_set_tables(ctx, tables)
     if profile:
         mpt_set_profiling(ctx, True)
     opt = mpt_solve(ctx, workspace, stream)

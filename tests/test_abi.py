@@ -198,3 +198,26 @@ def test_staged_solve_host_checks(mpt):
     assert lib.mpt_solve_resume(ctx.handle, fake, 1 << 30, 15) == 1  # past the last step
     assert lib.mpt_solve_resume(ctx.handle, None, 1 << 30, 1) == 1  # needs a workspace
     mpt.mpt_destroy(ctx)
+
+
+def test_lean_tables_host_checks(mpt):
+    import ctypes
+
+    lib = mpt.load()
+    inst = I.random_instance(14, 40, 3, seed=2)
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    full = mpt.mpt_workspace_bytes(ctx)
+    assert lib.mpt_set_tables(ctx.handle, 2) == 1
+    assert lib.mpt_set_tables(ctx.handle, 1) == 0
+    lean = mpt.mpt_workspace_bytes(ctx)
+    assert full - lean == 12 * (1 << 14)  # 16 bytes of w(I) and F become 4
+    pF, pS, pW = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+    assert lib.mpt_tables(ctx.handle, ctypes.byref(pF), ctypes.byref(pW), ctypes.byref(pS)) == 1  # lean: no int64 tables
+    assert lib.mpt_tables32(ctx.handle, ctypes.byref(pF), ctypes.byref(pS)) == 7  # not solved yet
+    assert lib.mpt_set_tables(ctx.handle, 0) == 0
+    assert lib.mpt_tables32(ctx.handle, ctypes.byref(pF), ctypes.byref(pS)) == 1  # int64 layout
+    mpt.mpt_destroy(ctx)
+    heavy = I.random_instance(8, 16, 4, seed=3, wmin=1 << 27, wmax=1 << 28)  # sum_i w(R_i) >= 2^31
+    ctx = mpt.mpt_create(heavy.weights, heavy.bits)
+    assert lib.mpt_set_tables(ctx.handle, 1) == 3
+    mpt.mpt_destroy(ctx)
