@@ -5,10 +5,13 @@
 // groups of 10-15 requests; Sec. 7: real request groups of at most 13): many
 // independent groups, each small enough that its 2^m tables fit on chip.
 // Per block, in order:
-//   1. gather the instance's (chunk, request) occurrences and sort them by
-//      chunk id (bitonic sort), so that each distinct chunk x gets its
-//      request set N_x (S_x of Sec. 3) by OR-ing its run;
-//   2. g(T) = sum of w(x) over N_x = T, then superset sums: wI(S) = w(I(S));
+//   1. gather the instance's (chunk, request) occurrences into a hash table
+//      in shared memory, so that each distinct chunk x gets its request set
+//      N_x (S_x of Sec. 3) by OR-ing its requests;
+//   2. g(T) = sum of w(x) over N_x = T, then superset sums: wI(S) = w(I(S)),
+//      in the F table itself: entry S holds w(I(S)) until the recurrence
+//      finishes S and writes F(S) over it (only S's finisher reads w(I(S)),
+//      and F is read only at finished subsets of lower layers);
 //   3. the Sec. 3.1 recurrence layer by layer, F(S) = min over splits of
 //      F(A) + F(S \ A) - wI(S), the split named by its part A holding the
 //      lowest request of S and the smallest such A kept on ties;
@@ -16,7 +19,13 @@
 //      (depth of the highest node on its path inside N_x, chunk id), and the
 //      left-to-right leaf order (Thm 7).
 // Values are kept in 32 bits: the host accepts an instance only when
-// sum_i w(R_i) < 2^31, so every F and every split sum fits.
+// sum_i w(R_i) < 2^31, so every F and every split sum fits.  When also
+// sum_i w(R_i) < 2^(32-m) (the common case), the F table holds F << m and the
+// key of split A is F[A] + F[S \ A] + A = ((F(A) + F(S \ A)) << m) + A: one
+// 32-bit minimum picks the least value and, among equal values, the least A.
+// Otherwise keys are (value << 16 | A) in 64 bits.
+// The host launches one grid per instance size m (blocks indexed through a
+// list of instances), so that shared memory is sized for that m.
 #include "mpt_internal.cuh"
 
 namespace mpt {
@@ -24,108 +33,167 @@ namespace {
 
 constexpr int kBatchThreads = 256;
 
-__device__ __forceinline__ int block_exclusive_scan(int v, int* tmp) {
-  // tmp: kBatchThreads ints of shared memory
+
+// Step 1: the instance's distinct chunks cx[0..nd) (in no particular order)
+// with their request sets cN -- N_x = S_x of Sec. 3 -- through a hash table
+// in shared memory: tkey[0..2*occ_cap) (chunk id or -1) and tmask (request
+// bits), open addressing with linear probing.  The table has at least twice
+// as many slots as occurrences, so every insertion ends within `size` probes.
+__device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap, const int64_t* __restrict__ req_off,
+                            const int64_t* __restrict__ chunks, int32_t* tkey, uint32_t* tmask, int32_t* cx,
+                            uint32_t* cN, int* ndistinct_s) {
+  __shared__ int roff[16];  // the instance's request offsets, relative to o0
+  int& ndistinct = *ndistinct_s;
   const int t = threadIdx.x;
-  tmp[t] = v;
-  __syncthreads();
-  for (int off = 1; off < kBatchThreads; off <<= 1) {
-    const int add = t >= off ? tmp[t - off] : 0;
-    __syncthreads();
-    tmp[t] += add;
-    __syncthreads();
+  const int size = 2 * occ_cap;  // a power of two
+  const int lg = 31 - __clz(size);
+  if (t == 0) ndistinct = 0;
+  if (t <= m) roff[t] = (int)(req_off[r0 + t] - o0);
+  for (int h = t; h < size; h += kBatchThreads) {
+    tkey[h] = -1;
+    tmask[h] = 0;
   }
-  const int incl = tmp[t];
   __syncthreads();
-  return incl - v;
+  for (int j = t; j < occ; j += kBatchThreads) {
+    int i = 0;
+    while (roff[i + 1] <= j) ++i;  // the request whose slot range holds j
+    const int32_t x = (int32_t)chunks[o0 + j];
+    uint32_t h = lg > 0 ? ((uint32_t)x * 2654435761u) >> (32 - lg) : 0u;
+    for (int probe = 0; probe < size; ++probe) {
+      const int32_t old = atomicCAS(&tkey[h], -1, x);
+      if (old == -1 || old == x) {
+        atomicOr(&tmask[h], 1u << i);
+        break;
+      }
+      h = (h + 1u) & (uint32_t)(size - 1);
+    }
+  }
+  __syncthreads();
+  for (int h = t; h < size; h += kBatchThreads) {
+    const int32_t x = tkey[h];
+    if (x >= 0) {
+      const int u = atomicAdd(&ndistinct, 1);
+      cx[u] = x;
+      cN[u] = tmask[h];
+    }
+  }
+  __syncthreads();
+  return ndistinct;
+}
+
+// Step 4: the hierarchy walk of the Thm 1 proof from the split table
+// (split(S) for S = 0 .. 2^m - 1; shared or global), the permutations and the
+// left-to-right leaf order.  Every thread of the block calls it after the
+// split table is complete and visible.
+template <typename SplitT>
+__device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int64_t* __restrict__ req_off,
+                           const SplitT* split, unsigned long long* keys, const int32_t* cx, const uint32_t* cN,
+                           int nd, int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out,
+                           int32_t* __restrict__ status) {
+  __shared__ uint32_t anc[16][16];
+  __shared__ int leaf_depth[16], fill[16], dfs_s[16];
+  __shared__ int bad;
+  const int t = threadIdx.x;
+  const int N = 1 << m;
+  if (t < 16) {
+    fill[t] = 0;
+    leaf_depth[t] = 0;
+  }
+  if (t == 0) {
+    bad = 0;
+    uint32_t stk[32];
+    int stk_d[32];
+    int sp = 0, nleaf = 0;
+    stk[sp] = (uint32_t)N - 1u;
+    stk_d[sp] = 0;
+    ++sp;
+    while (sp > 0 && !bad) {
+      --sp;
+      const uint32_t S = stk[sp];
+      const int d = stk_d[sp];
+      for (uint32_t rr = S; rr; rr &= rr - 1) anc[__ffs(rr) - 1][d] = S;
+      if ((S & (S - 1)) == 0) {
+        const int i = __ffs(S) - 1;
+        leaf_depth[i] = d;
+        dfs_s[nleaf++] = i;
+        continue;
+      }
+      const uint32_t A = (uint32_t)split[S];
+      if (A == 0 || (A & ~S) != 0 || A == S || sp + 2 > 32) {
+        bad = 1;
+        break;
+      }
+      stk[sp] = S ^ A;
+      stk_d[sp] = d + 1;
+      ++sp;
+      stk[sp] = A;
+      stk_d[sp] = d + 1;
+      ++sp;
+    }
+  }
+  __syncthreads();
+  if (bad) {
+    if (t == 0) status[inst] = 1;
+    return;
+  }
+  if (t < m) dfs_out[r0 + t] = dfs_s[t];
+  // keys (depth, chunk id) into each request's own slot range, then rank them
+  for (int u = t; u < nd; u += kBatchThreads) {
+    const uint32_t Nx = cN[u];
+    for (uint32_t rr = Nx; rr; rr &= rr - 1) {
+      const int i = __ffs(rr) - 1;
+      int d = 0;
+      while (d < leaf_depth[i] && (anc[i][d] & ~Nx) != 0) ++d;
+      const int slot = atomicAdd(&fill[i], 1);
+      const int64_t base = req_off[r0 + i] - o0;
+      keys[base + slot] = ((unsigned long long)d << 32) | (unsigned long long)(uint32_t)cx[u];
+    }
+  }
+  __syncthreads();
+  const int lane = t & 31, warp = t >> 5;
+  for (int i = warp; i < m; i += kBatchThreads / 32) {
+    const int64_t base = req_off[r0 + i] - o0;
+    const int len = (int)(req_off[r0 + i + 1] - req_off[r0 + i]);
+    for (int j = lane; j < len; j += 32) {
+      const unsigned long long kj = keys[base + j];
+      int rank = 0;
+      for (int q = 0; q < len; ++q) rank += keys[base + q] < kj;
+      perm_out[o0 + base + rank] = (int64_t)(kj & 0xFFFFFFFFull);
+    }
+  }
+  if (t == 0) status[inst] = 0;
 }
 
 __global__ void __launch_bounds__(kBatchThreads)
 k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
               const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
-              const int64_t* __restrict__ tab_off, int occ_cap, int max_m, int64_t* __restrict__ opt_out,
+              const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list,
+              const uint8_t* __restrict__ packed_ok, int occ_cap, int max_m, int64_t* __restrict__ opt_out,
               int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out, int64_t* __restrict__ perm_out,
               int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  const int inst = blockIdx.x;
+  const int inst = inst_list[blockIdx.x];
+  const bool packed = packed_ok[inst] != 0;
   const int64_t r0 = inst_req[inst], r1 = inst_req[inst + 1];
   const int m = (int)(r1 - r0);
   const int64_t o0 = req_off[r0], o1 = req_off[r1];
   const int occ = (int)(o1 - o0);
   const int N = 1 << m;
-  int P2 = 1;
-  while (P2 < occ) P2 <<= 1;
 
   // shared layout (sized for max_m and occ_cap by the host)
   unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);  // [occ_cap] sort keys, later walk keys
-  uint32_t* wI = reinterpret_cast<uint32_t*>(keys + occ_cap);                  // [2^max_m]
-  uint32_t* F = wI + (1 << max_m);                                              // [2^max_m]
+  uint32_t* F = reinterpret_cast<uint32_t*>(keys + occ_cap);                   // [2^max_m] w(I(S)), then F(S)
+  uint32_t* wI = F;
   uint16_t* split = reinterpret_cast<uint16_t*>(F + (1 << max_m));             // [2^max_m]
   int32_t* cx = reinterpret_cast<int32_t*>(split + (1 << max_m));              // [occ_cap] distinct chunk ids
   uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                    // [occ_cap] their request sets
-  int* tmp = reinterpret_cast<int*>(cN + occ_cap);                              // [kBatchThreads]
-  __shared__ uint32_t anc[16][16];
-  __shared__ int leaf_depth[16], fill[16], dfs_s[16];
-  __shared__ int ndistinct, bad;
-
+  uint32_t* tmask = cN + occ_cap;                                                // [2 * occ_cap] hash-table masks
+  __shared__ int ndistinct;
   const int t = threadIdx.x;
-  if (t == 0) {
-    bad = 0;
-    ndistinct = 0;
-  }
-  // 1. occurrences -> sort keys (chunk id << 4 | request), padding at the end
-  for (int j = t; j < P2; j += kBatchThreads) keys[j] = ~0ull;
-  __syncthreads();
-  for (int i = 0; i < m; ++i) {
-    const int64_t a = req_off[r0 + i] - o0, b = req_off[r0 + i + 1] - o0;
-    for (int64_t j = a + t; j < b; j += kBatchThreads)
-      keys[j] = ((unsigned long long)chunks[o0 + j] << 4) | (unsigned long long)i;
-  }
-  __syncthreads();
-  for (int size = 2; size <= P2; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      for (int j = t; j < P2; j += kBatchThreads) {
-        const int p = j ^ stride;
-        if (p > j) {
-          const bool up = (j & size) == 0;
-          const unsigned long long a = keys[j], b = keys[p];
-          if ((a > b) == up) {
-            keys[j] = b;
-            keys[p] = a;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
-  // distinct chunks: run starts, their ranks, and request sets
-  for (int base = 0; base < occ; base += kBatchThreads) {
-    const int j = base + t;
-    const bool start = j < occ && (j == 0 || (keys[j] >> 4) != (keys[j - 1] >> 4));
-    const int rank = block_exclusive_scan(start ? 1 : 0, tmp);
-    const int before = ndistinct;
-    __syncthreads();
-    if (start) {
-      cx[before + rank] = (int32_t)(keys[j] >> 4);
-      cN[before + rank] = 0;
-    }
-    if (t == kBatchThreads - 1) ndistinct = before + rank + (start ? 1 : 0);
-    __syncthreads();
-  }
-  // request bits: each occurrence ORs its request into its chunk's run
-  for (int j = t; j < occ; j += kBatchThreads) {
-    // the run of occurrence j is the number of run starts at or before j, minus one
-    int lo = 0, hi = ndistinct - 1;
-    const int32_t x = (int32_t)(keys[j] >> 4);
-    while (lo < hi) {  // cx is increasing: find the entry equal to x
-      const int mid = (lo + hi) >> 1;
-      if (cx[mid] < x) lo = mid + 1; else hi = mid;
-    }
-    atomicOr(&cN[lo], 1u << (keys[j] & 15ull));
-  }
+  const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
+                              cN, &ndistinct);
   for (int S = t; S < N; S += kBatchThreads) wI[S] = 0;
   __syncthreads();
-  const int nd = ndistinct;
 
   // 2. g(T), then superset sums over the m request bits
   for (int u = t; u < nd; u += kBatchThreads) atomicAdd(&wI[cN[u]], (uint32_t)weights[cx[u]]);
@@ -139,14 +207,58 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   }
 
   // 3. the recurrence, one popcount layer at a time
+  const int vshift = packed ? m : 0;  // F holds F << vshift
   for (int S = t; S < N; S += kBatchThreads) {
     if ((S & (S - 1)) == 0) {
-      F[S] = S ? wI[S] : 0u;
+      F[S] = S ? wI[S] << vshift : 0u;
       split[S] = 0;
     }
   }
   __syncthreads();
-  for (int k = 2; k <= m; ++k) {
+  for (int k = 2; packed && k <= m; ++k) {
+    const int count = (int)c_binom.v[m][k];
+    // lanes per subset: enough to keep the block busy, at most 32; lanes
+    // split the parts on the LOWEST bits of S \ lowbit(S), so the lanes of a
+    // subset read F at different banks whenever those requests are low
+    int g = 0;
+    while ((count << (g + 1)) <= kBatchThreads && g < 5 && g < k - 1) ++g;
+    const int G = 1 << g;
+    const int per_pass = kBatchThreads >> g;
+    for (int base = 0; base < count; base += per_pass) {
+      const int idx = base + (t >> g);
+      const uint32_t r = (uint32_t)t & (uint32_t)(G - 1);
+      uint32_t best = 0xFFFFFFFFu;
+      uint32_t S = 0;
+      if (idx < count) {
+        S = colex_unrank((unsigned long long)idx, k, m);
+        const uint32_t low = S & (~S + 1u);
+        const uint32_t rest = S ^ low;
+        uint32_t lo = 0, rr = rest;
+        for (int q = 0; q < g; ++q) {
+          const uint32_t lb = rr & (~rr + 1u);
+          lo |= lb;
+          rr ^= lb;
+        }
+        const uint32_t freem = rest ^ lo;
+        const uint32_t fixed = deposit_bits(r, lo);
+        const uint32_t lowfixed = low | fixed;
+        const bool last_lane = fixed == lo;  // only this lane meets part == rest (A = S)
+        uint32_t sub = 0;
+        do {
+          const uint32_t A = lowfixed | sub;
+          if (!(last_lane && sub == freem)) best = min(best, F[A] + F[S ^ A] + A);
+          sub = (sub - freem) & freem;
+        } while (sub != 0);
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) best = min(best, __shfl_xor_sync(0xFFFFFFFFu, best, off));
+      if (idx < count && r == 0) {
+        F[S] = ((best >> m) - wI[S]) << m;
+        split[S] = (uint16_t)(best & (uint32_t)(N - 1));
+      }
+    }
+    __syncthreads();
+  }
+  for (int k = 2; !packed && k <= m; ++k) {
     const int count = (int)c_binom.v[m][k];
     // lanes per subset: enough to keep the block busy, at most 32
     int g = 0;
@@ -196,97 +308,324 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   // outputs: tables and OPT
   const int64_t tb = tab_off[inst];
   for (int S = t; S < N; S += kBatchThreads) {
-    F_out[tb + S] = (int64_t)F[S];
+    F_out[tb + S] = (int64_t)(F[S] >> vshift);
     split_out[tb + S] = split[S];
   }
-  if (t == 0) opt_out[inst] = (int64_t)F[N - 1];
+  if (t == 0) opt_out[inst] = (int64_t)(F[N - 1] >> vshift);
 
   // 4. hierarchy walk
-  if (t < 16) {
+  __syncthreads();
+  batch_walk(inst, m, r0, o0, req_off, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+}
 
-    fill[t] = 0;
-    leaf_depth[t] = 0;
+// ---------------------------------------------------------------------------
+// Row-blocked recurrence for instances with m >= 6 and packed keys.
+//
+// The 2^m subsets U = (s1, s2) are 2^(m-5) rows s1 of 32 entries s2, stored
+// at row_pos(s1) * 36 + s2 (rows padded to 36 words and XOR-placed so that
+// the 16-byte chunks of different rows fall in different bank groups).  Two
+// tables per row:
+//   Gp(X) = (F(X) << m) + X,   Gc(X) = F(X) << m,
+// so Gp(A) + Gc(B) = ((F(A) + F(B)) << m) + A: an unsigned min over splits
+// picks the least value and, among equal values, the least A.  Before U is
+// finished, Gp(U) holds w(I(U)) (superset sums in place).
+// A split of U names the part A holding lowbit(U):
+//   * s2 != 0: A = (a1, a2) with a2 holding lowbit(s2), any a1 within s1;
+//     - a1 not in {0, s1}: rows a1 and s1 ^ a1 were finished at an earlier
+//       level of |s1| -- a register convolution of two rows restricted to
+//       a2 holding lowbit(s2) (121 add-min pairs);
+//     - a1 = 0 (B in this row) and a1 = s1 (A in this row, a2 != s2): the
+//       in-row recurrence, in increasing s2, in registers;
+//   * s2 = 0: A = (a1, 0) with a1 holding lowbit(s1), a1 != s1 -- the
+//     entry-0 column of the same row pairs.
+// Levels go by |s1|; within a level, phase A (row pairs, several lanes per
+// row) then phase B (one thread per row finishes it).
+// ---------------------------------------------------------------------------
+constexpr int kBRow = 32;
+constexpr int kBRowStride = 36;
+constexpr int kBMaxLevelRows = 70;  // C(8, 4): the most rows of one level (m = 13)
+constexpr int kBkStride = kBRow + 1; // phase A minima: 33 words a row, so rows read by one warp use different banks
+static_assert((kBMaxLevelRows * kBkStride * 4) % 8 == 0, "the sort keys after the minima need 8-byte alignment");
+
+__device__ __forceinline__ int brow_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
+__device__ __forceinline__ int bidx(uint32_t U) { return brow_pos(U >> 5) * kBRowStride + (int)(U & 31u); }
+
+__device__ __forceinline__ void bload_row(uint32_t (&v)[kBRow], const uint32_t* p) {
+  const uint4* q = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+  for (int c = 0; c < kBRow / 4; ++c) {
+    const uint4 t = q[c];
+    v[4 * c] = t.x;
+    v[4 * c + 1] = t.y;
+    v[4 * c + 2] = t.z;
+    v[4 * c + 3] = t.w;
   }
+}
+
+__device__ __forceinline__ void bstore_row(uint32_t* p, const uint32_t (&v)[kBRow]) {
+  uint4* q = reinterpret_cast<uint4*>(p);
+#pragma unroll
+  for (int c = 0; c < kBRow / 4; ++c) q[c] = make_uint4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+}
+
+// acc[s2] = min over a2 within s2 holding lowbit(s2) of x[a2] + y[s2 ^ a2], s2 = 1..31
+__device__ __forceinline__ void bconv_restricted(uint32_t (&acc)[kBRow], const uint32_t (&x)[kBRow],
+                                                 const uint32_t (&y)[kBRow]) {
+#pragma unroll
+  for (int a2 = 1; a2 < kBRow; ++a2) {
+#pragma unroll
+    for (int s2 = 1; s2 < kBRow; ++s2) {
+      if ((a2 & s2) == a2 && (a2 & (s2 & -s2)) != 0) acc[s2] = min(acc[s2], x[a2] + y[s2 ^ a2]);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kBatchThreads)
+k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
+             const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
+             const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list, int occ_cap, int mm,
+             int64_t* __restrict__ opt_out, int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out,
+             int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int inst = inst_list[blockIdx.x];
+  const int64_t r0 = inst_req[inst], r1 = inst_req[inst + 1];
+  const int m = (int)(r1 - r0);  // == mm
+  const int64_t o0 = req_off[r0], o1 = req_off[r1];
+  const int occ = (int)(o1 - o0);
+  const int N = 1 << m;
+  const int nb = m - 5;
+  const int R = 1 << nb;
+  const uint32_t mask = (uint32_t)N - 1u;
+  const int64_t tb = tab_off[inst];
+
+  uint32_t* Gp = reinterpret_cast<uint32_t*>(smem_raw);                          // [R * 36]
+  uint32_t* Gc = Gp + (1 << (mm - 5)) * kBRowStride;                               // [R * 36]
+  uint32_t* bk = Gc + (1 << (mm - 5)) * kBRowStride;                               // [70 * 33] phase A minima
+  unsigned long long* keys = reinterpret_cast<unsigned long long*>(bk + kBMaxLevelRows * kBkStride);  // [occ_cap]
+  int32_t* cx = reinterpret_cast<int32_t*>(keys + occ_cap);                        // [occ_cap]
+  uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                        // [occ_cap]
+  uint32_t* tmask = cN + occ_cap;                                                  // [2 * occ_cap] hash-table masks
+  uint16_t* split = reinterpret_cast<uint16_t*>(tmask + 2 * occ_cap);              // [2^m] for the walk
+  __shared__ int ndistinct;
+  const int t = threadIdx.x;
+
+  const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
+                              cN, &ndistinct);
+
+  // g and the superset sums, in the padded row layout: the five in-row bits
+  // per row in registers, then one row-pair pass per row bit
+  for (int i = t; i < R * kBRowStride; i += kBatchThreads) Gp[i] = 0;
+  __syncthreads();
+  for (int u = t; u < nd; u += kBatchThreads) atomicAdd(&Gp[bidx(cN[u])], (uint32_t)weights[cx[u]]);
+  __syncthreads();
+  for (int r = t; r < R; r += kBatchThreads) {
+    uint32_t v[kBRow];
+    uint32_t* row = Gp + brow_pos((uint32_t)r) * kBRowStride;
+    bload_row(v, row);
+#pragma unroll
+    for (int j = 0; j < 5; ++j)
+#pragma unroll
+      for (int x = 0; x < kBRow; ++x)
+        if (!(x & (1 << j))) v[x] += v[x | (1 << j)];
+    bstore_row(row, v);
+  }
+  __syncthreads();
+  for (int jr = 0; jr < nb; ++jr) {
+    for (int p = t; p < (R >> 1); p += kBatchThreads) {
+      const uint32_t r = (uint32_t)(((p >> jr) << (jr + 1)) | (p & ((1 << jr) - 1)));
+      uint32_t v[kBRow], u[kBRow];
+      uint32_t* row = Gp + brow_pos(r) * kBRowStride;
+      bload_row(v, row);
+      bload_row(u, Gp + brow_pos(r | (1u << jr)) * kBRowStride);
+#pragma unroll
+      for (int x = 0; x < kBRow; ++x) v[x] += u[x];
+      bstore_row(row, v);
+    }
+    __syncthreads();
+  }
+
+  // level 0: row 0, the recurrence on the five low requests
   if (t == 0) {
-    uint32_t stk[32];
-    int stk_d[32];
-    int sp = 0, nleaf = 0;
-    stk[sp] = (uint32_t)N - 1u;
-    stk_d[sp] = 0;
-    ++sp;
-    while (sp > 0 && !bad) {
-      --sp;
-      const uint32_t S = stk[sp];
-      const int d = stk_d[sp];
-      for (uint32_t rr = S; rr; rr &= rr - 1) anc[__ffs(rr) - 1][d] = S;
-      if ((S & (S - 1)) == 0) {
-        const int i = __ffs(S) - 1;
-        leaf_depth[i] = d;
-        dfs_s[nleaf++] = i;
-        continue;
+    uint32_t zp[kBRow], zc[kBRow];
+#pragma unroll
+    for (int s2 = 0; s2 < kBRow; ++s2) {
+      const uint32_t wv = Gp[s2];
+      uint32_t f, A;
+      if (s2 == 0) {
+        f = 0;
+        A = 0;
+      } else if ((s2 & (s2 - 1)) == 0) {
+        f = wv;
+        A = 0;
+      } else {
+        uint32_t key = 0xFFFFFFFFu;
+#pragma unroll
+        for (int a2 = 1; a2 < kBRow; ++a2)
+          if ((a2 & s2) == a2 && (a2 & (s2 & -s2)) != 0 && a2 != s2) key = min(key, zp[a2] + zc[s2 ^ a2]);
+        f = (key >> m) - wv;
+        A = key & mask;
       }
-      const uint32_t A = split[S];
-      if (A == 0 || (A & ~S) != 0 || A == S || sp + 2 > 32) {
-        bad = 1;
-        break;
-      }
-      stk[sp] = S ^ A;
-      stk_d[sp] = d + 1;
-      ++sp;
-      stk[sp] = A;
-      stk_d[sp] = d + 1;
-      ++sp;
+      zp[s2] = (f << m) + (uint32_t)s2;
+      zc[s2] = f << m;
+      split[s2] = (uint16_t)A;
+    }
+#pragma unroll
+    for (int s2 = 0; s2 < kBRow; ++s2) {
+      Gp[s2] = zp[s2];
+      Gc[s2] = zc[s2];
     }
   }
   __syncthreads();
-  if (bad) {
-    if (t == 0) status[inst] = 1;
-    return;
-  }
-  if (t < m) dfs_out[r0 + t] = dfs_s[t];
-  // keys (depth, chunk id) into each request's own slot range, then rank them
-  for (int u = t; u < nd; u += kBatchThreads) {
-    const uint32_t Nx = cN[u];
-    for (uint32_t rr = Nx; rr; rr &= rr - 1) {
-      const int i = __ffs(rr) - 1;
-      int d = 0;
-      while (d < leaf_depth[i] && (anc[i][d] & ~Nx) != 0) ++d;
-      const int slot = atomicAdd(&fill[i], 1);
-      const int64_t base = req_off[r0 + i] - o0;
-      keys[base + slot] = ((unsigned long long)d << 32) | (unsigned long long)(uint32_t)cx[u];
+
+  for (int p1 = 1; p1 <= nb; ++p1) {
+    const int rows = (int)c_binom.v[nb][p1];
+    if (p1 >= 2) {
+      // phase A: row pairs (a1, s1 ^ a1), a1 not in {0, s1}; G lanes per row
+      const int g = p1 > 3 ? p1 - 3 : 0;
+      const int G = 1 << g;
+      const int ri = t >> g;
+      const uint32_t r = (uint32_t)t & (uint32_t)(G - 1);
+      uint32_t acc[kBRow];
+#pragma unroll
+      for (int i = 0; i < kBRow; ++i) acc[i] = 0xFFFFFFFFu;
+      if (ri < rows) {
+        const uint32_t s1 = colex_unrank((unsigned long long)ri, p1, nb);
+        const uint32_t lowb = s1 & (~s1 + 1u);
+        uint32_t hi = 0, rr = s1;
+        for (int q = 0; q < g; ++q) {
+          const uint32_t top = 1u << (31 - __clz(rr));
+          hi |= top;
+          rr ^= top;
+        }
+        const uint32_t freem = s1 ^ hi;
+        const uint32_t fixed = deposit_bits(r, hi);
+        uint32_t sub = 0;
+        do {
+          const uint32_t a1 = fixed | sub;
+          if (a1 != 0 && a1 != s1) {
+            uint32_t x[kBRow], y[kBRow];
+            bload_row(x, Gp + brow_pos(a1) * kBRowStride);
+            bload_row(y, Gc + brow_pos(s1 ^ a1) * kBRowStride);
+            bconv_restricted(acc, x, y);
+            if (a1 & lowb) acc[0] = min(acc[0], x[0] + y[0]);
+          }
+          sub = (sub - freem) & freem;
+        } while (sub != 0);
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) {
+#pragma unroll
+        for (int i = 0; i < kBRow; ++i) acc[i] = min(acc[i], __shfl_xor_sync(0xFFFFFFFFu, acc[i], off));
+      }
+      if (ri < rows && r == 0) {
+#pragma unroll
+        for (int i = 0; i < kBRow; ++i) bk[ri * kBkStride + i] = acc[i];
+      }
+      __syncthreads();
     }
+    // phase B: one thread finishes each row of the level
+    if (t < rows) {
+      const uint32_t s1 = colex_unrank((unsigned long long)t, p1, nb);
+      const uint32_t S1 = s1 << 5;
+      uint32_t* prow = Gp + brow_pos(s1) * kBRowStride;
+      uint32_t zp[kBRow], zcs[kBRow], cc[kBRow];
+      bload_row(zp, Gp);   // row 0 is at position 0
+      bload_row(zcs, Gc);
+#pragma unroll
+      for (int i = 0; i < kBRow; ++i) zcs[i] += S1;  // Gc(0, x) + (s1 << 5): the A-part of a1 = s1 splits
+#pragma unroll
+      for (int blk = 0; blk < kBRow / 8; ++blk) {
+        uint32_t wv[8], bkv[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          wv[q] = prow[blk * 8 + q];
+          bkv[q] = p1 >= 2 ? bk[t * kBkStride + blk * 8 + q] : 0xFFFFFFFFu;
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int s2 = blk * 8 + q;
+          uint32_t f, A;
+          if (s2 == 0 && p1 == 1) {  // U = (s1, 0) is a single request
+            f = wv[q];
+            A = 0;
+          } else {
+            // two independent minima (a1 = 0 and a1 = s1) shorten the chains
+            uint32_t k0 = bkv[q], k1 = 0xFFFFFFFFu;
+            if (s2 != 0) {
+#pragma unroll
+              for (int a2 = 1; a2 < kBRow; ++a2) {
+                if ((a2 & s2) == a2 && (a2 & (s2 & -s2)) != 0) {
+                  k0 = min(k0, zp[a2] + cc[s2 ^ a2]);                             // a1 = 0
+                  if (a2 != s2) k1 = min(k1, cc[a2] + zcs[s2 ^ a2] + (uint32_t)a2);  // a1 = s1
+                }
+              }
+            }
+            const uint32_t key = min(k0, k1);
+            f = (key >> m) - wv[q];
+            A = key & mask;
+          }
+          cc[s2] = f << m;
+          split[S1 | (uint32_t)s2] = (uint16_t)A;
+        }
+      }
+      uint32_t gp[kBRow];
+#pragma unroll
+      for (int i = 0; i < kBRow; ++i) gp[i] = cc[i] + (S1 | (uint32_t)i);
+      bstore_row(prow, gp);
+      bstore_row(Gc + brow_pos(s1) * kBRowStride, cc);
+    }
+    __syncthreads();
   }
+
+  // outputs: tables and OPT
+  for (int U = t; U < N; U += kBatchThreads) {
+    F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m);
+    split_out[tb + U] = split[U];
+  }
+  if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   __syncthreads();
-  const int lane = t & 31, warp = t >> 5;
-  for (int i = warp; i < m; i += kBatchThreads / 32) {
-    const int64_t base = req_off[r0 + i] - o0;
-    const int len = (int)(req_off[r0 + i + 1] - req_off[r0 + i]);
-    for (int j = lane; j < len; j += 32) {
-      const unsigned long long kj = keys[base + j];
-      int rank = 0;
-      for (int q = 0; q < len; ++q) rank += keys[base + q] < kj;
-      perm_out[o0 + base + rank] = (int64_t)(kj & 0xFFFFFFFFull);
-    }
-  }
-  if (t == 0) status[inst] = 0;
+  batch_walk(inst, m, r0, o0, req_off, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 }  // namespace
 
 size_t batch_smem_bytes(int max_m, int occ_cap) {
-  return (size_t)occ_cap * 8 + ((size_t)4 << max_m) * 2 + ((size_t)2 << max_m) + (size_t)occ_cap * 8 +
-         (size_t)kBatchThreads * 4 + 64;
+  return (size_t)occ_cap * 8 + ((size_t)4 << max_m) + ((size_t)2 << max_m) + (size_t)occ_cap * 8 +
+         (size_t)occ_cap * 8 + 64;
 }
 
-cudaError_t launch_batch(int batch, int max_m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
-                         const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off, int64_t* opt,
-                         int64_t* F, uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status,
-                         cudaStream_t stream) {
-  const size_t smem = batch_smem_bytes(max_m, occ_cap);
+// One grid over `count` instances of size m (ids inst_list[0..count)).
+cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
+                         const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
+                         const int32_t* inst_list, const uint8_t* packed_ok, int64_t* opt, int64_t* F,
+                         uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream) {
+  const size_t smem = batch_smem_bytes(m, occ_cap);
   cudaError_t e = cudaFuncSetAttribute(k_batch_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_batch_solve<<<(unsigned)batch, kBatchThreads, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off, occ_cap,
-                                                                  max_m, opt, F, split, perm, dfs, status);
+  k_batch_solve<<<(unsigned)count, kBatchThreads, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off,
+                                                                  inst_list, packed_ok, occ_cap, m, opt, F, split,
+                                                                  perm, dfs, status);
+  return cudaGetLastError();
+}
+
+size_t batch_rows_smem_bytes(int m, int occ_cap) {
+  const size_t R = (size_t)1 << (m - 5);
+  return 2 * R * kBRowStride * 4 + (size_t)kBMaxLevelRows * kBkStride * 4 + (size_t)occ_cap * 16 +
+         (size_t)occ_cap * 8 + ((size_t)2 << m) + 64;
+}
+
+// One grid of the row-blocked kernel over `count` instances of size m >= 6
+// whose request weights allow packed keys.
+cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
+                              const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
+                              const int32_t* inst_list, int64_t* opt, int64_t* F, uint32_t* split, int64_t* perm,
+                              int32_t* dfs, int32_t* status, cudaStream_t stream) {
+  if (m < 6 || m > 13) return cudaErrorInvalidValue;
+  const size_t smem = batch_rows_smem_bytes(m, occ_cap);
+  cudaError_t e = cudaFuncSetAttribute(k_batch_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_batch_rows<<<(unsigned)count, kBatchThreads, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off,
+                                                                 inst_list, occ_cap, m, opt, F, split, perm, dfs,
+                                                                 status);
   return cudaGetLastError();
 }
 

@@ -1,5 +1,6 @@
 // C ABI of the batched small-instance solver (include/mpt.h, mpt_batch_*):
-// argument checks, workspace carve-up and the one launch of k_batch_solve.
+// argument checks, workspace carve-up and one k_batch_solve launch per
+// instance size m.
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
@@ -12,10 +13,14 @@
 
 namespace mpt {
 size_t batch_smem_bytes(int max_m, int occ_cap);
-cudaError_t launch_batch(int batch, int max_m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
-                         const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off, int64_t* opt,
-                         int64_t* F, uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status,
-                         cudaStream_t stream);
+cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
+                         const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
+                         const int32_t* inst_list, const uint8_t* packed_ok, int64_t* opt, int64_t* F,
+                         uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream);
+cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
+                              const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
+                              const int32_t* inst_list, int64_t* opt, int64_t* F, uint32_t* split, int64_t* perm,
+                              int32_t* dfs, int32_t* status, cudaStream_t stream);
 }  // namespace mpt
 
 struct mpt_batch {
@@ -23,6 +28,13 @@ struct mpt_batch {
   int64_t n = 0, requests = 0, occurrences = 0, table_entries = 0;
   int max_m = 0, occ_cap = 1;
   std::vector<int64_t> w, inst_req, req_off, chunks, tab_off;
+  // instances grouped by size m: inst_list[group_start[m] .. group_start[m+1]),
+  // those for the row-blocked kernel (m >= 6, packed keys) first, up to
+  // group_rows_end[m]
+  std::vector<int32_t> inst_list;
+  std::vector<int64_t> group_start, group_rows_end;
+  std::vector<int> group_occ_cap;
+  std::vector<uint8_t> packed_ok;  // sum_i w(R_i) < 2^(32 - m): 32-bit keys
   // results of the last solve
   bool solved = false;
   std::vector<int64_t> opt, perm;
@@ -41,7 +53,8 @@ constexpr int kBatchMaxOcc = 2048;
 struct BatchCarve {
   int64_t *weights, *inst_req, *req_off, *chunks, *tab_off, *opt, *F, *perm;
   uint32_t* split;
-  int32_t *dfs, *status;
+  int32_t *dfs, *status, *inst_list;
+  uint8_t* packed_ok;
 };
 
 size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
@@ -62,6 +75,8 @@ size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
   c->perm = reinterpret_cast<int64_t*>(take((size_t)std::max<int64_t>(b->occurrences, 1) * 8));
   c->dfs = reinterpret_cast<int32_t*>(take((size_t)b->requests * 4));
   c->status = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
+  c->inst_list = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
+  c->packed_ok = reinterpret_cast<uint8_t*>(take((size_t)b->batch));
   return off;
 }
 
@@ -91,6 +106,8 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
   if (!c) return MPT_ERR_OUT_OF_MEMORY;
   try {
     c->tab_off.resize((size_t)batch + 1);
+    c->packed_ok.assign((size_t)batch, 0);
+    std::vector<int> inst_occ((size_t)batch);
     int64_t tab = 0;
     std::vector<int64_t> ids;
     for (int32_t b = 0; b < batch; ++b) {
@@ -121,8 +138,28 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
       tab += (int64_t)1 << m;
       c->max_m = std::max(c->max_m, m);
       while (c->occ_cap < occ) c->occ_cap <<= 1;
+      c->packed_ok[(size_t)b] = sum < ((int64_t)1 << (32 - m)) ? 1 : 0;
+      inst_occ[(size_t)b] = (int)occ;
     }
     c->tab_off[(size_t)batch] = tab;
+    // group the instances by m (stable), each group with its own occurrence cap
+    c->group_start.assign(kBatchMaxM + 2, 0);
+    for (int32_t b = 0; b < batch; ++b) ++c->group_start[(size_t)(inst_requests[b + 1] - inst_requests[b]) + 1];
+    for (int m = 1; m <= kBatchMaxM + 1; ++m) c->group_start[(size_t)m] += c->group_start[(size_t)m - 1];
+    c->inst_list.resize((size_t)batch);
+    c->group_occ_cap.assign(kBatchMaxM + 1, 1);
+    std::vector<int64_t> fill(c->group_start.begin(), c->group_start.end());
+    for (int pass = 0; pass < 2; ++pass) {
+      for (int32_t b = 0; b < batch; ++b) {
+        const int m = (int)(inst_requests[b + 1] - inst_requests[b]);
+        const bool rows = m >= 6 && c->packed_ok[(size_t)b];
+        if (rows != (pass == 0)) continue;
+        c->inst_list[(size_t)fill[(size_t)m]++] = b;
+        int& cap = c->group_occ_cap[(size_t)m];
+        while (cap < inst_occ[(size_t)b]) cap <<= 1;
+      }
+      if (pass == 0) c->group_rows_end.assign(fill.begin(), fill.end());
+    }
     c->table_entries = tab;
     c->w.assign(weights, weights + n_chunks);
     c->inst_req.assign(inst_requests, inst_requests + batch + 1);
@@ -190,9 +227,19 @@ mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_byt
   h2d(c.req_off, b->req_off.data(), ((size_t)b->requests + 1) * 8);
   h2d(c.chunks, b->chunks.data(), (size_t)b->occurrences * 8);
   h2d(c.tab_off, b->tab_off.data(), (B + 1) * 8);
-  if (e == cudaSuccess)
-    e = mpt::launch_batch(b->batch, b->max_m, b->occ_cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off, c.opt,
-                          c.F, c.split, c.perm, c.dfs, c.status, stream);
+  h2d(c.inst_list, b->inst_list.data(), B * 4);
+  h2d(c.packed_ok, b->packed_ok.data(), B);
+  for (int m = 1; m <= kBatchMaxM && e == cudaSuccess; ++m) {
+    const int64_t g0 = b->group_start[(size_t)m], gr = b->group_rows_end[(size_t)m],
+                  g1 = b->group_start[(size_t)m + 1];
+    const int cap = b->group_occ_cap[(size_t)m];
+    if (gr > g0)
+      e = mpt::launch_batch_rows((int)(gr - g0), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
+                                 c.inst_list + g0, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+    if (e == cudaSuccess && g1 > gr)
+      e = mpt::launch_batch((int)(g1 - gr), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
+                            c.inst_list + gr, c.packed_ok, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+  }
   d2h(b->opt.data(), c.opt, B * 8);
   d2h(b->status.data(), c.status, B * 4);
   d2h(b->perm.data(), c.perm, (size_t)b->occurrences * 8);

@@ -92,3 +92,21 @@ def test_batch_large_requests(mpt):
     """Requests of up to 150 chunks (near the 2048-occurrence limit at m = 13)."""
     weights, batch = rag_batch(40, 20000, seed=2, m_range=(10, 13), k_range=(100, 150), pool_size=400)
     check_batch(mpt, weights, batch)
+
+
+def test_batch_mixed_key_widths(mpt):
+    """Instances whose request weights need the 64-bit keys (sum_i w(R_i) >=
+    2^(32 - m)) next to ones that use the packed 32-bit keys, sizes shuffled
+    so the per-size launches must map results back to their instances."""
+    rng = np.random.default_rng(71)
+    n = 400
+    heavy = rng.integers(60_000, 120_000, size=n, dtype=np.int64)
+    batch = []
+    for _ in range(60):
+        m = int(rng.integers(2, 14))
+        batch.append([sorted(set(int(x) for x in rng.choice(n, size=int(rng.integers(1, 12)), replace=False)))
+                      for _ in range(m)])
+    sums = [sum(int(heavy[x]) for r in reqs for x in r) for reqs in batch]
+    assert any(s >= 1 << (32 - len(reqs)) for s, reqs in zip(sums, batch))
+    assert any(s < 1 << (32 - len(reqs)) for s, reqs in zip(sums, batch))
+    check_batch(mpt, heavy, batch)
