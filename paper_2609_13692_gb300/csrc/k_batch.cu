@@ -41,8 +41,7 @@ constexpr int kBatchThreads = 256;
 // as many slots as occurrences, so every insertion ends within `size` probes.
 __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap, const int64_t* __restrict__ req_off,
                             const int64_t* __restrict__ chunks, int32_t* tkey, uint32_t* tmask, int32_t* cx,
-                            uint32_t* cN, int* ndistinct_s) {
-  __shared__ int roff[16];  // the instance's request offsets, relative to o0
+                            uint32_t* cN, int* roff, int* ndistinct_s) {
   int& ndistinct = *ndistinct_s;
   const int t = threadIdx.x;
   const int size = 2 * occ_cap;  // a power of two
@@ -85,10 +84,11 @@ __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap,
 // (split(S) for S = 0 .. 2^m - 1; shared or global), the permutations and the
 // left-to-right leaf order.  Every thread of the block calls it after the
 // split table is complete and visible.
+// roff: the request offsets staged by batch_gather (shared memory).
 template <typename SplitT>
-__device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int64_t* __restrict__ req_off,
-                           const SplitT* split, unsigned long long* keys, const int32_t* cx, const uint32_t* cN,
-                           int nd, int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out,
+__device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int* roff, const SplitT* split,
+                           unsigned long long* keys, const int32_t* cx, const uint32_t* cN, int nd,
+                           int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out,
                            int32_t* __restrict__ status) {
   __shared__ uint32_t anc[16][16];
   __shared__ int leaf_depth[16], fill[16], dfs_s[16];
@@ -145,15 +145,14 @@ __device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int64_
       int d = 0;
       while (d < leaf_depth[i] && (anc[i][d] & ~Nx) != 0) ++d;
       const int slot = atomicAdd(&fill[i], 1);
-      const int64_t base = req_off[r0 + i] - o0;
-      keys[base + slot] = ((unsigned long long)d << 32) | (unsigned long long)(uint32_t)cx[u];
+      keys[roff[i] + slot] = ((unsigned long long)d << 32) | (unsigned long long)(uint32_t)cx[u];
     }
   }
   __syncthreads();
   const int lane = t & 31, warp = t >> 5;
   for (int i = warp; i < m; i += kBatchThreads / 32) {
-    const int64_t base = req_off[r0 + i] - o0;
-    const int len = (int)(req_off[r0 + i + 1] - req_off[r0 + i]);
+    const int base = roff[i];
+    const int len = roff[i + 1] - roff[i];
     for (int j = lane; j < len; j += 32) {
       const unsigned long long kj = keys[base + j];
       int rank = 0;
@@ -189,9 +188,10 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                    // [occ_cap] their request sets
   uint32_t* tmask = cN + occ_cap;                                                // [2 * occ_cap] hash-table masks
   __shared__ int ndistinct;
+  __shared__ int roff[16];  // request offsets relative to o0
   const int t = threadIdx.x;
   const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
-                              cN, &ndistinct);
+                              cN, roff, &ndistinct);
   for (int S = t; S < N; S += kBatchThreads) wI[S] = 0;
   __syncthreads();
 
@@ -315,7 +315,7 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 
   // 4. hierarchy walk
   __syncthreads();
-  batch_walk(inst, m, r0, o0, req_off, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  batch_walk(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -409,8 +409,9 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   __shared__ int ndistinct;
   const int t = threadIdx.x;
 
+  __shared__ int roff[16];  // request offsets relative to o0
   const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
-                              cN, &ndistinct);
+                              cN, roff, &ndistinct);
 
   // g and the superset sums, in the padded row layout: the five in-row bits
   // per row in registers, then one row-pair pass per row bit
@@ -583,7 +584,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   }
   if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   __syncthreads();
-  batch_walk(inst, m, r0, o0, req_off, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  batch_walk(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 }  // namespace
