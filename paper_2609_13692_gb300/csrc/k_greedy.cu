@@ -10,10 +10,10 @@
 // Thm 1 proof.  Lower bound: sum_i w(R_i) - MaxSpanningTree(w(R_i cap R_j)).
 //
 // Kernels: k_pair_weights fills W[i][j] = w(R_i cap R_j) (sorted chunk lists,
-// merge-intersection); k_maxst runs Prim on W in one block; k_greedy_merge runs
-// all m - 1 merges in one block, keeping for every active slot its best
-// partner as a 64-bit key (weight, then the smallest slot pair) and rescanning
-// a row only when its best partner was merged; k_greedy_layout climbs each
+// merge-intersection); Borůvka rounds find the maximum spanning tree of W;
+// k_greedy_merge runs all m - 1 merges in one block, keeping for every active
+// slot an upper bound on its best partner as a 64-bit key (weight, then the
+// smallest slot pair) and rescanning a row only when its key is found stale; k_greedy_layout climbs each
 // (request, chunk) occurrence to the highest node whose signature still holds
 // the chunk, and ranks each request's chunks by (depth, chunk id).
 #include "../../include/mpt.h"
@@ -100,32 +100,84 @@ __device__ unsigned long long block_max_u64(unsigned long long v, unsigned long 
   return r;
 }
 
-// Prim's maximum spanning tree on W (one block).  tree_key[v]: heaviest edge
-// from v into the tree so far.
-__global__ void __launch_bounds__(kGreedyThreads)
-k_maxst(int m, const uint32_t* __restrict__ W, uint32_t* __restrict__ tree_key, uint8_t* __restrict__ in_tree,
-        unsigned long long* __restrict__ out) {
-  __shared__ unsigned long long red[33];
-  for (int v = threadIdx.x; v < m; v += blockDim.x) {
-    tree_key[v] = W[v];  // row 0
-    in_tree[v] = v == 0;
+// Maximum spanning tree of W (Borůvka).  Edges are ordered by pair_key
+// (weight, then the smaller slot pair), so every edge key is distinct and the
+// tree is unique; its weight is the maximum spanning-tree weight (Sec. 6.3).
+// A round: each vertex's heaviest edge to another component (warp per row),
+// each component's heaviest (atomicMax), components hook along them (a pair
+// of components that chose the same edge keeps the smaller id as root, and
+// that edge is counted once), then every vertex jumps to its root.  Every
+// round at least halves the number of components.
+__global__ void k_bv_vertex_best(int m, const uint32_t* __restrict__ W, const int32_t* __restrict__ comp,
+                                 unsigned long long* __restrict__ cbest) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int v = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; v < m; v += warps) {
+    const int cv = comp[v];
+    unsigned long long b = 0;
+    for (int u = lane; u < m; u += 32)
+      if (comp[u] != cv) b = max(b, pair_key((uint32_t)v, (uint32_t)u, W[(size_t)v * m + u]));
+    for (int off = 16; off > 0; off >>= 1) b = max(b, __shfl_xor_sync(0xFFFFFFFFu, b, off));
+    if (lane == 0 && b) atomicMax(&cbest[cv], b);
   }
-  __syncthreads();
-  unsigned long long total = 0;
-  for (int it = 1; it < m; ++it) {
-    unsigned long long cand = 0;
-    for (int v = threadIdx.x; v < m; v += blockDim.x)
-      if (!in_tree[v]) cand = max(cand, ((unsigned long long)tree_key[v] << 20) | (unsigned long long)((1u << 20) - 1u - v));
-    const unsigned long long b = block_max_u64(cand, red);
-    const int v0 = (int)((1u << 20) - 1u - (uint32_t)(b & ((1u << 20) - 1u)));
-    total += b >> 20;
-    if (threadIdx.x == 0) in_tree[v0] = 1;
-    __syncthreads();
-    for (int v = threadIdx.x; v < m; v += blockDim.x)
-      if (!in_tree[v]) tree_key[v] = max(tree_key[v], W[(size_t)v0 * m + v]);
-    __syncthreads();
+}
+
+__global__ void k_bv_hook(int m, const int32_t* __restrict__ comp, const unsigned long long* __restrict__ cbest,
+                          int32_t* __restrict__ parent, unsigned long long* __restrict__ total) {
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < m; c += gridDim.x * blockDim.x) {
+    if (comp[c] != c) continue;  // not a component root
+    const unsigned long long k = cbest[c];
+    if (k == 0) {
+      parent[c] = c;
+      continue;
+    }
+    uint32_t a, b;
+    key_pair(k, &a, &b);
+    const int o = comp[a] == c ? comp[b] : comp[a];
+    const bool mutual = cbest[o] == k;
+    parent[c] = (mutual && c < o) ? c : o;
+    if (!(mutual && o < c)) atomicAdd(total, k >> 28);
   }
-  if (threadIdx.x == 0) *out = total;
+}
+
+__global__ void k_bv_jump(int m, int32_t* __restrict__ comp, const int32_t* __restrict__ parent) {
+  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < m; v += gridDim.x * blockDim.x) {
+    int r = comp[v];
+    for (int step = 0; step < m && parent[r] != r; ++step) r = parent[r];
+    comp[v] = r;
+  }
+}
+
+__global__ void k_bv_reset(int m, unsigned long long* __restrict__ cbest) {
+  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < m; v += gridDim.x * blockDim.x) cbest[v] = 0;
+}
+
+__global__ void k_iota32(int m, int32_t* __restrict__ a) {
+  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < m; v += gridDim.x * blockDim.x) a[v] = v;
+}
+
+
+// All m - 1 merges (one block).  best[d] is an upper bound on row d's best
+// pair key: pair weights only decrease as clusters merge, so a key stays an
+// upper bound until its row is rescanned.  The largest bound is merged only
+// if it is still exact (both slots active, weight unchanged); otherwise its
+// rows are rescanned and the choice is repeated.  Every rescan makes a row
+// exact, so a step repeats at most m times (kept as a hard cap).
+// Weight of sig_d (sorted, in global memory) within the merged signature
+// s_new (sorted, shared memory): binary search of each chunk of sig_d.
+__device__ __forceinline__ uint32_t sig_weight_in(const int32_t* __restrict__ sd, int ld, const int32_t* s_new,
+                                                  int ln, const int64_t* __restrict__ w) {
+  uint32_t s = 0;
+  for (int q = 0; q < ld; ++q) {
+    const int32_t x = sd[q];
+    int lo = 0, hi = ln;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (s_new[mid] < x) lo = mid + 1; else hi = mid;
+    }
+    if (lo < ln && s_new[lo] == x) s += (uint32_t)w[x];
+  }
+  return s;
 }
 
 __device__ unsigned long long block_row_best(int m, int d, const uint32_t* __restrict__ W,
@@ -136,12 +188,10 @@ __device__ unsigned long long block_row_best(int m, int d, const uint32_t* __res
   return block_max_u64(bb, red);
 }
 
-// All m - 1 merges (one block).  best[d] is an upper bound on row d's best
-// pair key: pair weights only decrease as clusters merge, so a key stays an
-// upper bound until its row is rescanned.  The largest bound is merged only
-// if it is still exact (both slots active, weight unchanged); otherwise its
-// rows are rescanned and the choice is repeated.  Every rescan makes a row
-// exact, so a step repeats at most m times (kept as a hard cap).
+// All m - 1 merges in one block, with lazy best keys: best[d] is an upper
+// bound on slot d's best pair key (weights only decrease as signatures
+// shrink).  The largest key is merged only if it is still exact; otherwise
+// the rows of its two slots are rescanned and the search repeats.
 __global__ void __launch_bounds__(kGreedyThreads)
 k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, int32_t* __restrict__ len,
                uint32_t* __restrict__ W, unsigned long long* __restrict__ best, uint8_t* __restrict__ active,
@@ -149,8 +199,10 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
                int32_t* __restrict__ children, int32_t* __restrict__ node_sig, int32_t* __restrict__ node_len,
                int32_t* __restrict__ error) {
   __shared__ unsigned long long red[33];
-  __shared__ int32_t s_new[kSigMax];
+  __shared__ int32_t s_a[kSigMax], s_b[kSigMax], s_new[kSigMax];
   __shared__ int s_len;
+  __shared__ int warp_cnt[kGreedyThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int d = threadIdx.x; d < m; d += blockDim.x) {
     active[d] = 1;
     node[d] = d;
@@ -169,7 +221,7 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
       if (active[a] && active[b] && W[(size_t)a * m + b] == v) break;
       if (++tries > m + 1) {
         if (threadIdx.x == 0) atomicOr(error, 1);
-        break;
+        return;
       }
       if (active[a]) {
         const unsigned long long r = block_row_best(m, (int)a, W, active, red);
@@ -181,30 +233,43 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
       }
       __syncthreads();
     }
+    // merged signature: the chunks of a that b holds, in order
+    const int la = len[a], lb = len[b];
+    for (int q = threadIdx.x; q < la; q += blockDim.x) s_a[q] = sig[(size_t)a * kSigMax + q];
+    for (int q = threadIdx.x; q < lb; q += blockDim.x) s_b[q] = sig[(size_t)b * kSigMax + q];
+    __syncthreads();
+    bool keep = false;
+    int32_t x = 0;
+    if (threadIdx.x < la) {
+      x = s_a[threadIdx.x];
+      int lo = 0, hi = lb;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (s_b[mid] < x) lo = mid + 1; else hi = mid;
+      }
+      keep = lo < lb && s_b[lo] == x;
+    }
+    const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
+    if (lane == 0) warp_cnt[warp] = __popc(bal);
+    __syncthreads();
+    if (keep) {
+      int before = __popc(bal & ((1u << lane) - 1u));
+      for (int q = 0; q < warp; ++q) before += warp_cnt[q];  // kSigMax <= 128: at most four warps
+      s_new[before] = x;
+    }
     if (threadIdx.x == 0) {
+      int n = 0;
+      for (int q = 0; q < (kSigMax + 31) / 32; ++q) n += warp_cnt[q];
+      s_len = n;
       merges[2 * t] = (int32_t)a;
       merges[2 * t + 1] = (int32_t)b;
       values[t] = v;
       children[2 * t] = node[a];
       children[2 * t + 1] = node[b];
-      const int32_t* sa = sig + (size_t)a * kSigMax;
-      const int32_t* sb = sig + (size_t)b * kSigMax;
-      int i = 0, j = 0, n = 0;
-      while (i < len[a] && j < len[b]) {
-        if (sa[i] == sb[j]) {
-          s_new[n++] = sa[i];
-          ++i;
-          ++j;
-        } else if (sa[i] < sb[j]) {
-          ++i;
-        } else {
-          ++j;
-        }
-      }
-      s_len = n;
     }
     __syncthreads();
-    for (int q = threadIdx.x; q < s_len; q += blockDim.x) {
+    const int ln = s_len;
+    for (int q = threadIdx.x; q < ln; q += blockDim.x) {
       sig[(size_t)a * kSigMax + q] = s_new[q];
       node_sig[(size_t)t * kSigMax + q] = s_new[q];
     }
@@ -213,16 +278,16 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
     for (int d = threadIdx.x; d < m; d += blockDim.x) {
       if (!active[d] || d == (int)a || d == (int)b) continue;
       const uint32_t wa = W[(size_t)a * m + d], wb = W[(size_t)b * m + d];
-      const uint32_t wv = (wa == 0 || wb == 0 || s_len == 0)
+      const uint32_t wv = (wa == 0 || wb == 0 || ln == 0)
                               ? 0u
-                              : sig_weight(s_new, s_len, sig + (size_t)d * kSigMax, len[d], w);
+                              : sig_weight_in(sig + (size_t)d * kSigMax, len[d], s_new, ln, w);
       W[(size_t)a * m + d] = wv;
       W[(size_t)d * m + a] = wv;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-      len[a] = s_len;
-      node_len[t] = s_len;
+      len[a] = ln;
+      node_len[t] = ln;
       node[a] = m + t;
       active[b] = 0;
     }
@@ -359,8 +424,8 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
                o_nsig = take(M * kSigMax * 4), o_nlen = take(M * 4), o_roff = take((M + 1) * 8),
                o_chunks = take((size_t)std::max<int64_t>(occ, 1) * 8), o_par = take(2 * M * 4),
                o_dep = take(2 * M * 4), o_stk = take(2 * M * 4), o_keys = take((size_t)std::max<int64_t>(occ, 1) * 8),
-               o_perm = take((size_t)std::max<int64_t>(occ, 1) * 8), o_dfs = take(M * 4), o_tk = take(M * 4),
-               o_int = take(M), o_mst = take(8);
+               o_perm = take((size_t)std::max<int64_t>(occ, 1) * 8), o_dfs = take(M * 4), o_comp = take(M * 4),
+               o_bpar = take(M * 4), o_cbest = take(M * 8), o_mst = take(8);
   char* d = nullptr;
   if (cudaMalloc(&d, off) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
   mpt_status st = MPT_OK;
@@ -377,6 +442,7 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
   h2d(o_roff, req_offsets, (M + 1) * 8);
   h2d(o_chunks, chunk_ids, (size_t)occ * 8);
   if (e == cudaSuccess) e = cudaMemsetAsync(d + o_re, 0, 4, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d + o_mst, 0, 8, stream);
   auto I64 = [&](size_t o) { return reinterpret_cast<int64_t*>(d + o); };
   auto I32 = [&](size_t o) { return reinterpret_cast<int32_t*>(d + o); };
   auto U32 = [&](size_t o) { return reinterpret_cast<uint32_t*>(d + o); };
@@ -384,8 +450,21 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
   if (e == cudaSuccess) {
     dim3 grid((unsigned)((m + 255) / 256), (unsigned)m);
     k_pair_weights<<<grid, 256, 0, stream>>>(m, I32(o_sig), I32(o_len), I64(o_w), U32(o_W));
-    k_maxst<<<1, kGreedyThreads, 0, stream>>>(m, U32(o_W), U32(o_tk), reinterpret_cast<uint8_t*>(d + o_int),
-                                               U64(o_mst));
+    {
+      // maximum spanning tree by Borůvka rounds (each at least halves the components)
+      const unsigned vb = (unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, 152 * 32);
+      const unsigned eb = (unsigned)std::min<int64_t>((m + 255) / 256, 152 * 8);
+      k_iota32<<<eb, 256, 0, stream>>>(m, I32(o_comp));
+      k_bv_reset<<<eb, 256, 0, stream>>>(m, U64(o_cbest));
+      int rounds = 1;
+      while ((1 << rounds) < m) ++rounds;
+      for (int r = 0; r < rounds; ++r) {
+        k_bv_vertex_best<<<vb, 256, 0, stream>>>(m, U32(o_W), I32(o_comp), U64(o_cbest));
+        k_bv_hook<<<eb, 256, 0, stream>>>(m, I32(o_comp), U64(o_cbest), I32(o_bpar), U64(o_mst));
+        k_bv_jump<<<eb, 256, 0, stream>>>(m, I32(o_comp), I32(o_bpar));
+        k_bv_reset<<<eb, 256, 0, stream>>>(m, U64(o_cbest));
+      }
+    }
     k_row_best<<<(unsigned)((m * 32 + 255) / 256), 256, 0, stream>>>(m, U32(o_W), U64(o_best));
     k_greedy_merge<<<1, kGreedyThreads, 0, stream>>>(m, I64(o_w), I32(o_sig), I32(o_len), U32(o_W), U64(o_best),
                                                       reinterpret_cast<uint8_t*>(d + o_act), I32(o_node), I32(o_mer),
