@@ -180,56 +180,85 @@ __device__ __forceinline__ uint32_t sig_weight_in(const int32_t* __restrict__ sd
   return s;
 }
 
-__device__ unsigned long long block_row_best(int m, int d, const uint32_t* __restrict__ W,
-                                             const uint8_t* __restrict__ active, unsigned long long* red) {
+
+// All m - 1 merges in one block, with lazy best keys: sb[d] (shared memory)
+// is an upper bound on slot d's best pair key (weights only decrease as
+// signatures shrink), 0 once d is merged away, and gmax[g] is the largest of
+// sb[32 g .. 32 g + 31].  The largest key is merged only if it is still
+// exact; otherwise the rows of its two slots are rescanned and the search
+// repeats.
+constexpr int kMaxGroups = kMaxGreedyM / 32;
+
+__device__ __forceinline__ void refresh_group(int m, int g, const unsigned long long* sb, unsigned long long* gmax) {
+  if (threadIdx.x < 32) {
+    const int d = g * 32 + (int)threadIdx.x;
+    unsigned long long v = d < m ? sb[d] : 0ull;
+    for (int off = 16; off > 0; off >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, off));
+    if (threadIdx.x == 0) gmax[g] = v;
+  }
+}
+
+__device__ unsigned long long smem_row_best(int m, int d, const uint32_t* __restrict__ W, const uint8_t* act,
+                                            unsigned long long* red) {
   unsigned long long bb = 0;
+  const uint32_t* row = W + (size_t)d * m;
   for (int e = threadIdx.x; e < m; e += blockDim.x)
-    if (e != d && active[e]) bb = max(bb, pair_key((uint32_t)d, (uint32_t)e, W[(size_t)d * m + e]));
+    if (e != d && act[e]) bb = max(bb, pair_key((uint32_t)d, (uint32_t)e, row[e]));
   return block_max_u64(bb, red);
 }
 
-// All m - 1 merges in one block, with lazy best keys: best[d] is an upper
-// bound on slot d's best pair key (weights only decrease as signatures
-// shrink).  The largest key is merged only if it is still exact; otherwise
-// the rows of its two slots are rescanned and the search repeats.
 __global__ void __launch_bounds__(kGreedyThreads)
 k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, int32_t* __restrict__ len,
-               uint32_t* __restrict__ W, unsigned long long* __restrict__ best, uint8_t* __restrict__ active,
-               int32_t* __restrict__ node, int32_t* __restrict__ merges, int64_t* __restrict__ values,
-               int32_t* __restrict__ children, int32_t* __restrict__ node_sig, int32_t* __restrict__ node_len,
-               int32_t* __restrict__ error) {
+               uint32_t* __restrict__ W, const unsigned long long* __restrict__ best0, int32_t* __restrict__ node,
+               int32_t* __restrict__ merges, int64_t* __restrict__ values, int32_t* __restrict__ children,
+               int32_t* __restrict__ node_sig, int32_t* __restrict__ node_len, int32_t* __restrict__ error) {
+  extern __shared__ __align__(16) unsigned char gsm[];
+  unsigned long long* sb = reinterpret_cast<unsigned long long*>(gsm);        // [m]
+  unsigned long long* gmax = sb + m;                                          // [ceil(m / 32)]
+  uint8_t* act = reinterpret_cast<uint8_t*>(gmax + kMaxGroups);               // [m]
   __shared__ unsigned long long red[33];
   __shared__ int32_t s_a[kSigMax], s_b[kSigMax], s_new[kSigMax];
   __shared__ int s_len;
   __shared__ int warp_cnt[kGreedyThreads / 32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int groups = (m + 31) / 32;
   for (int d = threadIdx.x; d < m; d += blockDim.x) {
-    active[d] = 1;
+    act[d] = 1;
     node[d] = d;
+    sb[d] = best0[d];
+  }
+  __syncthreads();
+  for (int g = warp; g < groups; g += kGreedyThreads / 32) {
+    const int d = g * 32 + lane;
+    unsigned long long v = d < m ? sb[d] : 0ull;
+    for (int off = 16; off > 0; off >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, off));
+    if (lane == 0) gmax[g] = v;
   }
   __syncthreads();
   for (int t = 0; t < m - 1; ++t) {
     uint32_t a = 0, b = 0, v = 0;
     int tries = 0;
     for (;;) {
-      unsigned long long c = 0;
-      for (int d = threadIdx.x; d < m; d += blockDim.x)
-        if (active[d]) c = max(c, best[d]);
+      const unsigned long long c = (int)threadIdx.x < groups ? gmax[threadIdx.x] : 0ull;
       const unsigned long long top = block_max_u64(c, red);
       key_pair(top, &a, &b);
       v = (uint32_t)(top >> 28);
-      if (active[a] && active[b] && W[(size_t)a * m + b] == v) break;
-      if (++tries > m + 1) {
+      if (top != 0 && act[a] && act[b] && W[(size_t)a * m + b] == v) break;
+      if (top == 0 || ++tries > m + 1) {
         if (threadIdx.x == 0) atomicOr(error, 1);
         return;
       }
-      if (active[a]) {
-        const unsigned long long r = block_row_best(m, (int)a, W, active, red);
-        if (threadIdx.x == 0) best[a] = r;
+      if (act[a]) {
+        const unsigned long long r = smem_row_best(m, (int)a, W, act, red);
+        if (threadIdx.x == 0) sb[a] = r;
+        __syncthreads();
+        refresh_group(m, (int)a >> 5, sb, gmax);
       }
-      if (active[b]) {
-        const unsigned long long r = block_row_best(m, (int)b, W, active, red);
-        if (threadIdx.x == 0) best[b] = r;
+      if (act[b]) {
+        const unsigned long long r = smem_row_best(m, (int)b, W, act, red);
+        if (threadIdx.x == 0) sb[b] = r;
+        __syncthreads();
+        refresh_group(m, (int)b >> 5, sb, gmax);
       }
       __syncthreads();
     }
@@ -240,7 +269,7 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
     __syncthreads();
     bool keep = false;
     int32_t x = 0;
-    if (threadIdx.x < la) {
+    if ((int)threadIdx.x < la) {
       x = s_a[threadIdx.x];
       int lo = 0, hi = lb;
       while (lo < hi) {
@@ -276,7 +305,7 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
     // new pair weights of the merged slot: zero wherever either old weight was
     // zero (the merged signature is a subset of both)
     for (int d = threadIdx.x; d < m; d += blockDim.x) {
-      if (!active[d] || d == (int)a || d == (int)b) continue;
+      if (!act[d] || d == (int)a || d == (int)b) continue;
       const uint32_t wa = W[(size_t)a * m + d], wb = W[(size_t)b * m + d];
       const uint32_t wv = (wa == 0 || wb == 0 || ln == 0)
                               ? 0u
@@ -289,14 +318,21 @@ k_greedy_merge(int m, const int64_t* __restrict__ w, int32_t* __restrict__ sig, 
       len[a] = ln;
       node_len[t] = ln;
       node[a] = m + t;
-      active[b] = 0;
+      act[b] = 0;
+      sb[b] = 0;
     }
     __syncthreads();
-    const unsigned long long r = block_row_best(m, (int)a, W, active, red);
-    if (threadIdx.x == 0) best[a] = r;
+    const unsigned long long r = smem_row_best(m, (int)a, W, act, red);
+    if (threadIdx.x == 0) sb[a] = r;
+    __syncthreads();
+    refresh_group(m, (int)a >> 5, sb, gmax);
+    __syncthreads();
+    refresh_group(m, (int)b >> 5, sb, gmax);
     __syncthreads();
   }
 }
+
+size_t merge_smem_bytes(int m) { return (size_t)m * 8 + (size_t)kMaxGroups * 8 + (size_t)m + 16; }
 
 // Parent and depth of every tree node and the left-to-right leaf order (one thread).
 __global__ void k_greedy_tree(int m, const int32_t* __restrict__ children, int32_t* __restrict__ parent,
@@ -419,7 +455,7 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
   };
   const size_t M = (size_t)m;
   const size_t o_w = take((size_t)n_chunks * 8), o_sig = take(M * kSigMax * 4), o_len = take(M * 4),
-               o_W = take(M * M * 4), o_best = take(M * 8), o_act = take(M), o_node = take(M * 4),
+               o_W = take(M * M * 4), o_best = take(M * 8), o_node = take(M * 4),
                o_re = take(M * 4 + 4), o_mer = take(M * 8), o_val = take(M * 8), o_ch = take(M * 8),
                o_nsig = take(M * kSigMax * 4), o_nlen = take(M * 4), o_roff = take((M + 1) * 8),
                o_chunks = take((size_t)std::max<int64_t>(occ, 1) * 8), o_par = take(2 * M * 4),
@@ -466,9 +502,14 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
       }
     }
     k_row_best<<<(unsigned)((m * 32 + 255) / 256), 256, 0, stream>>>(m, U32(o_W), U64(o_best));
-    k_greedy_merge<<<1, kGreedyThreads, 0, stream>>>(m, I64(o_w), I32(o_sig), I32(o_len), U32(o_W), U64(o_best),
-                                                      reinterpret_cast<uint8_t*>(d + o_act), I32(o_node), I32(o_mer),
-                                                      I64(o_val), I32(o_ch), I32(o_nsig), I32(o_nlen), I32(o_re));
+    {
+      const size_t msm = merge_smem_bytes(m);
+      e = cudaFuncSetAttribute(k_greedy_merge, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)msm);
+      if (e == cudaSuccess)
+        k_greedy_merge<<<1, kGreedyThreads, msm, stream>>>(m, I64(o_w), I32(o_sig), I32(o_len), U32(o_W), U64(o_best),
+                                                           I32(o_node), I32(o_mer), I64(o_val), I32(o_ch), I32(o_nsig),
+                                                           I32(o_nlen), I32(o_re));
+    }
     k_greedy_tree<<<1, 1, 0, stream>>>(m, I32(o_ch), I32(o_par), I32(o_dep), I32(o_stk), I32(o_dfs));
     const int64_t eblocks = std::min<int64_t>((std::max<int64_t>(occ, 1) + 255) / 256, 152 * 16);
     k_greedy_emit<<<(unsigned)eblocks, 256, 0, stream>>>(m, I32(o_nsig), I32(o_nlen), I64(o_roff), I64(o_chunks),
