@@ -184,7 +184,7 @@ def run_reference(args):
     from paper_2609_13692_gb300 import instances
 
     inst = instances.config(WORKLOAD, seed=0)
-    m_sub = ORACLE_SAMPLE_REQUESTS
+    m_sub = args.ref_requests
     for _ in range(args.warmup):
         oracle_sample(inst, m_sub)
     total_splits, total_t, cores = 0, 0.0, 1
@@ -556,6 +556,8 @@ def main():
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-requests", type=int, default=ORACLE_SAMPLE_REQUESTS,
+                    help="reference arm: requests of the workload in each step's oracle sample")
     ap.add_argument("--tables", choices=["int64", "lean"], default="int64",
                     help="table layout of the exact solve (lean: one int32 table, F over w(I))")
     ap.add_argument("--mode", choices=["solve", "batch", "greedy", "cache"], default="solve",

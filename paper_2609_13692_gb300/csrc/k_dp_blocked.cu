@@ -646,15 +646,15 @@ int blocked_max_launches(const Shape& s) { return 2 * (s.L + 1); }
 
 cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
                               BlockedTiming* timing, int step_begin, int step_end) {
-  static bool attr_done = false;
-  if (!attr_done) {
+  {
+    // the attributes belong to the current device: set them on every call (a
+    // host-side call, negligible against a solve), so that any device works
     cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(k_dp_tile_rows<int64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(k_dp_tile_rows<int32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
     if (e != cudaSuccess) return e;
-    attr_done = true;
   }
   const int b = s.b, L = s.L;
   constexpr unsigned long long evals_per_pair = 531441ull;  // 3^12 splits per pair of windows
