@@ -242,3 +242,40 @@ def test_m31_extension(mpt):
             idx = torch.from_numpy(_submask_index(S)).to(F_d.device)
             f, a, w = O.recompute_local(inst.weights, inst.bits, S, F_d[idx].cpu().numpy())
             assert (f, a, w) == (int(F_d[S].item()), int(split_d[S].item()) & 0xFFFFFFFF, int(wI_d[S].item()))
+
+
+def test_concurrent_contexts_on_streams(mpt):
+    """Independent contexts solved at the same time on different streams (own
+    workspaces) give the same tables as solving them one after the other: no
+    state is shared between contexts."""
+    insts = [I.rag_pools(20, 5000, 6, 40, 8, 1.1, seed=s) for s in (21, 22)]
+    insts.append(I.random_instance(15, 80, (2, 9), seed=23, wmin=200_000, wmax=400_000))  # general kernels
+    seq = []
+    for inst in insts:
+        r = mpt.solve(inst.weights, inst.bits)
+        seq.append((r.opt, [t.clone() for t in mpt.mpt_tables(r.ctx)], r.permutations()))
+    streams = [torch.cuda.Stream() for _ in insts]
+    ctxs, wss = [], []
+    for inst in insts:
+        c = mpt.mpt_create(inst.weights, inst.bits)
+        ctxs.append(c)
+        wss.append(torch.empty(mpt.mpt_workspace_bytes(c), dtype=torch.uint8, device="cuda"))
+    import threading
+
+    out = [None] * len(insts)
+
+    def run(i):
+        out[i] = mpt.mpt_solve(ctxs[i], wss[i], streams[i].cuda_stream)
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(len(insts))]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    torch.cuda.synchronize()
+    for i, (opt, tables, perms) in enumerate(seq):
+        assert out[i] == opt
+        for a, b in zip(tables, mpt.mpt_tables(ctxs[i])):
+            assert torch.equal(a, b)
+        offs, chunks, dfs = mpt.mpt_layout(ctxs[i])
+        assert [chunks[offs[j]:offs[j + 1]].tolist() for j in range(len(offs) - 1)] == perms
