@@ -39,6 +39,7 @@ constexpr int kBatchThreads = 256;
 // in shared memory: tkey[0..2*occ_cap) (chunk id or -1) and tmask (request
 // bits), open addressing with linear probing.  The table has at least twice
 // as many slots as occurrences, so every insertion ends within `size` probes.
+template <int TPI>
 __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap, const int64_t* __restrict__ req_off,
                             const int64_t* __restrict__ chunks, int32_t* tkey, uint32_t* tmask, int32_t* cx,
                             uint32_t* cN, int* roff, int* ndistinct_s) {
@@ -48,12 +49,12 @@ __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap,
   const int lg = 31 - __clz(size);
   if (t == 0) ndistinct = 0;
   if (t <= m) roff[t] = (int)(req_off[r0 + t] - o0);
-  for (int h = t; h < size; h += kBatchThreads) {
+  for (int h = t; h < size; h += TPI) {
     tkey[h] = -1;
     tmask[h] = 0;
   }
   __syncthreads();
-  for (int j = t; j < occ; j += kBatchThreads) {
+  for (int j = t; j < occ; j += TPI) {
     int i = 0;
     while (roff[i + 1] <= j) ++i;  // the request whose slot range holds j
     const int32_t x = (int32_t)chunks[o0 + j];
@@ -68,7 +69,7 @@ __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap,
     }
   }
   __syncthreads();
-  for (int h = t; h < size; h += kBatchThreads) {
+  for (int h = t; h < size; h += TPI) {
     const int32_t x = tkey[h];
     if (x >= 0) {
       const int u = atomicAdd(&ndistinct, 1);
@@ -85,7 +86,7 @@ __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap,
 // left-to-right leaf order.  Every thread of the block calls it after the
 // split table is complete and visible.
 // roff: the request offsets staged by batch_gather (shared memory).
-template <typename SplitT>
+template <int TPI, typename SplitT>
 __device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int* roff, const SplitT* split,
                            unsigned long long* keys, const int32_t* cx, const uint32_t* cN, int nd,
                            int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out,
@@ -138,7 +139,7 @@ __device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int* r
   }
   if (t < m) dfs_out[r0 + t] = dfs_s[t];
   // keys (depth, chunk id) into each request's own slot range, then rank them
-  for (int u = t; u < nd; u += kBatchThreads) {
+  for (int u = t; u < nd; u += TPI) {
     const uint32_t Nx = cN[u];
     for (uint32_t rr = Nx; rr; rr &= rr - 1) {
       const int i = __ffs(rr) - 1;
@@ -150,7 +151,7 @@ __device__ void batch_walk(int inst, int m, int64_t r0, int64_t o0, const int* r
   }
   __syncthreads();
   const int lane = t & 31, warp = t >> 5;
-  for (int i = warp; i < m; i += kBatchThreads / 32) {
+  for (int i = warp; i < m; i += TPI / 32) {
     const int base = roff[i];
     const int len = roff[i + 1] - roff[i];
     for (int j = lane; j < len; j += 32) {
@@ -190,8 +191,8 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   __shared__ int ndistinct;
   __shared__ int roff[16];  // request offsets relative to o0
   const int t = threadIdx.x;
-  const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
-                              cN, roff, &ndistinct);
+  const int nd = batch_gather<kBatchThreads>(m, r0, o0, occ, occ_cap, req_off, chunks,
+                                             reinterpret_cast<int32_t*>(keys), tmask, cx, cN, roff, &ndistinct);
   for (int S = t; S < N; S += kBatchThreads) wI[S] = 0;
   __syncthreads();
 
@@ -315,7 +316,7 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 
   // 4. hierarchy walk
   __syncthreads();
-  batch_walk(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  batch_walk<kBatchThreads>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -345,7 +346,39 @@ constexpr int kBRow = 32;
 constexpr int kBRowStride = 36;
 constexpr int kBMaxLevelRows = 70;  // C(8, 4): the most rows of one level (m = 13)
 constexpr int kBkStride = kBRow + 1; // phase A minima: 33 words a row, so rows read by one warp use different banks
-static_assert((kBMaxLevelRows * kBkStride * 4) % 8 == 0, "the sort keys after the minima need 8-byte alignment");
+
+// rows of the largest level C(nb, nb / 2), rounded up to even so that the
+// 64-bit keys after the minima stay 8-byte aligned
+__host__ __device__ constexpr int batch_level_rows(int nb) {
+  int c = 1;
+  for (int i = 0; i < nb / 2; ++i) c = c * (nb - i) / (i + 1);
+  return (c + 1) & ~1;
+}
+static_assert(batch_level_rows(8) == kBMaxLevelRows, "the most rows of one level (m = 13)");
+
+// threads per block of the row-blocked kernel for m requests: enough lanes for
+// the busiest level (rows x lanes per row) -- 30 up to m = 11, 84 at m = 12,
+// 224 at m = 13
+constexpr int batch_rows_threads(int m) { return m <= 11 ? 64 : (m == 12 ? 128 : 256); }
+
+// lanes the busiest level needs: rows C(nb, p1) times 2^(p1 - 3) lanes per row
+// in phase A, C(nb, p1) threads in phase B
+constexpr int batch_rows_lanes(int nb) {
+  int most = 0;
+  for (int p1 = 1; p1 <= nb; ++p1) {
+    int c = 1;
+    for (int i = 0; i < p1; ++i) c = c * (nb - i) / (i + 1);
+    const int lanes = c * (p1 > 3 ? 1 << (p1 - 3) : 1);
+    most = lanes > most ? lanes : most;
+  }
+  return most;
+}
+constexpr bool batch_rows_fit() {
+  for (int m = 6; m <= 13; ++m)
+    if (batch_rows_lanes(m - 5) > batch_rows_threads(m) || batch_level_rows(m - 5) > batch_rows_threads(m)) return false;
+  return true;
+}
+static_assert(batch_rows_fit(), "every level of the row-blocked kernel fits its block");
 
 __device__ __forceinline__ int brow_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
 __device__ __forceinline__ int bidx(uint32_t U) { return brow_pos(U >> 5) * kBRowStride + (int)(U & 31u); }
@@ -380,7 +413,8 @@ __device__ __forceinline__ void bconv_restricted(uint32_t (&acc)[kBRow], const u
   }
 }
 
-__global__ void __launch_bounds__(kBatchThreads)
+template <int TPI>
+__global__ void __launch_bounds__(TPI)
 k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
              const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
              const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list, int occ_cap, int mm,
@@ -400,8 +434,9 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 
   uint32_t* Gp = reinterpret_cast<uint32_t*>(smem_raw);                          // [R * 36]
   uint32_t* Gc = Gp + (1 << (mm - 5)) * kBRowStride;                               // [R * 36]
-  uint32_t* bk = Gc + (1 << (mm - 5)) * kBRowStride;                               // [70 * 33] phase A minima
-  unsigned long long* keys = reinterpret_cast<unsigned long long*>(bk + kBMaxLevelRows * kBkStride);  // [occ_cap]
+  uint32_t* bk = Gc + (1 << (mm - 5)) * kBRowStride;                               // [level rows * 33] phase A minima
+  unsigned long long* keys =
+      reinterpret_cast<unsigned long long*>(bk + batch_level_rows(mm - 5) * kBkStride);  // [occ_cap]
   int32_t* cx = reinterpret_cast<int32_t*>(keys + occ_cap);                        // [occ_cap]
   uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                        // [occ_cap]
   uint32_t* tmask = cN + occ_cap;                                                  // [2 * occ_cap] hash-table masks
@@ -410,16 +445,16 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   const int t = threadIdx.x;
 
   __shared__ int roff[16];  // request offsets relative to o0
-  const int nd = batch_gather(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask, cx,
-                              cN, roff, &ndistinct);
+  const int nd = batch_gather<TPI>(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask,
+                                   cx, cN, roff, &ndistinct);
 
   // g and the superset sums, in the padded row layout: the five in-row bits
   // per row in registers, then one row-pair pass per row bit
-  for (int i = t; i < R * kBRowStride; i += kBatchThreads) Gp[i] = 0;
+  for (int i = t; i < R * kBRowStride; i += TPI) Gp[i] = 0;
   __syncthreads();
-  for (int u = t; u < nd; u += kBatchThreads) atomicAdd(&Gp[bidx(cN[u])], (uint32_t)weights[cx[u]]);
+  for (int u = t; u < nd; u += TPI) atomicAdd(&Gp[bidx(cN[u])], (uint32_t)weights[cx[u]]);
   __syncthreads();
-  for (int r = t; r < R; r += kBatchThreads) {
+  for (int r = t; r < R; r += TPI) {
     uint32_t v[kBRow];
     uint32_t* row = Gp + brow_pos((uint32_t)r) * kBRowStride;
     bload_row(v, row);
@@ -432,7 +467,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   }
   __syncthreads();
   for (int jr = 0; jr < nb; ++jr) {
-    for (int p = t; p < (R >> 1); p += kBatchThreads) {
+    for (int p = t; p < (R >> 1); p += TPI) {
       const uint32_t r = (uint32_t)(((p >> jr) << (jr + 1)) | (p & ((1 << jr) - 1)));
       uint32_t v[kBRow], u[kBRow];
       uint32_t* row = Gp + brow_pos(r) * kBRowStride;
@@ -578,13 +613,13 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   }
 
   // outputs: tables and OPT
-  for (int U = t; U < N; U += kBatchThreads) {
+  for (int U = t; U < N; U += TPI) {
     F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m);
     split_out[tb + U] = split[U];
   }
   if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   __syncthreads();
-  batch_walk(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  batch_walk<TPI>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 }  // namespace
@@ -610,7 +645,7 @@ cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, 
 
 size_t batch_rows_smem_bytes(int m, int occ_cap) {
   const size_t R = (size_t)1 << (m - 5);
-  return 2 * R * kBRowStride * 4 + (size_t)kBMaxLevelRows * kBkStride * 4 + (size_t)occ_cap * 16 +
+  return 2 * R * kBRowStride * 4 + (size_t)batch_level_rows(m - 5) * kBkStride * 4 + (size_t)occ_cap * 16 +
          (size_t)occ_cap * 8 + ((size_t)2 << m) + 64;
 }
 
@@ -622,11 +657,21 @@ cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weig
                               int32_t* dfs, int32_t* status, cudaStream_t stream) {
   if (m < 6 || m > 13) return cudaErrorInvalidValue;
   const size_t smem = batch_rows_smem_bytes(m, occ_cap);
-  cudaError_t e = cudaFuncSetAttribute(k_batch_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const int tpi = batch_rows_threads(m);
+  cudaError_t e = cudaSuccess;
+  auto go = [&](auto kernel) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess)
+      kernel<<<(unsigned)count, tpi, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off, inst_list, occ_cap, m,
+                                                      opt, F, split, perm, dfs, status);
+  };
+  if (tpi == 64)
+    go(k_batch_rows<64>);
+  else if (tpi == 128)
+    go(k_batch_rows<128>);
+  else
+    go(k_batch_rows<256>);
   if (e != cudaSuccess) return e;
-  k_batch_rows<<<(unsigned)count, kBatchThreads, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off,
-                                                                 inst_list, occ_cap, m, opt, F, split, perm, dfs,
-                                                                 status);
   return cudaGetLastError();
 }
 
