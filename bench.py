@@ -38,11 +38,10 @@ METRIC = "subset-splits evaluated/sec (≈3^m/2 per solve) and exact-MPT solve t
 WORKLOAD = 4
 ORACLE_SAMPLE_REQUESTS = 22  # reference arm: full oracle recurrence on the first 22 requests per step
 CPU_BASELINE_REQUESTS = 23  # cpu_baseline: one run on the first 23 requests (10-30 s of CPU work)
-# Integer ALU pipe: 152 SMs x 4 sub-partitions x 16 lanes per clock, at the
-# 2.07 GHz maximum SM clock.  Each split is one 32-bit add and min, which the
-# pair kernel issues as one instruction on that pipe (ncu: its arithmetic runs
-# on the ALU pipe; about 1.3 instructions per split in all).
-ALU_PEAK_TOPS = 152 * 64 * 2.070e9 / 1e12
+# Each split is one 32-bit add and min, which the pair kernel issues as one
+# instruction on the integer ALU pipe (ncu: its arithmetic runs on that pipe).
+# The pipe peak (SMs x 4 sub-partitions x 16 lanes per clock at the maximum SM
+# clock) is computed from the device where the roofline is reported.
 OPS_PER_SPLIT = 1
 
 
@@ -315,11 +314,18 @@ def run_ours(args):
         ops_per_launch = OPS_PER_SPLIT * prof_sum["splits_pairs"] / launches
         achieved = ops_per_launch / (avg_ms / 1000.0) / 1e12
         tr = load_traffic_profile()
-        roofline = {"bound": "alu", "kernel": "k_dp_pairs", "achieved": achieved, "peak": ALU_PEAK_TOPS,
-                    "unit": "Tops/s", "frac": achieved / ALU_PEAK_TOPS,
+        # integer ALU pipe: SMs (from the device) x 4 sub-partitions x 16 lanes
+        # per clock at the maximum SM clock nvidia-smi reports (2,070 MHz if
+        # it reports none)
+        sms = torch.cuda.get_device_properties(device).multi_processor_count
+        max_mhz = (clock_info or {}).get("sm_max_mhz") or 2070.0
+        alu_peak = sms * 64 * max_mhz * 1e6 / 1e12
+        roofline = {"bound": "alu", "kernel": "k_dp_pairs", "achieved": achieved, "peak": alu_peak,
+                    "unit": "Tops/s", "frac": achieved / alu_peak,
                     "traffic": (tr or {}).get("dram_bytes_per_launch"),
                     "ops_per_split": OPS_PER_SPLIT,
-                    "peak_basis": "152 SMs x 64 integer-ALU-pipe lanes x 2.07 GHz (one add-min per split)",
+                    "peak_basis": f"{sms} SMs x 64 integer-ALU-pipe lanes x {max_mhz / 1000:.3f} GHz "
+                                  "(one add-min per split)",
                     "share_of_step": prof_sum["ms_dp_pairs"] / (local_ms if local_ms > 0 else 1)}
     else:
         hbm = float(peaks.get("hbm_gbs", 6800.0))
@@ -327,7 +333,10 @@ def run_ours(args):
         roofline = {"bound": "hbm", "kernel": "k_dp_layer_*", "achieved": gbs, "peak": hbm, "unit": "GB/s",
                     "frac": gbs / hbm, "traffic": None, "bytes_per_split": 16}
     hbm = float(peaks.get("hbm_gbs", 6800.0))
-    gather_frac = (16.0 * value / world) / (hbm * 1e9)
+    # the naive recurrence reads 16 B per split at scattered subsets: against
+    # the measured random-gather bandwidth of a table of this size
+    gather_gbs = mpt.mpt_gather_bandwidth(min(m, 30), 1 << 28, stream.cuda_stream)
+    gather_frac = (16.0 * value / world) / (gather_gbs * 1e9)
 
     # CPU baseline: the oracle, timed on this host, bounded sample
     cpu = None
@@ -362,6 +371,8 @@ def run_ours(args):
                    "opt": opts[-1] if opts else None},
         "roofline": roofline,
         "gather_roofline_frac": gather_frac,
+        "gather_roofline": {"measured_gbs": gather_gbs, "table": f"2^{min(m, 30)} int64 entries",
+                            "bytes_per_split": 16, "vs_copy_peak_frac": (16.0 * value / world) / (hbm * 1e9)},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": "splits/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": e2e_steps, "path": "mpt_create(host arrays) + mpt_solve + mpt_layout(host arrays)"},

@@ -363,6 +363,16 @@ mpt_status mpt_layout_pinned(const int64_t* weights, int64_t n_chunks, int32_t m
 mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chunks, const uint64_t* d_req_bits, int32_t m,
                              int64_t* d_F, int64_t* d_wI, uint32_t* d_split, int64_t* d_opt, void* stream);
 
+/* Measurement helper, not part of the method: the useful bandwidth of
+ * uniformly random, independent 8-byte loads from a table of 2^log2_entries
+ * int64 entries -- the access pattern of the Sec. 3.1 recurrence without
+ * blocking (two table reads per split).  About `loads` loads (indices from a
+ * counter-based hash) are timed with CUDA events on `stream` after one
+ * warm-up pass; the table is allocated, filled and freed by the call on the
+ * current device.  gbps: 8 bytes per load / elapsed seconds / 1e9.
+ * 10 <= log2_entries <= 32.  Errors: INVALID_ARG, OUT_OF_MEMORY, CUDA. */
+mpt_status mpt_gather_bandwidth(int32_t log2_entries, int64_t loads, void* stream, double* gbps);
+
 /* Free the context and any workspace the library allocated.  NULL is a no-op. */
 void mpt_destroy(mpt_ctx* ctx);
 

@@ -42,7 +42,7 @@ EXPORTED = [
     "mpt_last_error", "mpt_solve_noalloc", "mpt_batch_create", "mpt_batch_workspace_bytes", "mpt_batch_solve",
     "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
     "mpt_cache_costs", "mpt_layout_pinned", "mpt_solve_steps", "mpt_solve_begin", "mpt_solve_layers",
-    "mpt_solve_end", "mpt_solve_resume", "mpt_set_tables", "mpt_tables32",
+    "mpt_solve_end", "mpt_solve_resume", "mpt_set_tables", "mpt_tables32", "mpt_gather_bandwidth",
 ]
 
 
@@ -128,6 +128,7 @@ def load() -> ctypes.CDLL:
         "mpt_solve_resume": ([vp, vp, sz, i32], ctypes.c_int),
         "mpt_set_tables": ([vp, i32], ctypes.c_int),
         "mpt_tables32": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp)], ctypes.c_int),
+        "mpt_gather_bandwidth": ([i32, i64, vp, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -651,3 +652,12 @@ def mpt_layout_pinned(weights, ranked, t: int, method: str = "exact",
            "mpt_layout_pinned")
     strings = [perm[offs[i]:offs[i + 1]].tolist() for i in range(m)]
     return PinnedResult(strings, order[:m], int(cost.value))
+
+
+def mpt_gather_bandwidth(log2_entries: int, loads: int = 1 << 28, stream: Optional[int] = None) -> float:
+    """Measured GB/s of uniformly random 8-byte loads from a 2^log2_entries int64 table."""
+    out = ctypes.c_double()
+    s = 0 if stream is None else int(stream)
+    _check(load().mpt_gather_bandwidth(int(log2_entries), int(loads), ctypes.c_void_p(s), ctypes.byref(out)),
+           "mpt_gather_bandwidth")
+    return float(out.value)
