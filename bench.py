@@ -22,6 +22,7 @@ import argparse
 import json
 import math
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -162,15 +163,30 @@ class ClockSampler:
 # CPU oracle legs
 # ---------------------------------------------------------------------------
 
-def oracle_sample(inst, m_sub: int):
-    """The oracle's full recurrence on the first ``m_sub`` requests of the instance."""
+def oracle_sample(inst, m_sub: int, threads: int = 0):
+    """The oracle's full recurrence on the first ``m_sub`` requests of the
+    instance (all host cores, or ``threads`` of them)."""
     import oracle
 
     bits = np.ascontiguousarray(inst.bits[:m_sub])
     t0 = time.perf_counter()
-    opt, F, wI, split = oracle.solve(inst.weights, bits)
+    opt, F, wI, split = oracle.solve(inst.weights, bits, threads=threads)
     dt = time.perf_counter() - t0
-    return splits_per_solve(m_sub), dt, oracle.max_threads()
+    return splits_per_solve(m_sub), dt, (threads or oracle.max_threads())
+
+
+def cpu_model() -> str:
+    """The host CPU as the OS names it (model name, else the Arm part id)."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+    except OSError:
+        return platform.processor() or platform.machine()
+    for key in ("model name", "Model", "CPU part"):
+        for line in info.splitlines():
+            if line.startswith(key):
+                return f"{platform.machine()} {key}: {line.split(':', 1)[1].strip()}"
+    return platform.machine()
 
 
 def run_reference(args):
@@ -342,9 +358,12 @@ def run_ours(args):
     cpu = None
     if not args.no_cpu_baseline and world == 1:
         s_sub, dt, cores = oracle_sample(inst, CPU_BASELINE_REQUESTS)
+        s1, dt1, _ = oracle_sample(inst, 19, threads=1)
         cpu = {"value": s_sub / dt, "unit": "splits/s", "cores": cores, "kind": "oracle",
                "sample": f"full oracle recurrence on the first {CPU_BASELINE_REQUESTS} of the {m} requests "
-                         f"({s_sub} splits, {dt:.1f} s)"}
+                         f"({s_sub} splits, {dt:.1f} s)",
+               "single_thread": {"value": s1 / dt1, "sample": f"first 19 requests ({s1} splits, {dt1:.1f} s)"},
+               "cpu": cpu_model()}
 
     solve_s = max_ms / 1000.0 / args.steps
     line = {
