@@ -522,27 +522,40 @@ def run_cache(args):
     torch.cuda.set_device(0)
     if not B.LIB.exists():
         B.build()
-    weights, ranked = instances.stream("nfcorpus-shaped", seed=0)
+    if args.cache_m:
+        # a longer stream of the same shape: pools scaled with the request count
+        c = dict(instances.STREAMS["nfcorpus-shaped"])
+        scale = args.cache_m / c["m"]
+        weights, ranked = instances.rag_ranked(args.cache_m, int(c["n"] * scale), max(1, int(c["pools"] * scale)),
+                                               c["pool_size"], c["k"], c["tail_s"], seed=0, w_mean=c["w_mean"],
+                                               wmin=c["wmin"], wmax=c["wmax"])
+    else:
+        weights, ranked = instances.stream("nfcorpus-shaped", seed=0)
     n, m = len(weights), len(ranked)
     one = float(np.mean([sum(int(weights[x]) for x in q) for q in ranked]))
     mult = [0.25, 0.5, 0.75, 0.9, 1, 4, 16, 64, 256, 1024]
     caps = [int(round(f * one)) for f in mult]
-    layouts = {"production": [list(r) for r in ranked], "greedy": mpt.mpt_greedy(weights, ranked).perms}
-    for t in (1, 2, 3):
-        layouts[f"pin_top{t}"] = mpt.mpt_layout_pinned(weights, ranked, t, "greedy").strings
+    layouts = {"production": [list(r) for r in ranked]}
+    if m <= 16384:  # the greedy hierarchy's limit
+        layouts["greedy"] = mpt.mpt_greedy(weights, ranked).perms
+        for t in (1, 2, 3):
+            layouts[f"pin_top{t}"] = mpt.mpt_layout_pinned(weights, ranked, t, "greedy").strings
     total = int(sum(int(weights[x]) for q in ranked for x in q))
     arrival = list(range(m))
-    g = layouts["greedy"]
+    g = layouts.get("greedy", layouts["production"])
+    # timed: the C ABI calls on a CSR built once (host arrays in and out)
+    g_csr = mpt.to_csr(g)
+    arr = np.arange(m, dtype=np.int32)
     for _ in range(args.warmup):
-        mpt.mpt_cache_costs(weights, g, caps, arrival)
+        mpt.mpt_cache_costs(weights, g_csr, caps, arr)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        mpt.mpt_cache_costs(weights, g, caps, arrival)
+        mpt.mpt_cache_costs(weights, g_csr, caps, arr)
     dt = (time.perf_counter() - t0) / args.steps
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        thm7 = mpt.mpt_serve_order(n, g)
+        thm7 = mpt.mpt_serve_order(n, g_csr)
     dt_order = (time.perf_counter() - t0) / args.steps
 
     table = {}
@@ -556,13 +569,15 @@ def run_cache(args):
         row["saving_vs_no_sharing"] = 1 - unb / total
         table[name] = row
     windows = {}
-    for W in (1, 128, 512, 2048, m):
+    for W in sorted({1, 128, 512, 2048, m}):
         order = mpt.mpt_serve_order(n, g, arrival, W).tolist()
         costs, unb = mpt.mpt_cache_costs(weights, g, caps[4:], order)
         windows["all" if W == m else str(W)] = {f"{f}x": round(c / unb - 1, 4) for f, c in zip(mult[4:], costs)}
     line = {"mode": "cache", "metric": "finite radix cache, prefill cost at 10 capacities per call",
             "value": dt, "unit": "s", "higher_is_better": False, "steps": args.steps,
-            "workload": f"nfcorpus-shaped stream: m = {m} requests, k = 8, one request = {one:.0f} tokens",
+            "timed_layout": "greedy" if "greedy" in layouts else "production",
+            "workload": f"nfcorpus-shaped stream: m = {m} requests, k = 8, one request = {one:.0f} tokens"
+                        + (" (scaled)" if args.cache_m else ""),
             "accesses": int(sum(len(q) for q in g)), "serve_order_s": dt_order,
             "capacities_in_requests": mult, "no_sharing_cost": total, "layouts": table,
             "window_excess_over_unbounded_greedy": windows,
@@ -596,6 +611,8 @@ def main():
                          "cache: finite-cache study on a request stream")
     ap.add_argument("--batch-size", type=int, default=20000)
     ap.add_argument("--greedy-m", type=int, default=3000)
+    ap.add_argument("--cache-m", type=int, default=0,
+                    help="cache mode: requests in a scaled stream (default: the 2,921-request stream)")
     args = ap.parse_args()
     if args.mode == "batch":
         run_batch(args)

@@ -12,6 +12,7 @@ there is no fallback: loading fails loudly if it is missing.
 from __future__ import annotations
 
 import ctypes
+import itertools
 from dataclasses import dataclass
 from typing import Optional
 
@@ -574,13 +575,32 @@ def mpt_greedy(weights, requests, stream: Optional[int] = None) -> GreedyResult:
 
 
 def _csr(strings):
-    """(offsets, ids) int64 arrays of a list of chunk-id lists; ids has >= 1 entry."""
+    """(offsets, ids) int64 arrays of a list of chunk-id lists (or such a pair
+    already built: a tuple of two arrays); ids has >= 1 entry."""
+    if isinstance(strings, tuple) and len(strings) == 2 and isinstance(strings[0], np.ndarray):
+        offs = np.ascontiguousarray(strings[0], dtype=np.int64)
+        ids = np.ascontiguousarray(strings[1], dtype=np.int64)
+        return offs, (ids if ids.size else np.zeros(1, dtype=np.int64))
+    lens = np.fromiter((len(r) for r in strings), dtype=np.int64, count=len(strings))
     offs = np.zeros(len(strings) + 1, dtype=np.int64)
-    for i, r in enumerate(strings):
-        offs[i + 1] = offs[i] + len(r)
-    ids = (np.concatenate([np.asarray(r, dtype=np.int64) for r in strings])
-           if int(offs[-1]) else np.zeros(1, dtype=np.int64))
-    return offs, np.ascontiguousarray(ids, dtype=np.int64)
+    np.cumsum(lens, out=offs[1:])
+    total = int(offs[-1])
+    ids = (np.fromiter(itertools.chain.from_iterable(strings), dtype=np.int64, count=total)
+           if total else np.zeros(1, dtype=np.int64))
+    return offs, ids
+
+
+def to_csr(strings):
+    """(offsets int64[m+1], ids int64) of a list of chunk-id lists, to pass to
+    mpt_serve_order / mpt_cache_costs in place of the list (built once)."""
+    return _csr(strings)
+
+
+def _count(strings) -> int:
+    """Number of strings in a list or in an (offsets, ids) pair."""
+    if isinstance(strings, tuple) and len(strings) == 2 and isinstance(strings[0], np.ndarray):
+        return int(strings[0].shape[0]) - 1
+    return len(strings)
 
 
 def mpt_serve_order(n_chunks: int, strings, arrival=None, window: int = 0,
@@ -589,7 +609,7 @@ def mpt_serve_order(n_chunks: int, strings, arrival=None, window: int = 0,
     sorted only inside consecutive windows of ``window`` arrivals of ``arrival``."""
     lib = load()
     offs, ids = _csr(strings)
-    m = len(strings)
+    m = _count(strings)
     arr = None if arrival is None else np.ascontiguousarray(arrival, dtype=np.int32)
     out = np.zeros(max(m, 1), dtype=np.int32)
     s = 0 if stream is None else int(stream)
@@ -606,7 +626,7 @@ def mpt_cache_costs(weights, strings, capacities, order=None, stream: Optional[i
     lib = load()
     w = np.ascontiguousarray(weights, dtype=np.int64)
     offs, ids = _csr(strings)
-    m = len(strings)
+    m = _count(strings)
     caps = np.ascontiguousarray(capacities, dtype=np.int64)
     if caps.size == 0:
         caps = np.zeros(1, dtype=np.int64)
