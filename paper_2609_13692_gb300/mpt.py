@@ -553,12 +553,8 @@ def mpt_greedy(weights, requests, stream: Optional[int] = None) -> GreedyResult:
     chunk-id lists) over the universe of ``weights``."""
     lib = load()
     w = np.ascontiguousarray(weights, dtype=np.int64)
-    offs = np.zeros(len(requests) + 1, dtype=np.int64)
-    for i, r in enumerate(requests):
-        offs[i + 1] = offs[i] + len(r)
-    ids = np.ascontiguousarray(np.concatenate([np.asarray(r, dtype=np.int64) for r in requests])
-                               if int(offs[-1]) else np.zeros(1, dtype=np.int64), dtype=np.int64)
-    m = len(requests)
+    offs, ids = _csr(requests)
+    m = _count(requests)
     cost, sav, lb = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
     merges = np.zeros(max(1, 2 * (m - 1)), dtype=np.int32)
     vals = np.zeros(max(1, m - 1), dtype=np.int64)
