@@ -87,6 +87,12 @@ def test_cache_costs_parity_small(mpt):
             costs, unb = mpt.mpt_cache_costs(w, s, caps, order)
             assert unb == trie
             assert costs.tolist() == O.radix_cache_costs(w, s, order, caps), (n, m)
+        # no capacities: only the unbounded cost; a prebuilt CSR gives the same answers
+        costs, unb = mpt.mpt_cache_costs(w, s, [], None)
+        assert costs.size == 0 and unb == trie
+        csr = mpt.to_csr(s)
+        assert mpt.mpt_cache_costs(w, csr, caps[:5], None)[0].tolist() == O.radix_cache_costs(w, s, list(range(m)), caps[:5])
+        assert mpt.mpt_serve_order(n, csr).tolist() == O.serve_order(s)
 
 
 def test_cache_costs_parity_stream(mpt):
