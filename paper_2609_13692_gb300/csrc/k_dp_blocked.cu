@@ -47,7 +47,7 @@ constexpr int kSharedOut = kSharedRows * kRow;
 constexpr int kSharedStride = kRow + 1;    // words per shared row in the per-pair minimum arrays
 constexpr int kSharedWords = kSharedRows * kSharedStride;
 constexpr int kSharedOwned = (kSharedOut + kPairThreads - 1) / kPairThreads;
-constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedWords) * (int)sizeof(uint32_t);
+constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedWords + kRow * kPairThreads) * (int)sizeof(uint32_t);
 constexpr int kMinPairsPerItem = 16;
 constexpr int kTileThreads = 512;
 constexpr int kMaxTileBits = 12;
@@ -232,6 +232,9 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   // window buffer c: X at smem + 2c * kWin, Y right after it; then two
   // per-pair minimum arrays of the shared rows
   uint32_t* smin = smem + 4 * kWin;
+  // Ta of each register output's running best, [output][thread]: written only
+  // when a pair strictly improves the best, by a predicated store
+  uint32_t* sbest_t = smin + 2 * kSharedWords;
 
   const uint32_t tile = blockIdx.x / items_per_tile;
   const uint32_t item = blockIdx.x % items_per_tile;
@@ -255,11 +258,11 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t es1 = extra & 0xFFu, ea1 = (extra >> 8) & 0xFFu, erow = (extra >> 16) & 0xFFu;
 
   for (int i = threadIdx.x; i < 2 * kSharedWords; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
-  uint32_t bk[kRow], bt[kRow], sbk[kSharedOwned], sbt[kSharedOwned];
+  uint32_t bk[kRow], sbk[kSharedOwned], sbt[kSharedOwned];
 #pragma unroll
   for (int i = 0; i < kRow; ++i) {
     bk[i] = 0xFFFFFFFFu;
-    bt[i] = 0;
+    sbest_t[i * kPairThreads + threadIdx.x] = 0;
   }
 #pragma unroll
   for (int j = 0; j < kSharedOwned; ++j) {
@@ -310,9 +313,8 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
 #pragma unroll
       for (int i = 0; i < kRow; ++i) {
         bool keep;  // true when the running best is <= this pair's minimum
-        const uint32_t m = __vibmin_u32(bk[i], acc[i], &keep);
-        bt[i] = keep ? bt[i] : Ta;
-        bk[i] = m;
+        bk[i] = __vibmin_u32(bk[i], acc[i], &keep);
+        if (!keep) sbest_t[i * kPairThreads + threadIdx.x] = Ta;
       }
       if (has_extra) {
         uint32_t x[kRow], y[kRow];
@@ -350,7 +352,7 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   __syncthreads();
 #pragma unroll
   for (int i = 0; i < kRow; ++i)
-    atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | bt[i]);
+    atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | sbest_t[i * kPairThreads + threadIdx.x]);
 #pragma unroll
   for (int j = 0; j < kSharedOwned; ++j) {
     const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
