@@ -126,17 +126,23 @@ mpt_status mpt_solve_resume(mpt_ctx* ctx, void* d_workspace, size_t workspace_by
  *   wI[S]    = w(I(S)); wI[0] = weight of the union of all requests,
  *   split[S] = the reported optimal split (see conventions).
  * The pointers live in the workspace and stay valid until the next solve or
- * mpt_destroy.  Any argument may be NULL.  Errors: INVALID_ARG (also when
- * the context uses MPT_TABLES_LEAN: see mpt_tables32), NOT_SOLVED. */
-mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split);
+ * mpt_destroy.  Any argument may be NULL.  The blocked recurrence keeps its
+ * tables in a tile-major (rotated) order; the first call after such a solve
+ * writes the natural-order views inside the workspace (a transpose of about
+ * 36 bytes per subset, ~1.5 ms at m = 28) on a stream of the context, on the
+ * device of the solve, and waits for it; later calls only return the
+ * pointers.  Errors: INVALID_ARG (also when the context uses
+ * MPT_TABLES_LEAN: see mpt_tables32), NOT_SOLVED, CUDA. */
+mpt_status mpt_tables(mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split);
 
 /* Table layout of the solve (Sec. 3.1 tables; N3 "leaner" form).
  *   MPT_TABLES_INT64 (default): w(I(S)) and F(S) in separate int64[2^m]
  *     tables (mpt_tables);
  *   MPT_TABLES_LEAN: one int32[2^m] table that holds w(I(S)) after K2 and
- *     F(S) once the recurrence has finished S (each entry is overwritten in
- *     place by the thread that finishes it), read with mpt_tables32; w(I(S))
- *     is then no longer available.  Allowed when sum_i w(R_i) < 2^31
+ *     F(S) afterwards (general path: each entry is overwritten in place by
+ *     the thread that finishes it; blocked path: F is written over it when
+ *     mpt_tables32 asks for the natural views), read with mpt_tables32;
+ *     w(I(S)) is then no longer available.  Allowed when sum_i w(R_i) < 2^31
  *     (MPT_ERR_OVERFLOW otherwise), which bounds every w(I(S)) and F(S).
  *     The blocked path's workspace falls from 28 to 16 bytes per subset
  *     (m = 32: 64 GiB instead of 112 GiB).
@@ -146,8 +152,9 @@ mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d
 mpt_status mpt_set_tables(mpt_ctx* ctx, int32_t kind);
 
 /* Device views of the lean tables of the last solve: F int32[2^m] and split
- * uint32[2^m] (as in mpt_tables).  Errors: INVALID_ARG (not lean), NOT_SOLVED. */
-mpt_status mpt_tables32(const mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split);
+ * uint32[2^m] (as in mpt_tables, including the conversion on the first call).
+ * Errors: INVALID_ARG (not lean), NOT_SOLVED, CUDA. */
+mpt_status mpt_tables32(mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split);
 
 /* Number of entries mpt_layout writes to perm_chunks: sum_i |R_i|. */
 mpt_status mpt_layout_size(const mpt_ctx* ctx, int64_t* total_chunks);

@@ -370,20 +370,18 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
 // by level in |U|, folding in the self pair (kh >= 1) or running the whole
 // recurrence on the inner bits (kh = 0).  One block per tile.  Used for tile 0
 // (any b <= 12); the tiles with kh >= 1 go to k_dp_tile_rows.
-// Tab: int64 tables, or the int32 lean table (wI and F the same array: every
-// entry's w(I(S)) is read before its F(S) is written, by the same block).
+// Both tile kernels read w(I) and write split in rotated order, one tile's
+// entries contiguous; F itself stays in Gp (F << b).
+// Tab: int64 w(I) table, or the int32 one of the lean layout.
 template <typename Tab>
 __device__ __forceinline__ int64_t load_wI(const Tab* p) {
-  if constexpr (sizeof(Tab) == 8)
-    return __ldg(p);
-  else
-    return (int64_t)*p;  // lean: the same array is written by this kernel
+  return (int64_t)__ldg(p);
 }
 
 template <typename Tab>
 __global__ void __launch_bounds__(kTileThreads)
-k_dp_tile(int L, int b, int kh, const Tab* wI, const unsigned long long* __restrict__ partial,
-          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, Tab* F, uint32_t* __restrict__ split) {
+k_dp_tile(int L, int b, int kh, const Tab* __restrict__ wIr, const unsigned long long* __restrict__ partial,
+          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot) {
   __shared__ uint32_t cur_p[1 << kMaxTileBits];   // this tile, F << b
   __shared__ uint32_t other_c[1 << kMaxTileBits]; // complement form: this tile (kh = 0) or tile 0 (kh >= 1)
   __shared__ uint16_t order[1 << kMaxTileBits];   // inner subsets sorted by size, then colex
@@ -455,30 +453,28 @@ k_dp_tile(int L, int b, int kh, const Tab* wI, const unsigned long long* __restr
         best = o < best ? o : best;
       }
       if (active && r == 0) {
-        const size_t S = ((size_t)U << L) | T;
+        const size_t idx = ((size_t)T << b) | U;
         int64_t f;
         uint32_t A;
-        if (S == 0) {
+        if (U == 0 && T == 0) {
           f = 0;
           A = 0;
         } else if (single) {
-          f = load_wI(wI + S);
+          f = load_wI(wIr + idx);
           A = 0;
         } else {
           const uint32_t key = (uint32_t)(best >> 32);
           const uint32_t Ua = (key & mask) + U - mask;
-          f = (int64_t)(key >> b) - load_wI(wI + S);
+          f = (int64_t)(key >> b) - load_wI(wIr + idx);
           A = (Ua << L) | (uint32_t)best;
         }
         const uint32_t gp = (uint32_t)f << b;
         const uint32_t gc = gp | (~U & mask);
         cur_p[U] = gp;
         if (kh == 0) other_c[U] = gc;
-        const size_t idx = ((size_t)T << b) | U;
         Gp[idx] = gp;
         Gc[idx] = gc;
-        F[S] = (Tab)f;
-        split[S] = A;
+        split_rot[idx] = A;
       }
     }
     start += (uint32_t)cnt;
@@ -497,17 +493,22 @@ k_dp_tile(int L, int b, int kh, const Tab* wI, const unsigned long long* __restr
 //     smaller than s2).
 // Rows are finished level by level in |s1|, so every row read is final.
 constexpr int kRowsThreads = 96;
-constexpr int kRowsSmemBytes = (2 * kWin + 2 * (1 << kB)) * (int)sizeof(uint32_t);
+constexpr int kBestWords = (1 << kB) + kRows;  // per-output arrays, rows 33 words apart
+constexpr int kRowsSmemBytes = (2 * kWin + 2 * kBestWords) * (int)sizeof(uint32_t);
+
+// Word of output U = (s1, s2) in a per-output array: rows are 33 words apart,
+// so threads that hold different rows and the same s2 hit different banks.
+__device__ __forceinline__ uint32_t best_word(uint32_t U) { return U + (U >> kB2); }
 
 template <typename Tab>
 __global__ void __launch_bounds__(kRowsThreads)
-k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restrict__ partial,
-               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, Tab* F, uint32_t* __restrict__ split) {
+k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long long* __restrict__ partial,
+               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot) {
   extern __shared__ __align__(16) uint32_t smem[];
   uint32_t* cur = smem;               // this tile, F << kB, padded rows
   uint32_t* zc = smem + kWin;         // tile 0, complement form, padded rows
   uint32_t* bkey = smem + 2 * kWin;   // best key per output so far
-  uint32_t* bsplit = bkey + (1 << kB);  // its Ta; after finishing, the split A
+  uint32_t* bsplit = bkey + kBestWords;  // its Ta; after finishing, the split A
   constexpr uint32_t kMask = (1u << kB) - 1u;
 
   const uint32_t tile = blockIdx.x;
@@ -521,21 +522,22 @@ k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restric
   }
   for (int u = threadIdx.x; u < (1 << kB); u += kRowsThreads) {
     const unsigned long long pv = kh >= 2 ? partial[((size_t)tile << kB) | (uint32_t)u] : ~0ull;
-    bkey[u] = (uint32_t)(pv >> 32);
-    bsplit[u] = (uint32_t)pv;
+    bkey[best_word((uint32_t)u)] = (uint32_t)(pv >> 32);
+    bsplit[best_word((uint32_t)u)] = (uint32_t)pv;
   }
   __syncthreads();
 
   for (int p1 = 0; p1 <= kB1; ++p1) {
     const int rows = (int)c_binom.v[kB1][p1];
-    // The threads that finish this level's rows fetch their w(I(S)) now, so
-    // that the strided gathers complete while phase A runs.
+    // The threads that finish this level's rows fetch their w(I(S)) (32
+    // consecutive rotated entries each) now, so that the loads complete while
+    // phase A runs.
     uint32_t wv[kRow];
     const bool finisher = (int)threadIdx.x < rows;
     const uint32_t s1f = finisher ? colex_unrank((unsigned long long)threadIdx.x, p1, kB1) : 0u;
     if (finisher) {
 #pragma unroll
-      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)load_wI(wI + (((size_t)((s1f << kB2) | (uint32_t)i) << L) | T));
+      for (int i = 0; i < kRow; ++i) wv[i] = (uint32_t)load_wI(wIr + (tbase | (s1f << kB2) | (uint32_t)i));
     }
     if (p1 >= 1) {
       // lanes per row chosen so that each lane runs at most 8 row pairs
@@ -578,9 +580,9 @@ k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restric
 #pragma unroll
         for (int i = 0; i < kRow; ++i) {
           const uint32_t U = (s1 << kB2) | (uint32_t)i;
-          if (acc[i] < bkey[U]) {
-            bkey[U] = acc[i];
-            bsplit[U] = T;
+          if (acc[i] < bkey[best_word(U)]) {
+            bkey[best_word(U)] = acc[i];
+            bsplit[best_word(U)] = T;
           }
         }
       }
@@ -598,7 +600,7 @@ k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restric
           if ((a2 & s2) == a2 && a2 != s2) key = min(key, c[a2] + z[s2 ^ a2]);
         }
         const uint32_t U = (s1 << kB2) | (uint32_t)s2;
-        uint32_t bk = bkey[U], bt = bsplit[U];
+        uint32_t bk = bkey[best_word(U)], bt = bsplit[best_word(U)];
         if (key < bk) {
           bk = key;
           bt = T;
@@ -613,7 +615,7 @@ k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restric
           A = (Ua << L) | bt;
         }
         c[s2] = f << kB;
-        bsplit[U] = A;
+        bsplit[best_word(U)] = A;
       }
       uint4* dst = reinterpret_cast<uint4*>(cur + row_pos(s1) * kRowStride);
 #pragma unroll
@@ -626,9 +628,7 @@ k_dp_tile_rows(int L, int kh, const Tab* wI, const unsigned long long* __restric
     const uint32_t gp = cur[row_pos((uint32_t)u >> kB2) * kRowStride + (u & (kRow - 1))];
     Gp[tbase | (uint32_t)u] = gp;
     Gc[tbase | (uint32_t)u] = gp | (~(uint32_t)u & kMask);
-    const size_t S = ((size_t)u << L) | T;
-    F[S] = (Tab)(gp >> kB);
-    split[S] = bsplit[u];
+    split_rot[tbase | (uint32_t)u] = bsplit[best_word((uint32_t)u)];
   }
 }
 
@@ -689,17 +689,17 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches], stream);
     if (kh == 0) {
       if (s.lean)
-        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.fw, nullptr, ws.Gp, ws.Gc, ws.fw, ws.split);
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.fw_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot);
       else
-        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI, nullptr, ws.Gp, ws.Gc, ws.F, ws.split);
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot);
     } else {
       const unsigned long long* part = kh >= 2 ? ws.partial : nullptr;
       if (s.lean)
-        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.fw, part, ws.Gp, ws.Gc,
-                                                                                  ws.fw, ws.split);
+        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.fw_rot, part, ws.Gp,
+                                                                                  ws.Gc, ws.split_rot);
       else
-        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.wI, part, ws.Gp, ws.Gc,
-                                                                                  ws.F, ws.split);
+        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.wI_rot, part, ws.Gp,
+                                                                                  ws.Gc, ws.split_rot);
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;

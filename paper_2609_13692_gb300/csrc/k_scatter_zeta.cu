@@ -8,7 +8,10 @@
 // which is the quantity w(I(B)) of the Sec. 3.1 recurrence.  K1 builds g and
 // the list of chunks that some request uses; K2 is the superset-sum (zeta)
 // transform over the 2^m table, done in shared-memory tiles so that each
-// pass streams the table once with coalesced 128-byte rows.
+// pass streams the table once with coalesced 128-byte rows.  For the blocked
+// recurrence g is indexed in its rotated order (rot_index): the superset
+// relation does not depend on the order of the index bits, so the same
+// transform then yields w(I(S)) at the rotated position of S.
 #include "mpt_internal.cuh"
 
 namespace mpt {
@@ -21,7 +24,7 @@ template <typename G>
 __global__ void __launch_bounds__(kScatterThreads)
 k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m, int64_t words,
           G* __restrict__ g, uint32_t* __restrict__ used_N, int32_t* __restrict__ used_x,
-          int32_t* __restrict__ counters, int64_t slots) {
+          int32_t* __restrict__ counters, int64_t slots, bool rotated, int L, int b) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
     const int64_t word = x >> 6;
@@ -29,7 +32,7 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
     uint32_t N = 0;
     for (int i = 0; i < m; ++i) N |= (uint32_t)((__ldg(&bits[(int64_t)i * words + word]) >> sh) & 1ull) << i;
     if (N) {
-      atomicAdd(&g[N], (G)w[x]);
+      atomicAdd(&g[rotated ? rot_index(N, L, b) : (size_t)N], (G)w[x]);
       const int k = atomicAdd(&counters[0], 1);
       if (k < slots) {
         used_N[k] = N;
@@ -106,14 +109,15 @@ cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t str
   int64_t blocks = (s.n + kScatterThreads - 1) / kScatterThreads;
   if (blocks > 152 * 16) blocks = 152 * 16;
   if (blocks < 1) blocks = 1;
+  void* g = g_table(s, ws);
   if (s.lean)
     k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
-        ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned int*>(ws.fw), ws.used_N, ws.used_x,
-        ws.counters, s.slots);
+        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned int*>(g), ws.used_N, ws.used_x, ws.counters,
+        s.slots, s.blocked, s.L, s.b);
   else
     k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
-        ws.weights, ws.bits, s.n, s.m, s.words, reinterpret_cast<unsigned long long*>(ws.wI), ws.used_N, ws.used_x,
-        ws.counters, s.slots);
+        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned long long*>(g), ws.used_N, ws.used_x,
+        ws.counters, s.slots, s.blocked, s.L, s.b);
   ++*launches;
   return cudaGetLastError();
 }
@@ -138,8 +142,8 @@ static cudaError_t zeta(const Shape& s, G* g, cudaStream_t stream, int* launches
 }
 
 cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
-  if (s.lean) return zeta(s, reinterpret_cast<unsigned int*>(ws.fw), stream, launches);
-  return zeta(s, reinterpret_cast<unsigned long long*>(ws.wI), stream, launches);
+  if (s.lean) return zeta(s, static_cast<unsigned int*>(g_table(s, ws)), stream, launches);
+  return zeta(s, static_cast<unsigned long long*>(g_table(s, ws)), stream, launches);
 }
 
 }  // namespace mpt

@@ -33,6 +33,13 @@ struct mpt_ctx {
   char* resident = nullptr;  // workspace whose input copies hold this context's instance
   int32_t staged_next = -1;  // staged solve: next step of the recurrence (-1: none begun)
   char* staged_base = nullptr;  // staged solve: its workspace
+  // blocked solves leave the tables in rotated order; the natural views are
+  // filled on the first mpt_tables / mpt_tables32 call after the solve, on a
+  // stream of the context, on the device of the solve
+  bool natural = false;
+  int device = 0;
+  cudaStream_t conv_stream = nullptr;
+  int conv_device = -1;
 };
 
 namespace {
@@ -103,9 +110,19 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws) {
     ws->Gp = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->Gc = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->partial = reinterpret_cast<unsigned long long*>(take((size_t)(s.partial_entries > 0 ? s.partial_entries : 1) * 8));
+    // The rotated tables share the buffers of the natural ones: w(I) sits in
+    // the F table (int64) or in fw (lean), split in the split table.  The
+    // natural views, when asked for, go to wI, F or fw (F from Gp) and, for
+    // split, to the Gc table, which the recurrence no longer needs.
+    ws->wI_rot = s.lean ? nullptr : ws->F;
+    ws->fw_rot = s.lean ? ws->fw : nullptr;
+    ws->split_rot = ws->split;
   } else {
     ws->Gp = ws->Gc = nullptr;
     ws->partial = nullptr;
+    ws->wI_rot = nullptr;
+    ws->fw_rot = nullptr;
+    ws->split_rot = nullptr;
   }
   ws->keys = reinterpret_cast<unsigned long long*>(take(slots * 8));
   ws->perm_offsets = reinterpret_cast<int64_t*>(take((size_t)(s.m + 1) * 8));
@@ -266,10 +283,7 @@ mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStrea
     MPT_CK(cudaMemcpyAsync(ws.bits, c->bits.data(), c->bits.size() * 8, cudaMemcpyHostToDevice, stream), "copy bits");
   }
   MPT_CK(cudaMemsetAsync(ws.counters, 0, 8 * 4, stream), "memset counters");
-  if (s.lean)
-    MPT_CK(cudaMemsetAsync(ws.fw, 0, N * 4, stream), "memset g");
-  else
-    MPT_CK(cudaMemsetAsync(ws.wI, 0, N * 8, stream), "memset g");
+  MPT_CK(cudaMemsetAsync(mpt::g_table(s, ws), 0, N * (s.lean ? 4 : 8), stream), "memset g");
   mark(1);
   MPT_CK(mpt::launch_scatter(s, ws, stream, launches), "scatter kernel");
   mark(2);
@@ -399,6 +413,8 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
     p.ms_walk = elapsed(ev[4], ev[5]);
     p.ms_d2h = elapsed(ev[5], ev[6]);
   }
+  c->natural = !s.blocked;
+  cudaGetDevice(&c->device);
   c->solved = true;
   *opt_cost = opt;
   return MPT_OK;
@@ -482,25 +498,71 @@ mpt_status mpt_solve_end(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes
   c->opt = opt;
   c->staged_next = -1;
   std::memset(&c->prof, 0, sizeof(c->prof));
+  c->natural = !c->shape.blocked;
+  cudaGetDevice(&c->device);
   c->solved = true;
   *opt_cost = opt;
   return MPT_OK;
 }
 
-mpt_status mpt_tables(const mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split) {
+}  // extern "C"
+
+namespace {
+
+// Fill the natural-order views of a blocked solve's tables (once per solve).
+mpt_status ensure_natural(mpt_ctx* c) {
+  if (c->natural) return MPT_OK;
+  const mpt::Shape& s = c->shape;
+  const mpt::Workspace& ws = c->ws;
+  int prev = 0;
+  MPT_CK(cudaGetDevice(&prev), "cudaGetDevice");
+  MPT_CK(cudaSetDevice(c->device), "cudaSetDevice");
+  mpt_status st = MPT_OK;
+  cudaError_t e = cudaSuccess;
+  if (c->conv_stream && c->conv_device != c->device) {
+    cudaStreamDestroy(c->conv_stream);
+    c->conv_stream = nullptr;
+  }
+  if (!c->conv_stream) {
+    e = cudaStreamCreateWithFlags(&c->conv_stream, cudaStreamNonBlocking);
+    c->conv_device = c->device;
+  }
+  if (e == cudaSuccess)
+    e = mpt::unrotate_tables(s, ws.split_rot, ws.Gc, ws.wI_rot, s.lean ? nullptr : ws.wI, ws.Gp,
+                             s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr, c->conv_stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->conv_stream);
+  if (e != cudaSuccess) st = cuda_fail(c, e, "natural-order tables");
+  cudaSetDevice(prev);
+  if (st == MPT_OK) c->natural = true;
+  return st;
+}
+
+// Natural split view: the split table (general path) or the Gc table that the
+// conversion wrote it to (blocked path).
+const uint32_t* natural_split(const mpt_ctx* c) { return c->shape.blocked ? c->ws.Gc : c->ws.split; }
+
+}  // namespace
+
+extern "C" {
+
+mpt_status mpt_tables(mpt_ctx* ctx, const int64_t** d_F, const int64_t** d_wI, const uint32_t** d_split) {
   if (!ctx || ctx->tables != MPT_TABLES_INT64) return MPT_ERR_INVALID_ARG;
   if (!ctx->solved) return MPT_ERR_NOT_SOLVED;
+  mpt_status st = ensure_natural(ctx);
+  if (st != MPT_OK) return st;
   if (d_F) *d_F = ctx->ws.F;
   if (d_wI) *d_wI = ctx->ws.wI;
-  if (d_split) *d_split = ctx->ws.split;
+  if (d_split) *d_split = natural_split(ctx);
   return MPT_OK;
 }
 
-mpt_status mpt_tables32(const mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split) {
+mpt_status mpt_tables32(mpt_ctx* ctx, const int32_t** d_F, const uint32_t** d_split) {
   if (!ctx || ctx->tables != MPT_TABLES_LEAN) return MPT_ERR_INVALID_ARG;
   if (!ctx->solved) return MPT_ERR_NOT_SOLVED;
+  mpt_status st = ensure_natural(ctx);
+  if (st != MPT_OK) return st;
   if (d_F) *d_F = ctx->ws.fw;
-  if (d_split) *d_split = ctx->ws.split;
+  if (d_split) *d_split = natural_split(ctx);
   return MPT_OK;
 }
 
@@ -557,6 +619,7 @@ void mpt_destroy(mpt_ctx* ctx) {
   if (!ctx) return;
   if (ctx->own_ws) cudaFree(ctx->own_ws);
   for (cudaEvent_t e : ctx->events) cudaEventDestroy(e);
+  if (ctx->conv_stream) cudaStreamDestroy(ctx->conv_stream);
   delete ctx;
 }
 

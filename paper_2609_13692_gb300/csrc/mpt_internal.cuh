@@ -91,15 +91,21 @@ struct Workspace {
   int32_t* used_x;    // [slots]  chunk id
   int32_t* counters;  // [8]      0: number of used chunks, 1: device error flags
   // tables, natural subset order (int64 tables: wI and F; lean: fw alone,
-  // w(I(S)) until the recurrence writes F(S) over it)
+  // w(I(S)) until the recurrence writes F(S) over it).  The blocked path
+  // leaves them in rotated order (below) and fills the natural views only
+  // when they are asked for (unrotate_tables).
   int64_t* wI;        // [2^m] or nullptr
   int64_t* F;         // [2^m] or nullptr
   int32_t* fw;        // [2^m] (lean) or nullptr
   uint32_t* split;    // [2^m]
-  // blocked DP working tables, rotated order (see k_dp_blocked.cu)
+  // blocked DP working tables, rotated order idx(S) = (T << b) | U with
+  // T = S mod 2^L and U = S >> L (see k_dp_blocked.cu)
   uint32_t* Gp;       // [2^m]  F << b
   uint32_t* Gc;       // [2^m]  (F << b) | (~u & (2^b - 1))
   unsigned long long* partial;  // [max tiles of one layer << b]
+  int64_t* wI_rot;    // [2^m] w(I(S)) at idx(S) (int64 tables), or nullptr
+  int32_t* fw_rot;    // [2^m] w(I(S)) at idx(S) (lean tables), or nullptr
+  uint32_t* split_rot;  // [2^m] split[S] at idx(S)
   // layout
   unsigned long long* keys;  // [slots]
   int64_t* perm_offsets;     // [m + 1]
@@ -121,6 +127,18 @@ struct Shape {
 };
 
 size_t carve_workspace(const Shape& s, char* base, Workspace* ws);
+
+// Rotated position of subset S in the blocked path's tables.
+__host__ __device__ __forceinline__ size_t rot_index(uint32_t S, int L, int b) {
+  return ((size_t)(S & ((1u << L) - 1u)) << b) | (size_t)(S >> L);
+}
+
+// The table K1 scatters into and K2 transforms: w(I) in rotated order for the
+// blocked path, natural order for the general one.
+inline void* g_table(const Shape& s, const Workspace& ws) {
+  if (s.lean) return s.blocked ? (void*)ws.fw_rot : (void*)ws.fw;
+  return s.blocked ? (void*)ws.wI_rot : (void*)ws.wI;
+}
 
 // ---------------------------------------------------------------------------
 // Launchers.  All enqueue on `stream` and return the launch error (if any).
@@ -150,6 +168,15 @@ int64_t blocked_partial_entries(int m, int b);
 int blocked_tile_bits(int m);
 
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
+
+// Natural-order tables from the blocked path's rotated ones (k_tables.cu):
+// split_nat[S] = split_rot[idx(S)]; wI_nat[S] = wI_rot[idx(S)] (int64
+// tables); F_nat[S] or F32_nat[S] = Gp[idx(S)] >> b.  Null destinations are
+// skipped; they run in this order, so a destination may be the source of an
+// earlier conversion.
+cudaError_t unrotate_tables(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat, const int64_t* wI_rot,
+                            int64_t* wI_nat, const uint32_t* Gp, int64_t* F_nat, int32_t* F32_nat,
+                            cudaStream_t stream);
 // eq. (1) for any number of strings by lexicographic sorting (k_sched.cu)
 mpt_status trie_cost_lex(const int64_t* weights, int64_t n_chunks, int64_t m, const int64_t* offsets,
                          const int64_t* chunks, cudaStream_t st, int64_t* cost);

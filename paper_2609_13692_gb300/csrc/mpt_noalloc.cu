@@ -156,19 +156,28 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   ws.Gp = reinterpret_cast<uint32_t*>(base + kOffGp);
   ws.Gc = reinterpret_cast<uint32_t*>(base + kOffGc);
   ws.partial = reinterpret_cast<unsigned long long*>(base + kOffPartial);
+  // The blocked recurrence works on rotated tables: w(I) in the caller's F
+  // table, split in its wI table; the natural outputs are written from them
+  // at the end (split, then wI, then F from Gp).
+  ws.wI_rot = s.blocked ? d_F : nullptr;
+  ws.fw_rot = nullptr;
+  ws.split_rot = s.blocked ? reinterpret_cast<uint32_t*>(d_wI) : nullptr;
 
   // The scratch keeps the previous call's contents: the counters must start
-  // at zero, and wI is accumulated into (the partial minima are reset by the
-  // blocked launcher before each layer; Gp and Gc are fully rewritten).
+  // at zero, and w(I) is accumulated into (the partial minima are reset by
+  // the blocked launcher before each layer; Gp and Gc are fully rewritten).
   int launches = 0;
   if (cudaMemsetAsync(ws.counters, 0, 8 * sizeof(int32_t), stream) != cudaSuccess ||
-      cudaMemsetAsync(ws.wI, 0, sizeof(int64_t) << m, stream) != cudaSuccess)
+      cudaMemsetAsync(mpt::g_table(s, ws), 0, sizeof(int64_t) << m, stream) != cudaSuccess)
     return MPT_ERR_CUDA;
   if (mpt::launch_scatter(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;
   if (mpt::launch_zeta(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;
   cudaError_t e = s.blocked ? mpt::launch_dp_blocked(s, ws, stream, &launches, nullptr)
                             : mpt::launch_dp_general(s, ws, stream, &launches);
   if (e != cudaSuccess) return MPT_ERR_CUDA;
+  if (s.blocked &&
+      mpt::unrotate_tables(s, ws.split_rot, d_split, ws.wI_rot, d_wI, ws.Gp, d_F, nullptr, stream) != cudaSuccess)
+    return MPT_ERR_CUDA;
   const size_t full = ((size_t)1 << m) - 1;
   if (cudaMemcpyAsync(d_opt, d_F + full, sizeof(int64_t), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
     return MPT_ERR_CUDA;
