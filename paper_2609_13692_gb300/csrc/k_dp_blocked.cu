@@ -632,6 +632,37 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
   }
 }
 
+// Items (blocks) per tile of one pair-kernel layer.  One block runs per SM,
+// every block of a layer takes about the same time per pair, and a block costs
+// about kItemOverheadPairs pairs more (its first window copy and its final
+// merge).  The layer then takes ceil(blocks / SMs) waves of (pairs per item +
+// overhead); take the item count that minimises that, fewer blocks on ties.
+// Items keep at least kMinPairsPerItem pairs.
+constexpr unsigned long long kItemOverheadPairs = 2;
+
+void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long long* items_out, uint32_t* ppi_out) {
+  const unsigned long long waves_of = sms > 0 ? (unsigned long long)sms : 1ull;
+  unsigned long long cap = (P + kMinPairsPerItem - 1) / kMinPairsPerItem;
+  if (cap < 1) cap = 1;
+  if (cap > 8192) cap = 8192;
+  unsigned long long best_t = ~0ull, best_items = 1;
+  uint32_t best_ppi = P;
+  for (unsigned long long it = 1; it <= cap; ++it) {
+    const uint32_t ppi = (uint32_t)((P + it - 1) / it);
+    const unsigned long long items = (P + ppi - 1) / ppi;
+    if (items != it) continue;  // the same split as a smaller count
+    const unsigned long long waves = (tiles * items + waves_of - 1) / waves_of;
+    const unsigned long long t = waves * ((unsigned long long)ppi + kItemOverheadPairs);
+    if (t < best_t) {
+      best_t = t;
+      best_items = items;
+      best_ppi = ppi;
+    }
+  }
+  *items_out = best_items;
+  *ppi_out = best_ppi;
+}
+
 }  // namespace
 
 int blocked_tile_bits(int m) { return m < kB ? m : kB; }
@@ -660,18 +691,20 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
   }
   const int b = s.b, L = s.L;
   constexpr unsigned long long evals_per_pair = 531441ull;  // 3^12 splits per pair of windows
+  int sms = 0, dev = 0;
+  {
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+  }
   if (step_end < 0 || step_end > L + 1) step_end = L + 1;
   for (int kh = step_begin < 0 ? 0 : step_begin; kh < step_end; ++kh) {
     const unsigned long long tiles = h_binom.v[L][kh];
     if (kh >= 2) {
       const uint32_t P = (1u << (kh - 1)) - 1u;
-      const unsigned long long target = 152ull * 8;
-      unsigned long long items = (target + tiles - 1) / tiles;
-      const unsigned long long cap = (P + kMinPairsPerItem - 1) / kMinPairsPerItem;
-      if (items > cap) items = cap;
-      if (items < 1) items = 1;
-      const uint32_t ppi = (uint32_t)((P + items - 1) / items);
-      items = (P + ppi - 1) / ppi;
+      unsigned long long items = 1;
+      uint32_t ppi = P;
+      choose_items(tiles, P, sms, &items, &ppi);
       cudaError_t e = cudaMemsetAsync(ws.partial, 0xFF, (size_t)(tiles << b) * sizeof(unsigned long long), stream);
       if (e != cudaSuccess) return e;
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches], stream);
