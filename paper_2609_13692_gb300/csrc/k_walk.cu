@@ -7,7 +7,9 @@
 // i at the highest node B on i's root-to-leaf path with B inside N_x (the
 // request set of x), and request i's permutation is R_i sorted by
 // (depth of that node, chunk id).  The left-to-right leaf order is the trie
-// DFS order that Thm 7 (Sec. 8) serves requests in.
+// DFS order that Thm 7 (Sec. 8) serves requests in.  After a blocked solve
+// split is read at the rotated position of each node and OPT = F(full) from
+// Gp = F << b; after a general one both are in natural order.
 //
 // Trie cost: a string's node at depth p is new exactly when no earlier
 // string shares its first p+1 symbols, so the trie weight is
