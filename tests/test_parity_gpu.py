@@ -67,6 +67,34 @@ def test_config2_leave_one_out(mpt):
     assert res.opt == O.loo_free(20) == 88
 
 
+def test_table_views_follow_each_solve(mpt):
+    """The blocked solve keeps its tables tile-major and fills the natural
+    views on the first table request: repeated requests return the same
+    views, and a second solve on the same context -- whose working tables
+    reuse the views' buffers -- fills them again, bit-exact (int64 and lean)."""
+    rng = np.random.default_rng(77)
+    m, n = 17, 60
+    reqs = [[int(x) for x in rng.choice(n, size=int(rng.integers(3, 9)), replace=False)] for _ in range(m)]
+    inst = I.Instance(rng.integers(1, 50, size=n).astype(np.int64), I.pack_requests(reqs, n))
+    opt, oF, owI, osplit = O.solve(inst.weights, inst.bits)
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    for rnd in range(2):
+        assert mpt.mpt_solve(ctx) == opt
+        first = mpt.mpt_tables(ctx)
+        again = mpt.mpt_tables(ctx)
+        assert [t.data_ptr() for t in first] == [t.data_ptr() for t in again]
+        F, wI, split = (t.cpu().numpy() for t in again)
+        assert np.array_equal(F, oF) and np.array_equal(wI, owI)
+        assert np.array_equal(split.view(np.uint32), osplit), rnd
+    mpt.mpt_set_tables(ctx, "lean")
+    for rnd in range(2):
+        assert mpt.mpt_solve(ctx) == opt
+        mpt.mpt_tables32(ctx)
+        F, split = (t.cpu().numpy() for t in mpt.mpt_tables32(ctx))
+        assert np.array_equal(F.astype(np.int64), oF)
+        assert np.array_equal(split.view(np.uint32), osplit), rnd
+
+
 @pytest.mark.parametrize("m", list(range(1, 19)))
 def test_random_sweep_blocked(mpt, m):
     rng = np.random.default_rng(1000 + m)
