@@ -6,7 +6,9 @@
 // Index layout.  Requests are split into a "tile" part T (requests 0..L-1)
 // and an "inner" part U (requests L..m-1, b = m - L <= 12 of them).  The
 // working tables are stored in rotated order idx(S) = (T << b) | U, so the
-// 2^b subsets sharing one T are contiguous (one 16 KB window per T).
+// 2^b subsets sharing one T are contiguous (one 16 KB window per T).  The
+// w(I) table the kernels read and the split table they write use the same
+// order; F itself exists only as Gp = F << b (below).
 //
 // Split structure.  A split of S = (T, U) is named by its part A = (Ta, Ua)
 // that holds the lowest request of S.  For T != 0 that request is in T, so
