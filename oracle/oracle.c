@@ -18,7 +18,7 @@
  *       F(S)   = min over S = A (+) B of F(A) + F(B) - w(I(S)).
  *     OPT_free = F([m]) (Thm 1, eq. 3).
  *
- * Readings where the paper is silent (each also listed in the design doc):
+ * Readings where the paper is silent:
  *   - the base case M({i}) = 0, i.e. F({i}) = w(R_i);
  *   - I(empty set) is the set of chunks used by at least one request, so
  *     wI[0] = w(R_1 u ... u R_m); the recurrence never reads it;
