@@ -296,7 +296,7 @@ def run_ours(args):
     local_ms = e0.elapsed_time(e1)
     max_ms = max_over_ranks(local_ms, world, device)
     value = world * splits * args.steps / (max_ms / 1000.0)
-    dp_mode = {1: "blocked", 2: "general"}.get(p["dp_mode"], "?")
+    dp_mode = {1: "blocked", 2: "general", 3: "wide"}.get(p["dp_mode"], "?")
 
     # ---- end to end through the C ABI with host buffers ----
     h2d = int(inst.weights.nbytes + inst.bits.nbytes)
@@ -324,7 +324,7 @@ def run_ours(args):
 
     # roofline of the dominant kernel (the pair kernel of the blocked DP)
     peaks = measured_peaks()
-    if dp_mode == "blocked" and prof_sum["ms_dp_pairs"] > 0:
+    if dp_mode in ("blocked", "wide") and prof_sum["ms_dp_pairs"] > 0:
         launches = max(1, prof_sum["launches_pairs"])
         avg_ms = prof_sum["ms_dp_pairs"] / launches
         ops_per_launch = OPS_PER_SPLIT * prof_sum["splits_pairs"] / launches
@@ -336,12 +336,14 @@ def run_ours(args):
         sms = torch.cuda.get_device_properties(device).multi_processor_count
         max_mhz = (clock_info or {}).get("sm_max_mhz") or 2070.0
         alu_peak = sms * 64 * max_mhz * 1e6 / 1e12
-        roofline = {"bound": "alu", "kernel": "k_dp_pairs", "achieved": achieved, "peak": alu_peak,
-                    "unit": "Tops/s", "frac": achieved / alu_peak,
-                    "traffic": (tr or {}).get("dram_bytes_per_launch"),
+        wide = dp_mode == "wide"
+        roofline = {"bound": "alu", "kernel": "k_dp_pairs_w" if wide else "k_dp_pairs", "achieved": achieved,
+                    "peak": alu_peak, "unit": "Tops/s", "frac": achieved / alu_peak,
+                    "traffic": None if wide else (tr or {}).get("dram_bytes_per_launch"),
                     "ops_per_split": OPS_PER_SPLIT,
                     "peak_basis": f"{sms} SMs x 64 integer-ALU-pipe lanes x {max_mhz / 1000:.3f} GHz "
-                                  "(one add-min per split)",
+                                  "(one add-min per split" + ("; 64-bit keys take several ALU instructions "
+                                                              "per split" if wide else "") + ")",
                     "share_of_step": prof_sum["ms_dp_pairs"] / (local_ms if local_ms > 0 else 1)}
     else:
         hbm = float(peaks.get("hbm_gbs", 6800.0))
@@ -377,7 +379,7 @@ def run_ours(args):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "u32" if dp_mode == "blocked" else "int64",
+        "dtype": {"blocked": "u32", "wide": "u64"}.get(dp_mode, "int64"),
         "data": "synthetic",
         "solve_time_s": solve_s,
         "config": {"workload": instances.CONFIG_NAMES[args.workload], "m": m, "n": inst.n,
@@ -597,7 +599,7 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--dp-mode", choices=["auto", "blocked", "general"], default="auto")
+    ap.add_argument("--dp-mode", choices=["auto", "blocked", "general", "wide"], default="auto")
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")

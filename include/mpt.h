@@ -53,11 +53,14 @@ typedef enum mpt_status {
 typedef struct mpt_ctx mpt_ctx;
 
 /* DP kernels mpt_solve may use.  AUTO picks BLOCKED whenever
- * sum_i w(R_i) < 2^20 (its 32-bit packed keys are then exact), else GENERAL. */
+ * sum_i w(R_i) < 2^20 (its 32-bit packed keys are then exact), else WIDE
+ * while sum_i w(R_i) < 2^51 (64-bit packed keys), else GENERAL.  All three
+ * return the same tables, OPT and layout. */
 typedef enum mpt_dp_mode {
   MPT_DP_AUTO = 0,
   MPT_DP_BLOCKED = 1, /* shared-memory tiled min-plus; needs sum_i w(R_i) < 2^20 */
-  MPT_DP_GENERAL = 2  /* one subset per thread or warp, int64 gathers from HBM/L2 */
+  MPT_DP_GENERAL = 2, /* one subset per thread or warp, int64 gathers from HBM/L2 */
+  MPT_DP_WIDE = 3     /* the tiled min-plus with 64-bit keys; needs sum_i w(R_i) < 2^51 */
 } mpt_dp_mode;
 
 /* Create a context for one instance (Sec. 2).
@@ -75,7 +78,7 @@ mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* 
 mpt_status mpt_workspace_bytes(const mpt_ctx* ctx, size_t* bytes);
 
 /* Choose the DP kernels (default MPT_DP_AUTO).  BLOCKED is refused with
- * OVERFLOW when sum_i w(R_i) >= 2^20. */
+ * OVERFLOW when sum_i w(R_i) >= 2^20, WIDE when sum_i w(R_i) >= 2^51. */
 mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode);
 
 /* Solve exactly (Sec. 3.1): scatter chunk weights by request set, superset
@@ -198,7 +201,7 @@ typedef struct mpt_profile {
   double splits_total;  /* (3^m + 1)/2 - 2^m */
   int64_t launches_pairs;
   int64_t launches_total; /* kernels launched by the last solve (memsets excluded) */
-  int32_t dp_mode;        /* MPT_DP_BLOCKED or MPT_DP_GENERAL as used */
+  int32_t dp_mode;        /* MPT_DP_BLOCKED, MPT_DP_WIDE or MPT_DP_GENERAL as used */
   int32_t tile_bits;      /* request bits per shared-memory tile (blocked mode) */
 } mpt_profile;
 

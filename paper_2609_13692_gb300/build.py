@@ -14,7 +14,7 @@ CSRC = PKG / "csrc"
 BUILD = PKG / "_build"
 LIB = BUILD / "libmpt.so"
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["k_scatter_zeta.cu", "k_dp_general.cu", "k_dp_blocked.cu", "k_walk.cu", "mpt_api.cu", "mpt_noalloc.cu", "k_batch.cu", "mpt_batch.cu", "k_greedy.cu", "k_sched.cu", "k_probe.cu", "k_tables.cu"]
+SOURCES = ["k_scatter_zeta.cu", "k_dp_general.cu", "k_dp_blocked.cu", "k_walk.cu", "mpt_api.cu", "mpt_noalloc.cu", "k_batch.cu", "mpt_batch.cu", "k_greedy.cu", "k_sched.cu", "k_probe.cu", "k_tables.cu", "k_dp_wide.cu"]
 
 
 def nvcc() -> str:

@@ -634,17 +634,21 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
   }
 }
 
+}  // namespace
+
+constexpr unsigned long long kItemOverheadPairs = 2;
+
 // Items (blocks) per tile of one pair-kernel layer.  One block runs per SM,
 // every block of a layer takes about the same time per pair, and a block costs
 // about kItemOverheadPairs pairs more (its first window copy and its final
 // merge).  The layer then takes ceil(blocks / SMs) waves of (pairs per item +
 // overhead); take the item count that minimises that, fewer blocks on ties.
-// Items keep at least kMinPairsPerItem pairs.
-constexpr unsigned long long kItemOverheadPairs = 2;
-
-void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long long* items_out, uint32_t* ppi_out) {
+// Items keep at least kMinPairsPerItem pairs; at most max_items per tile.
+void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long long max_items,
+                  unsigned long long* items_out, uint32_t* ppi_out) {
   const unsigned long long waves_of = sms > 0 ? (unsigned long long)sms : 1ull;
   unsigned long long cap = (P + kMinPairsPerItem - 1) / kMinPairsPerItem;
+  if (cap > max_items) cap = max_items;
   if (cap < 1) cap = 1;
   if (cap > 8192) cap = 8192;
   unsigned long long best_t = ~0ull, best_items = 1;
@@ -664,8 +668,6 @@ void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long l
   *items_out = best_items;
   *ppi_out = best_ppi;
 }
-
-}  // namespace
 
 int blocked_tile_bits(int m) { return m < kB ? m : kB; }
 
@@ -706,7 +708,7 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
       const uint32_t P = (1u << (kh - 1)) - 1u;
       unsigned long long items = 1;
       uint32_t ppi = P;
-      choose_items(tiles, P, sms, &items, &ppi);
+      choose_items(tiles, P, sms, ~0ull, &items, &ppi);
       cudaError_t e = cudaMemsetAsync(ws.partial, 0xFF, (size_t)(tiles << b) * sizeof(unsigned long long), stream);
       if (e != cudaSuccess) return e;
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches], stream);

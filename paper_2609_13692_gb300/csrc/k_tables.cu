@@ -21,6 +21,9 @@ struct Copy {
 struct GpToF {
   __device__ static uint32_t apply(uint32_t v, int b) { return v >> b; }
 };
+struct Gp64ToF {
+  __device__ static unsigned long long apply(unsigned long long v, int b) { return v >> b; }
+};
 
 // dst[(U << L) | T] = Op(src[(T << b) | U]) for T < 2^L, U < 2^b.
 template <typename Src, typename Dst, typename Op>
@@ -61,6 +64,20 @@ cudaError_t unrotate_tables(const Shape& s, const uint32_t* split_rot, uint32_t*
   if (wI_nat && (e = unrotate<int64_t, int64_t, Copy>(wI_rot, wI_nat, s.L, s.b, stream)) != cudaSuccess) return e;
   if (F_nat && (e = unrotate<uint32_t, int64_t, GpToF>(Gp, F_nat, s.L, s.b, stream)) != cudaSuccess) return e;
   if (F32_nat && (e = unrotate<uint32_t, int32_t, GpToF>(Gp, F32_nat, s.L, s.b, stream)) != cudaSuccess) return e;
+  return cudaSuccess;
+}
+
+cudaError_t unrotate_tables_wide(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat,
+                                 const int64_t* wI_rot, int64_t* wI_nat, const unsigned long long* Gp64,
+                                 int64_t* F_nat, int32_t* F32_nat, cudaStream_t stream) {
+  cudaError_t e = cudaSuccess;
+  if (split_nat && (e = unrotate<uint32_t, uint32_t, Copy>(split_rot, split_nat, s.L, s.b, stream)) != cudaSuccess)
+    return e;
+  if (wI_nat && (e = unrotate<int64_t, int64_t, Copy>(wI_rot, wI_nat, s.L, s.b, stream)) != cudaSuccess) return e;
+  if (F_nat && (e = unrotate<unsigned long long, int64_t, Gp64ToF>(Gp64, F_nat, s.L, s.b, stream)) != cudaSuccess)
+    return e;
+  if (F32_nat && (e = unrotate<unsigned long long, int32_t, Gp64ToF>(Gp64, F32_nat, s.L, s.b, stream)) != cudaSuccess)
+    return e;
   return cudaSuccess;
 }
 

@@ -9,7 +9,8 @@
 // (depth of that node, chunk id).  The left-to-right leaf order is the trie
 // DFS order that Thm 7 (Sec. 8) serves requests in.  After a blocked solve
 // split is read at the rotated position of each node and OPT = F(full) from
-// Gp = F << b; after a general one both are in natural order.
+// Gp = F << b (uint32, or uint64 on the wide path); after a general one both
+// are in natural order.
 //
 // Trie cost: a string's node at depth p is new exactly when no earlier
 // string shares its first p+1 symbols, so the trie weight is
@@ -24,7 +25,8 @@ constexpr int kMaxM = 32;
 
 __global__ void __launch_bounds__(kWalkThreads)
 k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F, const int32_t* __restrict__ F32,
-       const uint32_t* __restrict__ Gp, int L, int b, const uint32_t* __restrict__ used_N,
+       const uint32_t* __restrict__ Gp, const unsigned long long* __restrict__ Gp64, int L, int b,
+       const uint32_t* __restrict__ used_N,
        const int32_t* __restrict__ used_x, int32_t* __restrict__ counters, int64_t slots,
        unsigned long long* __restrict__ keys, int64_t* __restrict__ perm_offsets, int64_t* __restrict__ perm_chunks,
        int32_t* __restrict__ dfs, int64_t* __restrict__ opt) {
@@ -62,7 +64,7 @@ k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F,
         continue;
       }
       // blocked path: split and F (as F << b in Gp) in rotated order
-      const uint32_t A = Gp ? split[rot_index(S, L, b)] : split[S];
+      const uint32_t A = (Gp || Gp64) ? split[rot_index(S, L, b)] : split[S];
       if (A == 0 || (A & ~S) != 0 || A == S || sp + 2 > 2 * kMaxM) {
         bad = 1;
         break;
@@ -75,7 +77,9 @@ k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F,
       ++sp;
     }
     if (bad) atomicOr(&counters[1], kErrBadSplit);
-    *opt = Gp ? (int64_t)(Gp[rot_index(full, L, b)] >> b) : (F ? F[full] : (int64_t)F32[full]);
+    *opt = Gp64 ? (int64_t)(Gp64[rot_index(full, L, b)] >> b)
+           : Gp ? (int64_t)(Gp[rot_index(full, L, b)] >> b)
+                : (F ? F[full] : (int64_t)F32[full]);
   }
   __syncthreads();
   if (bad) return;
@@ -156,7 +160,8 @@ k_trie_cost(int m, const int64_t* __restrict__ w, const int64_t* __restrict__ of
 
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
   k_walk<<<1, kWalkThreads, 0, stream>>>(s.m, s.blocked ? ws.split_rot : ws.split, s.lean ? nullptr : ws.F,
-                                         s.lean ? ws.fw : nullptr, s.blocked ? ws.Gp : nullptr, s.L, s.b, ws.used_N,
+                                         s.lean ? ws.fw : nullptr, s.blocked && !s.wide ? ws.Gp : nullptr,
+                                         s.blocked && s.wide ? ws.Gp64 : nullptr, s.L, s.b, ws.used_N,
                                          ws.used_x, ws.counters, s.slots, ws.keys,
                                          ws.perm_offsets, ws.perm_chunks, ws.dfs, ws.opt);
   ++*launches;

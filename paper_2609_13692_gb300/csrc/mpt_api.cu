@@ -47,23 +47,36 @@ namespace {
 constexpr int kMaxRequests = 32;
 constexpr int64_t kSumLimit = (int64_t)1 << 62;
 
+constexpr int64_t kWideLimit = (int64_t)1 << 51;  // 64-bit keys: F(A) + F(B) < 2^52
+
 bool blocked_feasible(const mpt_ctx* c) {
   const int b = mpt::blocked_tile_bits(c->shape.m);
   return c->sum_w < ((int64_t)1 << (32 - b));
 }
 
+bool wide_feasible(const mpt_ctx* c) { return c->sum_w < kWideLimit; }
+
 bool use_blocked(const mpt_ctx* c) {
   if (c->mode == MPT_DP_GENERAL) return false;
-  return blocked_feasible(c);
+  if (c->mode == MPT_DP_BLOCKED) return blocked_feasible(c);
+  return wide_feasible(c);  // AUTO and WIDE: the 32- or the 64-bit keys
+}
+
+bool use_wide(const mpt_ctx* c) {
+  if (c->mode == MPT_DP_WIDE) return wide_feasible(c);
+  return c->mode == MPT_DP_AUTO && !blocked_feasible(c) && wide_feasible(c);
 }
 
 void refresh_shape(mpt_ctx* c) {
   mpt::Shape& s = c->shape;
   s.blocked = use_blocked(c);
+  s.wide = s.blocked && use_wide(c);
   s.lean = c->tables == MPT_TABLES_LEAN;
   s.b = mpt::blocked_tile_bits(s.m);
   s.L = s.m - s.b;
-  s.partial_entries = s.blocked ? mpt::blocked_partial_entries(s.m, s.b) : 0;
+  s.partial_entries = !s.blocked ? 0
+                      : s.wide   ? (mpt::wide_partial_slots(s.m, s.b) << s.b)
+                                 : mpt::blocked_partial_entries(s.m, s.b);
 }
 
 mpt_status cuda_fail(mpt_ctx* c, cudaError_t e, const char* what) {
@@ -106,14 +119,26 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws) {
     ws->fw = nullptr;
   }
   ws->split = reinterpret_cast<uint32_t*>(take(N * 4));
-  if (s.blocked) {
+  ws->Gp64 = ws->Gc64 = nullptr;
+  ws->partial_ta = nullptr;
+  if (s.blocked && s.wide) {
+    ws->Gp64 = reinterpret_cast<unsigned long long*>(take(N * 8));
+    ws->Gc64 = reinterpret_cast<unsigned long long*>(take(N * 8));
+    ws->Gp = ws->Gc = nullptr;
+    const size_t pe = (size_t)(s.partial_entries > 0 ? s.partial_entries : 1);
+    ws->partial = reinterpret_cast<unsigned long long*>(take(pe * 8));
+    ws->partial_ta = reinterpret_cast<uint32_t*>(take(pe * 4));
+  } else if (s.blocked) {
     ws->Gp = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->Gc = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->partial = reinterpret_cast<unsigned long long*>(take((size_t)(s.partial_entries > 0 ? s.partial_entries : 1) * 8));
+  }
+  if (s.blocked) {
     // The rotated tables share the buffers of the natural ones: w(I) sits in
     // the F table (int64) or in fw (lean), split in the split table.  The
     // natural views, when asked for, go to wI, F or fw (F from Gp) and, for
-    // split, to the Gc table, which the recurrence no longer needs.
+    // split, to the Gc table (32- or 64-bit), which the recurrence no longer
+    // needs.
     ws->wI_rot = s.lean ? nullptr : ws->F;
     ws->fw_rot = s.lean ? ws->fw : nullptr;
     ws->split_rot = ws->split;
@@ -202,8 +227,9 @@ mpt_status mpt_workspace_bytes(const mpt_ctx* ctx, size_t* bytes) {
 }
 
 mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode) {
-  if (!ctx || mode < MPT_DP_AUTO || mode > MPT_DP_GENERAL) return MPT_ERR_INVALID_ARG;
+  if (!ctx || mode < MPT_DP_AUTO || mode > MPT_DP_WIDE) return MPT_ERR_INVALID_ARG;
   if (mode == MPT_DP_BLOCKED && !blocked_feasible(ctx)) return MPT_ERR_OVERFLOW;
+  if (mode == MPT_DP_WIDE && !wide_feasible(ctx)) return MPT_ERR_OVERFLOW;
   ctx->mode = mode;
   refresh_shape(ctx);
   ctx->solved = false;
@@ -296,7 +322,9 @@ mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStrea
 mpt_status run_steps(mpt_ctx* c, const mpt::Workspace& ws, cudaStream_t stream, int* launches,
                      mpt::BlockedTiming* timing, int begin, int end) {
   const mpt::Shape& s = c->shape;
-  if (s.blocked) {
+  if (s.blocked && s.wide) {
+    MPT_CK(mpt::launch_dp_wide(s, ws, stream, launches, timing, begin, end), "wide blocked DP kernels");
+  } else if (s.blocked) {
     MPT_CK(mpt::launch_dp_blocked(s, ws, stream, launches, timing, begin, end), "blocked DP kernels");
   } else {
     MPT_CK(mpt::launch_dp_general(s, ws, stream, launches, begin, end), "general DP kernels");
@@ -390,7 +418,7 @@ mpt_status mpt_solve(mpt_ctx* ctx, void* d_workspace, size_t workspace_bytes, vo
   mpt_profile& p = c->prof;
   std::memset(&p, 0, sizeof(p));
   p.launches_total = launches;
-  p.dp_mode = s.blocked ? MPT_DP_BLOCKED : MPT_DP_GENERAL;
+  p.dp_mode = !s.blocked ? MPT_DP_GENERAL : (s.wide ? MPT_DP_WIDE : MPT_DP_BLOCKED);
   p.tile_bits = s.blocked ? s.b : 0;
   {
     // (3^m + 1)/2 - 2^m, exactly representable in a double for m <= 32
@@ -527,7 +555,11 @@ mpt_status ensure_natural(mpt_ctx* c) {
     e = cudaStreamCreateWithFlags(&c->conv_stream, cudaStreamNonBlocking);
     c->conv_device = c->device;
   }
-  if (e == cudaSuccess)
+  if (e == cudaSuccess && s.wide)
+    e = mpt::unrotate_tables_wide(s, ws.split_rot, reinterpret_cast<uint32_t*>(ws.Gc64), ws.wI_rot,
+                                  s.lean ? nullptr : ws.wI, ws.Gp64, s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr,
+                                  c->conv_stream);
+  else if (e == cudaSuccess)
     e = mpt::unrotate_tables(s, ws.split_rot, ws.Gc, ws.wI_rot, s.lean ? nullptr : ws.wI, ws.Gp,
                              s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr, c->conv_stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->conv_stream);
@@ -539,7 +571,10 @@ mpt_status ensure_natural(mpt_ctx* c) {
 
 // Natural split view: the split table (general path) or the Gc table that the
 // conversion wrote it to (blocked path).
-const uint32_t* natural_split(const mpt_ctx* c) { return c->shape.blocked ? c->ws.Gc : c->ws.split; }
+const uint32_t* natural_split(const mpt_ctx* c) {
+  if (!c->shape.blocked) return c->ws.split;
+  return c->shape.wide ? reinterpret_cast<const uint32_t*>(c->ws.Gc64) : c->ws.Gc;
+}
 
 }  // namespace
 

@@ -103,6 +103,11 @@ struct Workspace {
   uint32_t* Gp;       // [2^m]  F << b
   uint32_t* Gc;       // [2^m]  (F << b) | (~u & (2^b - 1))
   unsigned long long* partial;  // [max tiles of one layer << b]
+  // wide blocked path (64-bit keys): Gp and Gc hold uint64 entries, and the
+  // pair kernel leaves one (key, Ta) slot of 2^b entries per block
+  unsigned long long* Gp64;     // [2^m] or nullptr
+  unsigned long long* Gc64;     // [2^m] or nullptr
+  uint32_t* partial_ta;         // [partial_entries] (wide) or nullptr
   int64_t* wI_rot;    // [2^m] w(I(S)) at idx(S) (int64 tables), or nullptr
   int32_t* fw_rot;    // [2^m] w(I(S)) at idx(S) (lean tables), or nullptr
   uint32_t* split_rot;  // [2^m] split[S] at idx(S)
@@ -120,6 +125,7 @@ struct Shape {
   int64_t words;
   int64_t slots;    // sum_i |R_i|
   bool blocked;     // blocked DP tables present
+  bool wide;        // blocked path with 64-bit keys (sum_i w(R_i) >= 2^(32-b))
   bool lean;        // one int32 table for w(I(S)) then F(S)
   int b;            // tile bits (blocked)
   int L;            // m - b
@@ -167,6 +173,17 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
 int64_t blocked_partial_entries(int m, int b);
 int blocked_tile_bits(int m);
 
+// Pair ranges per tile for one pair-kernel layer (whole waves of one block
+// per SM; see k_dp_blocked.cu); at most max_items.
+void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long long max_items,
+                  unsigned long long* items, uint32_t* ppi);
+
+// Wide blocked path (k_dp_wide.cu): 64-bit keys, valid when
+// sum_i w(R_i) < 2^51.  Partial slots: blocks of one pair layer, at most.
+int64_t wide_partial_slots(int m, int b);
+cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
+                           BlockedTiming* timing, int step_begin = 0, int step_end = -1);
+
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
 
 // Natural-order tables from the blocked path's rotated ones (k_tables.cu):
@@ -177,6 +194,10 @@ cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream
 cudaError_t unrotate_tables(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat, const int64_t* wI_rot,
                             int64_t* wI_nat, const uint32_t* Gp, int64_t* F_nat, int32_t* F32_nat,
                             cudaStream_t stream);
+// The same for the wide path (F from the uint64 Gp table).
+cudaError_t unrotate_tables_wide(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat,
+                                 const int64_t* wI_rot, int64_t* wI_nat, const unsigned long long* Gp64,
+                                 int64_t* F_nat, int32_t* F32_nat, cudaStream_t stream);
 // eq. (1) for any number of strings by lexicographic sorting (k_sched.cu)
 mpt_status trie_cost_lex(const int64_t* weights, int64_t n_chunks, int64_t m, const int64_t* offsets,
                          const int64_t* chunks, cudaStream_t st, int64_t* cost);

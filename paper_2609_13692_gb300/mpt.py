@@ -21,8 +21,8 @@ import numpy as np
 from . import build as _build
 
 MPT_OK = 0
-MPT_DP_AUTO, MPT_DP_BLOCKED, MPT_DP_GENERAL = 0, 1, 2
-_MODES = {"auto": MPT_DP_AUTO, "blocked": MPT_DP_BLOCKED, "general": MPT_DP_GENERAL}
+MPT_DP_AUTO, MPT_DP_BLOCKED, MPT_DP_GENERAL, MPT_DP_WIDE = 0, 1, 2, 3
+_MODES = {"auto": MPT_DP_AUTO, "blocked": MPT_DP_BLOCKED, "general": MPT_DP_GENERAL, "wide": MPT_DP_WIDE}
 
 STATUS_NAMES = {
     0: "MPT_OK",

@@ -87,8 +87,26 @@ def test_workspace_and_modes(mpt):
     with pytest.raises(mpt.MPTError) as e:
         mpt.mpt_set_dp_mode(ctx2, "blocked")
     assert e.value.status == 3
+    # AUTO takes the 64-bit-key tiles there: uint64 working tables and per-block slots
+    heavy_auto = mpt.mpt_workspace_bytes(ctx2)
+    assert heavy_auto >= N * (8 + 8 + 4 + 8 + 8)
+    mpt.mpt_set_dp_mode(ctx2, "wide")
+    assert mpt.mpt_workspace_bytes(ctx2) == heavy_auto
+    mpt.mpt_set_dp_mode(ctx, "wide")  # allowed for light weights too
+    assert mpt.mpt_workspace_bytes(ctx) == heavy_auto
+    huge = I.Instance(np.full(20, 1 << 47, dtype=np.int64), inst.bits)  # sum_i w(R_i) >= 2^51
+    ctx3 = mpt.mpt_create(huge.weights, huge.bits)
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_set_dp_mode(ctx3, "wide")
+    assert e.value.status == 3
+    mpt.mpt_set_dp_mode(ctx3, "auto")
+    assert N * 20 <= mpt.mpt_workspace_bytes(ctx3) < auto  # the general kernels
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_set_dp_mode(ctx3, 4)
+    assert e.value.status == 1
     mpt.mpt_destroy(ctx)
     mpt.mpt_destroy(ctx2)
+    mpt.mpt_destroy(ctx3)
 
 
 def test_status_strings(mpt):

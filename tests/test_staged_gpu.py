@@ -25,17 +25,26 @@ def mpt():
 
 
 def _cases():
-    big = I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000)  # general kernels
+    big = I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000)  # sum_i w(R_i) > 2^20
     return [
-        ("blocked m=20", I.rag_pools(20, 5000, 6, 40, 8, 1.1, seed=3)),
-        ("blocked m=12 (one step)", I.config(1)),
-        ("blocked m=17", I.random_instance(17, 80, (2, 9), seed=9, wmin=1, wmax=60)),
-        ("general m=14", big),
+        ("blocked m=20", I.rag_pools(20, 5000, 6, 40, 8, 1.1, seed=3), "auto"),
+        ("blocked m=12 (one step)", I.config(1), "auto"),
+        ("blocked m=17", I.random_instance(17, 80, (2, 9), seed=9, wmin=1, wmax=60), "auto"),
+        ("general m=14", big, "general"),
+        ("wide m=14 (64-bit keys chosen by AUTO)", big, "auto"),
+        ("wide m=17", I.random_instance(17, 80, (2, 9), seed=9, wmin=1, wmax=60), "wide"),
     ]
 
 
-def _one_shot(mpt, inst):
+def _ctx(mpt, inst, mode):
     ctx = mpt.mpt_create(inst.weights, inst.bits)
+    if mode != "auto":
+        mpt.mpt_set_dp_mode(ctx, mode)
+    return ctx
+
+
+def _one_shot(mpt, inst, mode="auto"):
+    ctx = _ctx(mpt, inst, mode)
     opt = mpt.mpt_solve(ctx)
     F, wI, split = (t.clone() for t in mpt.mpt_tables(ctx))
     lay = mpt.mpt_layout(ctx)
@@ -46,13 +55,13 @@ def _same_layout(a, b):
     return all(np.array_equal(np.asarray(x), np.asarray(y)) for x, y in zip(a, b))
 
 
-@pytest.mark.parametrize("idx", range(4))
+@pytest.mark.parametrize("idx", range(6))
 def test_staged_with_checkpoint_every_step(mpt, idx):
     import torch
 
-    name, inst = _cases()[idx]
-    opt, F, wI, split, lay = _one_shot(mpt, inst)
-    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    name, inst, mode = _cases()[idx]
+    opt, F, wI, split, lay = _one_shot(mpt, inst, mode)
+    ctx = _ctx(mpt, inst, mode)
     steps = mpt.mpt_solve_steps(ctx)
     ws = torch.empty(mpt.mpt_workspace_bytes(ctx), dtype=torch.uint8, device="cuda")
     mpt.mpt_solve_begin(ctx, ws)
@@ -73,7 +82,7 @@ def test_staged_with_checkpoint_every_step(mpt, idx):
 def test_resume_in_fresh_context(mpt):
     import torch
 
-    name, inst = _cases()[0]
+    name, inst, _ = _cases()[0]
     opt, F, wI, split, lay = _one_shot(mpt, inst)
     ctx = mpt.mpt_create(inst.weights, inst.bits)
     steps = mpt.mpt_solve_steps(ctx)
