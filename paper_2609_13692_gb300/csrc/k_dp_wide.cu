@@ -14,9 +14,9 @@
 // convolution (81 add-min steps) of row a1 of X with row s1 ^ a1 of Y into
 // the 16 outputs of row s1.  The 3^8 = 6561 units of a window pair come in
 // 1645 chunks (the units of one row with fixed low bits: 4, or 1-2 for the
-// rows with fewer than 2 bits).  Thread t takes 7 consecutive chunks
-// (t < 109) or 6, so warps 0..3 run 7 chunk-times and warps 4..7 six: each
-// sub-partition issues 13 chunk-times per pair for 12.85 of work.  A thread
+// rows with fewer than 2 bits), cut into 256 ranges of 7 or 6 consecutive
+// chunks; warps 0..3 run the 7-chunk ranges and warps 4..7 the others, so
+// each sub-partition issues 13 chunk-times per pair for 12.85 of work.  A thread
 // keeps one row's 16 minima in registers while its chunks stay in that row,
 // and merges them into a per-pair shared array (64-bit atomicMin) when the
 // row changes.  Owners fold the array into running (key, Ta) bests after
@@ -74,8 +74,9 @@ constexpr uint32_t deposit8(uint32_t q, uint32_t mask) {
 
 struct WidePlan {
   uint32_t chunk[kWChunks];          // s1 | fixed << 8 | free << 16
-  uint16_t start[kWThreads + 1];     // thread t runs chunks [start[t], start[t + 1])
-  int nchunk;
+  uint16_t first[kWThreads];         // thread t runs chunks first[t] .. first[t] + count[t] - 1
+  uint16_t count[kWThreads];
+  int nchunk, total;
 };
 
 // Chunks in increasing row order.  Rows with >= 2 bits: the two highest bits
@@ -105,17 +106,29 @@ constexpr WidePlan make_wide_plan() {
     for (uint32_t v = 0; v < (1u << (p - 2)); ++v) pl.chunk[n++] = s1 | (deposit8(v, lowm) << 8) | (top << 16);
   }
   pl.nchunk = n;
+  // Ranges r = 0..255 of consecutive chunks, 7 for r < 109 and 6 after.  Lane
+  // l of warp w runs range 4 l + w (warps 0..3) or 128 + 4 l + (w - 4): the
+  // 7-chunk ranges stay on warps 0..3, and neighbouring lanes work 4 ranges
+  // (about 26 chunks) apart, mostly in different rows, so their flushes do
+  // not hit the same words.
+  int firsts[kWThreads] = {};
   int c = 0;
-  for (int t = 0; t < kWThreads; ++t) {
-    pl.start[t] = (uint16_t)c;
-    c += t < kWLong ? 7 : 6;
+  for (int r = 0; r < kWThreads; ++r) {
+    firsts[r] = c;
+    c += r < kWLong ? 7 : 6;
   }
-  pl.start[kWThreads] = (uint16_t)c;
+  pl.total = c;
+  for (int t = 0; t < kWThreads; ++t) {
+    const int w = t / 32, l = t % 32;
+    const int r = w < 4 ? 4 * l + w : 128 + 4 * l + (w - 4);
+    pl.first[t] = (uint16_t)firsts[r];
+    pl.count[t] = (uint16_t)(r < kWLong ? 7 : 6);
+  }
   return pl;
 }
 
 constexpr WidePlan kWidePlanHost = make_wide_plan();
-static_assert(kWidePlanHost.nchunk == kWChunks && kWidePlanHost.start[kWThreads] == kWChunks, "chunk plan");
+static_assert(kWidePlanHost.nchunk == kWChunks && kWidePlanHost.total == kWChunks, "chunk plan");
 static __constant__ WidePlan c_wplan = make_wide_plan();
 
 // Row placement: the low 3 row bits XOR-ed with higher ones; linear over GF(2).
@@ -182,7 +195,13 @@ k_dp_pairs_w(const u64* __restrict__ Gp, const u64* __restrict__ Gc, u64* __rest
   const uint32_t R = T ^ low;
   const uint32_t q0 = item * pairs_per_item;
   const uint32_t q1 = min(q0 + pairs_per_item, pairs_per_tile);
-  const uint32_t c0 = c_wplan.start[threadIdx.x], c1 = c_wplan.start[threadIdx.x + 1];
+  // this thread's chunks, read from constant memory once (lanes read
+  // different entries, which the constant cache serves one at a time)
+  const uint32_t c0 = c_wplan.first[threadIdx.x];
+  const int nch = (int)c_wplan.count[threadIdx.x];
+  uint32_t chunks[7];
+#pragma unroll
+  for (int i = 0; i < 7; ++i) chunks[i] = i < nch ? c_wplan.chunk[c0 + i] : 0u;
 
   for (int i = threadIdx.x; i < 2 * (1 << kWB); i += kWThreads) pmin[i] = ~0ull;
   u64 bk[kWOwned];
@@ -221,8 +240,10 @@ k_dp_pairs_w(const u64* __restrict__ Gp, const u64* __restrict__ Gc, u64* __rest
       u64 acc[kWRow];
 #pragma unroll
       for (int i = 0; i < kWRow; ++i) acc[i] = ~0ull;
-      for (uint32_t c = c0; c < c1; ++c) {
-        const uint32_t ch = c_wplan.chunk[c];
+#pragma unroll
+      for (int c = 0; c < 7; ++c) {
+        if (c >= nch) break;
+        const uint32_t ch = chunks[c];
         const uint32_t s1 = ch & 0xFFu, fixed = (ch >> 8) & 0xFFu, freem = (ch >> 16) & 0xFFu;
         if (s1 != row) {
           if (row != 0xFFFFFFFFu) {
@@ -237,6 +258,7 @@ k_dp_pairs_w(const u64* __restrict__ Gp, const u64* __restrict__ Gc, u64* __rest
         const uint32_t b0 = freem & (~freem + 1u), b1 = freem ^ b0;
         const int nunits = freem == 0 ? 1 : (b1 == 0 ? 2 : 4);
         uint32_t pa = row_pos_w(fixed);
+#pragma unroll 1
         for (int k = 0; k < nunits; ++k) {
           // Gray order over the free bits: fixed, ^b0, ^b1, ^b0
           if (k > 0) pa ^= row_pos_w((k & 1) ? b0 : b1);
