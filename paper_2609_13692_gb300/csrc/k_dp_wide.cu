@@ -131,6 +131,36 @@ constexpr WidePlan kWidePlanHost = make_wide_plan();
 static_assert(kWidePlanHost.nchunk == kWChunks && kWidePlanHost.total == kWChunks, "chunk plan");
 static __constant__ WidePlan c_wplan = make_wide_plan();
 
+// The 4096 subsets of 12 inner bits sorted by size, then colex rank: the order
+// in which the tile kernel finishes them.  The same for every tile, so it is
+// a static table (global memory, read with coalesced loads) rather than being
+// recomputed per block from the binomial table, whose per-thread indices the
+// constant cache would serve one by one.
+struct OrderTable {
+  uint16_t v[1 << kWB];
+};
+
+constexpr OrderTable make_order12() {
+  OrderTable t{};
+  uint32_t start[kWB + 2] = {};
+  for (int p = 0; p <= kWB; ++p) start[p + 1] = start[p] + (uint32_t)h_binom.v[kWB][p];
+  for (uint32_t u = 0; u < (1u << kWB); ++u) {
+    uint32_t r = 0, s = u;
+    int k = 1;
+    while (s) {
+      int pos = 0;
+      while (!((s >> pos) & 1u)) ++pos;
+      r += (uint32_t)h_binom.v[pos][k];
+      ++k;
+      s &= s - 1;
+    }
+    t.v[start[popc8(u)] + r] = (uint16_t)u;
+  }
+  return t;
+}
+
+static __device__ const OrderTable g_order12 = make_order12();
+
 // Row placement: the low 3 row bits XOR-ed with higher ones; linear over GF(2).
 __device__ __forceinline__ uint32_t row_pos_w(uint32_t r) { return r ^ (((r >> 3) ^ (r >> 6)) & 7u); }
 
@@ -320,10 +350,14 @@ k_dp_tile_w(int L, int b, int kh, const Tab* __restrict__ wIr, const u64* __rest
   const uint32_t mask = (uint32_t)size - 1u;
 
   for (int u = threadIdx.x; u < size; u += kWTileThreads) {
-    const int p = __popc(u);
-    uint32_t start = 0;
-    for (int j = 0; j < p; ++j) start += (uint32_t)c_binom.v[b][j];
-    order[start + colex_rank((uint32_t)u)] = (uint16_t)u;
+    if (b == kWB) {
+      order[u] = g_order12.v[u];
+    } else {  // fewer than 12 requests: tile 0 only, one block
+      const int p = __popc(u);
+      uint32_t start = 0;
+      for (int j = 0; j < p; ++j) start += (uint32_t)c_binom.v[b][j];
+      order[start + colex_rank((uint32_t)u)] = (uint16_t)u;
+    }
     if (kh >= 1) oc[u] = Gc[u];
   }
   __syncthreads();
