@@ -137,3 +137,21 @@ def test_wide_lean_tables(mpt):
     F2, s2 = mpt.mpt_tables32(ctx2)
     assert torch.equal(F1, F2.to(torch.int64)) and torch.equal(s1, s2)
     assert o1 == O.solve(inst.weights, inst.bits)[0]
+
+
+@pytest.mark.parametrize("m", [19, 20, 21, 22])
+def test_wide_equals_narrow_medium(mpt, m):
+    """The 64-bit keys forced on RAG-shaped instances the 32-bit keys also hold:
+    every table equal on the device (layers with several blocks per tile)."""
+    import torch
+
+    inst = I.rag_pools(m, 5000, 6, 40, 8, 1.1, seed=100 + m)
+    narrow = mpt.solve(inst.weights, inst.bits, profile=True)
+    wide = mpt.solve(inst.weights, inst.bits, mode="wide", profile=True)
+    assert mpt.mpt_get_profile(narrow.ctx)["dp_mode"] == 1
+    assert mpt.mpt_get_profile(wide.ctx)["dp_mode"] == 3
+    assert wide.opt == narrow.opt
+    for a, b in zip(mpt.mpt_tables(narrow.ctx), mpt.mpt_tables(wide.ctx)):
+        assert torch.equal(a, b)
+    assert wide.permutations() == narrow.permutations()
+    assert wide.dfs_order.tolist() == narrow.dfs_order.tolist()
