@@ -189,6 +189,8 @@ def mpt_workspace_bytes(ctx: Context) -> int:
 
 
 def mpt_set_dp_mode(ctx: Context, mode: str | int) -> None:
+    """DP kernels: "auto" (default), "blocked" (32-bit keys), "wide" (64-bit
+    keys) or "general"; see ``mpt_set_dp_mode`` in mpt.h."""
     code = _MODES[mode] if isinstance(mode, str) else int(mode)
     _check(load().mpt_set_dp_mode(ctx.handle, code), "mpt_set_dp_mode", ctx)
 
