@@ -239,3 +239,38 @@ def test_lean_tables_host_checks(mpt):
     ctx = mpt.mpt_create(heavy.weights, heavy.bits)
     assert lib.mpt_set_tables(ctx.handle, 1) == 3
     mpt.mpt_destroy(ctx)
+
+
+def test_helper_argument_checks(mpt):
+    """Host-side checks of mpt_trie_cost, mpt_solve_noalloc and
+    mpt_gather_bandwidth, all returned before any CUDA call."""
+    import ctypes
+
+    lib = mpt.load()
+    p64 = lambda a: a.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
+    w = np.array([3, 4, 5], dtype=np.int64)
+    cost = ctypes.c_int64()
+    offs = np.array([0, 2, 3], dtype=np.int64)
+    ch = np.array([0, 1, 2], dtype=np.int64)
+    assert lib.mpt_trie_cost(None, 3, 2, p64(offs), p64(ch), ctypes.byref(cost)) == 1
+    assert lib.mpt_trie_cost(p64(w), 3, 0, p64(offs), p64(ch), ctypes.byref(cost)) == 1
+    bad_first = np.array([1, 2, 3], dtype=np.int64)
+    assert lib.mpt_trie_cost(p64(w), 3, 2, p64(bad_first), p64(ch), ctypes.byref(cost)) == 1
+    decreasing = np.array([0, 2, 1], dtype=np.int64)
+    assert lib.mpt_trie_cost(p64(w), 3, 2, p64(decreasing), p64(ch), ctypes.byref(cost)) == 1
+    out_of_range = np.array([0, 1, 3], dtype=np.int64)
+    assert lib.mpt_trie_cost(p64(w), 3, 2, p64(offs), p64(out_of_range), ctypes.byref(cost)) == 1
+    zero_w = np.array([3, 0, 5], dtype=np.int64)
+    assert lib.mpt_trie_cost(p64(zero_w), 3, 2, p64(offs), p64(ch), ctypes.byref(cost)) == 1
+    # mpt_solve_noalloc: null device pointers, then m beyond its 20-request limit
+    dummy = ctypes.c_void_p(256)
+    args = [dummy, 3, dummy, 21, dummy, dummy, dummy, dummy, None]
+    assert lib.mpt_solve_noalloc(None, *args[1:]) == 1
+    assert lib.mpt_solve_noalloc(*args) == 2
+    assert lib.mpt_solve_noalloc(dummy, 0, dummy, 5, dummy, dummy, dummy, dummy, None) == 1
+    # mpt_gather_bandwidth: table size and load count
+    gbps = ctypes.c_double()
+    assert lib.mpt_gather_bandwidth(9, 1000, None, ctypes.byref(gbps)) == 1
+    assert lib.mpt_gather_bandwidth(33, 1000, None, ctypes.byref(gbps)) == 1
+    assert lib.mpt_gather_bandwidth(20, 0, None, ctypes.byref(gbps)) == 1
+    assert lib.mpt_gather_bandwidth(20, 1000, None, None) == 1
