@@ -414,7 +414,7 @@ __device__ __forceinline__ void bconv_restricted(uint32_t (&acc)[kBRow], const u
 }
 
 template <int TPI>
-__global__ void __launch_bounds__(TPI)
+__global__ void __launch_bounds__(TPI, TPI >= 256 ? 3 : (TPI == 128 ? 6 : 12))  // 12 warps or more per SM
 k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
              const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
              const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list, int occ_cap, int mm,
@@ -432,9 +432,10 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   const uint32_t mask = (uint32_t)N - 1u;
   const int64_t tb = tab_off[inst];
 
+  // Gp(X) = (F(X) << m) + X only: the complement form Gc(X) = Gp(X) - X is
+  // formed from it when a row is loaded
   uint32_t* Gp = reinterpret_cast<uint32_t*>(smem_raw);                          // [R * 36]
-  uint32_t* Gc = Gp + (1 << (mm - 5)) * kBRowStride;                               // [R * 36]
-  uint32_t* bk = Gc + (1 << (mm - 5)) * kBRowStride;                               // [level rows * 33] phase A minima
+  uint32_t* bk = Gp + (1 << (mm - 5)) * kBRowStride;                               // [level rows * 33] phase A minima
   unsigned long long* keys =
       reinterpret_cast<unsigned long long*>(bk + batch_level_rows(mm - 5) * kBkStride);  // [occ_cap]
   int32_t* cx = reinterpret_cast<int32_t*>(keys + occ_cap);                        // [occ_cap]
@@ -506,10 +507,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       split[s2] = (uint16_t)A;
     }
 #pragma unroll
-    for (int s2 = 0; s2 < kBRow; ++s2) {
-      Gp[s2] = zp[s2];
-      Gc[s2] = zc[s2];
-    }
+    for (int s2 = 0; s2 < kBRow; ++s2) Gp[s2] = zp[s2];
   }
   __syncthreads();
 
@@ -541,7 +539,10 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
           if (a1 != 0 && a1 != s1) {
             uint32_t x[kBRow], y[kBRow];
             bload_row(x, Gp + brow_pos(a1) * kBRowStride);
-            bload_row(y, Gc + brow_pos(s1 ^ a1) * kBRowStride);
+            bload_row(y, Gp + brow_pos(s1 ^ a1) * kBRowStride);
+            const uint32_t yb = (s1 ^ a1) << 5;
+#pragma unroll
+            for (int i = 0; i < kBRow; ++i) y[i] -= yb | (uint32_t)i;  // Gc = Gp - X
             bconv_restricted(acc, x, y);
             if (a1 & lowb) acc[0] = min(acc[0], x[0] + y[0]);
           }
@@ -565,9 +566,9 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       uint32_t* prow = Gp + brow_pos(s1) * kBRowStride;
       uint32_t zp[kBRow], zcs[kBRow], cc[kBRow];
       bload_row(zp, Gp);   // row 0 is at position 0
-      bload_row(zcs, Gc);
+      bload_row(zcs, Gp);
 #pragma unroll
-      for (int i = 0; i < kBRow; ++i) zcs[i] += S1;  // Gc(0, x) + (s1 << 5): the A-part of a1 = s1 splits
+      for (int i = 0; i < kBRow; ++i) zcs[i] += S1 - (uint32_t)i;  // Gc(0, x) + (s1 << 5): the A-part of a1 = s1 splits
 #pragma unroll
       for (int blk = 0; blk < kBRow / 8; ++blk) {
         uint32_t wv[8], bkv[8];
@@ -607,7 +608,6 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 #pragma unroll
       for (int i = 0; i < kBRow; ++i) gp[i] = cc[i] + (S1 | (uint32_t)i);
       bstore_row(prow, gp);
-      bstore_row(Gc + brow_pos(s1) * kBRowStride, cc);
     }
     __syncthreads();
   }
@@ -645,7 +645,7 @@ cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, 
 
 size_t batch_rows_smem_bytes(int m, int occ_cap) {
   const size_t R = (size_t)1 << (m - 5);
-  return 2 * R * kBRowStride * 4 + (size_t)batch_level_rows(m - 5) * kBkStride * 4 + (size_t)occ_cap * 16 +
+  return R * kBRowStride * 4 + (size_t)batch_level_rows(m - 5) * kBkStride * 4 + (size_t)occ_cap * 16 +
          (size_t)occ_cap * 8 + ((size_t)2 << m) + 64;
 }
 
