@@ -324,11 +324,12 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 //
 // The 2^m subsets U = (s1, s2) are 2^(m-5) rows s1 of 32 entries s2, stored
 // at row_pos(s1) * 36 + s2 (rows padded to 36 words and XOR-placed so that
-// the 16-byte chunks of different rows fall in different bank groups).  Two
-// tables per row:
-//   Gp(X) = (F(X) << m) + X,   Gc(X) = F(X) << m,
+// the 16-byte chunks of different rows fall in different bank groups).  The
+// keys are
+//   Gp(X) = (F(X) << m) + X,   Gc(X) = F(X) << m = Gp(X) - X,
 // so Gp(A) + Gc(B) = ((F(A) + F(B)) << m) + A: an unsigned min over splits
-// picks the least value and, among equal values, the least A.  Before U is
+// picks the least value and, among equal values, the least A.  Only Gp is
+// stored; a row is turned into its Gc form when it is loaded.  Before U is
 // finished, Gp(U) holds w(I(U)) (superset sums in place).
 // A split of U names the part A holding lowbit(U):
 //   * s2 != 0: A = (a1, a2) with a2 holding lowbit(s2), any a1 within s1;
