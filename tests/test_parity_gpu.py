@@ -276,6 +276,49 @@ def test_m31_extension(mpt):
             assert (f, a, w) == (int(F_d[S].item()), int(split_d[S].item()) & 0xFFFFFFFF, int(wI_d[S].item()))
 
 
+def test_m32_maximum(mpt):
+    """m = 32, the largest instance the ABI takes (subset masks use all 32 bits,
+    2^32-entry tables), on lean tables: layout trie cost = OPT, bounds, sampled
+    subsets of every size whose split attains F(S) with w(I(S)) recomputed by
+    direct intersection, random other splits never better, and small subsets
+    recomputed by the oracle from their own submask tables."""
+    inst = I.config(7)
+    m = inst.m
+    assert m == 32
+    res = mpt.solve(inst.weights, inst.bits, tables="lean")
+    F_d, split_d = mpt.mpt_tables32(res.ctx)
+    assert O.trie_cost(inst.weights, res.permutations()) == res.opt
+    assert mpt.mpt_trie_cost(inst.weights, res.perm_offsets, res.perm_chunks) == res.opt
+    R = O.request_sets(inst.weights, inst.bits)
+    assert all(sorted(p) == sorted(R[i]) for i, p in enumerate(res.permutations()))
+    assert O.spanning_tree_bound(inst.weights, inst.bits) <= res.opt <= O.global_order_cost(inst.weights, inst.bits)
+    rng = np.random.default_rng(32)
+    full = (1 << m) - 1
+    assert int(F_d[full].item()) == res.opt
+    Ss = [full] + [int(sum(1 << int(i) for i in rng.choice(m, size=k, replace=False)))
+                   for k in range(2, m + 1) for _ in range(3)]
+    wI = {S: O.wI_one(inst.weights, inst.bits, S) for S in Ss}
+    for S in Ss:
+        A = int(split_d[S].item()) & 0xFFFFFFFF
+        assert A & S == A and A & (S & -S) and A != S
+        assert int(F_d[S].item()) == int(F_d[A].item()) + int(F_d[S ^ A].item()) - wI[S]
+    for _ in range(100):  # random other splits never beat the chosen one
+        S = Ss[int(rng.integers(0, len(Ss)))]
+        low = S & -S
+        rest = S ^ low
+        sub = sum(1 << i for i in range(m) if (rest >> i) & 1 and rng.random() < 0.5)
+        if sub == rest:
+            continue
+        A = low | sub
+        assert int(F_d[A].item()) + int(F_d[S ^ A].item()) - wI[S] >= int(F_d[S].item())
+    for k in range(2, 13):
+        for _ in range(3):
+            S = int(sum(1 << int(i) for i in rng.choice(m, size=k, replace=False)))
+            idx = torch.from_numpy(_submask_index(S)).to(F_d.device)
+            f, a, w = O.recompute_local(inst.weights, inst.bits, S, F_d[idx].to(torch.int64).cpu().numpy())
+            assert (f, a) == (int(F_d[S].item()), int(split_d[S].item()) & 0xFFFFFFFF)
+
+
 def test_concurrent_contexts_on_streams(mpt):
     """Independent contexts solved at the same time on different streams (own
     workspaces) give the same tables as solving them one after the other: no
