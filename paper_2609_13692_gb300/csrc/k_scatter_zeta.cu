@@ -67,6 +67,56 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_low(G* __restrict__ g, in
   for (int i = threadIdx.x; i < size; i += blockDim.x) tile[i] = t[i];
 }
 
+// The same for tb = 12 with fewer barriers: thread t holds 8 consecutive
+// entries (bits 0-2 in registers), bits 3-7 are the lane bits (warp shuffles),
+// then one shared-memory pass regroups the tile so that each thread holds 8
+// entries 256 apart (bits 8-10 in registers) and bit 11 is one shared-memory
+// stage.  Sums are order-independent, so every stage is the same add.
+template <typename G>
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_low12(G* __restrict__ g) {
+  static_assert(kZetaThreads * 8 == (1 << kZetaLowBits), "8 entries per thread");
+  __shared__ G t[1 << kZetaLowBits];
+  G* tile = g + ((size_t)blockIdx.x << kZetaLowBits);
+  const int tid = threadIdx.x, lane = tid & 31;
+  G v[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = tile[tid * 8 + i];
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (!(i & (1 << j))) v[i] += v[i | (1 << j)];
+#pragma unroll
+  for (int j = 0; j < 5; ++j) {
+    const bool low = !(lane & (1 << j));  // this lane's entries have bit 3 + j clear
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const G o = __shfl_xor_sync(0xFFFFFFFFu, v[i], 1 << j);
+      if (low) v[i] += o;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t[tid * 8 + i] = v[i];
+  __syncthreads();
+  // regroup: thread t takes entries base + 256 k, k < 8 (bits 8-10)
+  const int base = (tid & 255) | ((tid >> 8) << 11);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) v[k] = t[base + 256 * k];
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (!(k & (1 << j))) v[k] += v[k | (1 << j)];
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < 8; ++k) t[base + 256 * k] = v[k];
+  __syncthreads();
+  // bit 11, then write back
+  for (int i = tid; i < (1 << (kZetaLowBits - 1)); i += kZetaThreads) t[i] += t[i | (1 << 11)];
+  __syncthreads();
+  for (int i = tid; i < (1 << kZetaLowBits); i += kZetaThreads) tile[i] = t[i];
+}
+
 // Superset sums over index bits [lo, lo + tb): each block owns 16 adjacent
 // columns (bits below lo) and all 2^tb values of those bits, for one value of
 // the bits above; rows of 16 entries are contiguous 128-byte segments.
@@ -103,6 +153,61 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_high(G* __restrict__ g, i
   }
 }
 
+// k_zeta_high for tb = 8 with fewer barriers: thread t owns column t & 15
+// and holds 8 rows ((t >> 4) * 8 + i: row bits 0-2 in registers, row bit 3 by
+// a warp shuffle); one shared-memory pass regroups so that each thread holds
+// rows 16 apart (row bits 4-6 in registers), and row bit 7 is one
+// shared-memory stage.
+template <typename G>
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_high8(G* __restrict__ g, int lo) {
+  static_assert(kZetaThreads * 8 == (1 << kZetaHighBits) * kZetaCols, "8 entries per thread");
+  __shared__ G t[(1 << kZetaHighBits) * kZetaCols];
+  const size_t col_groups = ((size_t)1 << lo) / kZetaCols;
+  const size_t cg = blockIdx.x % col_groups;
+  const size_t top = blockIdx.x / col_groups;
+  G* base = g + (top << (lo + kZetaHighBits)) + cg * kZetaCols;
+  const int tid = threadIdx.x, c = tid & (kZetaCols - 1), rg = tid >> 4;
+  G v[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = base[((size_t)(rg * 8 + i) << lo) + c];
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if (!(i & (1 << j))) v[i] += v[i | (1 << j)];
+  {
+    const bool low = !(rg & 1);  // row bit 3 clear; the partner row group is lane ^ 16
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const G o = __shfl_xor_sync(0xFFFFFFFFu, v[i], 16);
+      if (low) v[i] += o;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t[(rg * 8 + i) * kZetaCols + c] = v[i];
+  __syncthreads();
+  // regroup: rows (rg & 15) | (k << 4) | ((rg >> 4) << 7), k < 8 (row bits 4-6)
+  const int r0 = (rg & 15) | ((rg >> 4) << 7);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) v[k] = t[(r0 | (k << 4)) * kZetaCols + c];
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (!(k & (1 << j))) v[k] += v[k | (1 << j)];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) t[(r0 | (k << 4)) * kZetaCols + c] = v[k];
+  __syncthreads();
+  // row bit 7: rows r < 128 take row r + 128
+  constexpr int kHalf = (1 << (kZetaHighBits - 1)) * kZetaCols;
+  for (int i = tid; i < kHalf; i += kZetaThreads) t[i] += t[i + kHalf];
+  __syncthreads();
+  for (int e = tid; e < (1 << kZetaHighBits) * kZetaCols; e += kZetaThreads) {
+    const int r = e / kZetaCols, cc = e % kZetaCols;
+    base[((size_t)r << lo) + cc] = t[e];
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
@@ -126,14 +231,20 @@ template <typename G>
 static cudaError_t zeta(const Shape& s, G* g, cudaStream_t stream, int* launches) {
   const int tb = s.m < kZetaLowBits ? s.m : kZetaLowBits;
   const size_t low_blocks = (size_t)1 << (s.m - tb);
-  k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb);
+  if (tb == kZetaLowBits)
+    k_zeta_low12<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g);
+  else
+    k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb);
   ++*launches;
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   for (int lo = tb; lo < s.m; lo += kZetaHighBits) {
     const int hb = (s.m - lo) < kZetaHighBits ? (s.m - lo) : kZetaHighBits;
     const size_t blocks = ((size_t)1 << s.m) / (((size_t)1 << hb) * kZetaCols);
-    k_zeta_high<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, hb);
+    if (hb == kZetaHighBits)
+      k_zeta_high8<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo);
+    else
+      k_zeta_high<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, hb);
     ++*launches;
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
