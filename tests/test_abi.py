@@ -274,3 +274,31 @@ def test_helper_argument_checks(mpt):
     assert lib.mpt_gather_bandwidth(33, 1000, None, ctypes.byref(gbps)) == 1
     assert lib.mpt_gather_bandwidth(20, 0, None, ctypes.byref(gbps)) == 1
     assert lib.mpt_gather_bandwidth(20, 1000, None, None) == 1
+
+
+def test_caller_workspace_checks(mpt):
+    """A caller workspace below mpt_workspace_bytes() or off a 256-byte
+    boundary is refused by mpt_solve, mpt_solve_begin and mpt_solve_resume
+    before any copy or launch (the fake pointers are never dereferenced)."""
+    import ctypes
+
+    lib = mpt.load()
+    inst = I.random_instance(12, 30, 3, seed=4)
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    need = mpt.mpt_workspace_bytes(ctx)
+    opt = ctypes.c_int64()
+    aligned, misaligned = ctypes.c_void_p(1 << 20), ctypes.c_void_p((1 << 20) + 16)
+    assert lib.mpt_solve(ctx.handle, aligned, need - 1, None, ctypes.byref(opt)) == 5
+    assert lib.mpt_solve(ctx.handle, misaligned, need, None, ctypes.byref(opt)) == 1
+    assert lib.mpt_solve(ctx.handle, aligned, need, None, None) == 1  # no place for OPT
+    assert lib.mpt_solve(None, aligned, need, None, ctypes.byref(opt)) == 1
+    assert lib.mpt_solve_begin(ctx.handle, aligned, need - 256, None) == 5
+    assert lib.mpt_solve_begin(ctx.handle, misaligned, need, None) == 1
+    assert lib.mpt_solve_resume(ctx.handle, aligned, need - 1, 1) == 5
+    assert lib.mpt_solve_resume(ctx.handle, misaligned, need, 1) == 1
+    # a refused call leaves nothing begun and nothing solved
+    assert lib.mpt_solve_layers(ctx.handle, aligned, need, None, 1, None) == 7
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_layout(ctx)
+    assert e.value.status == 7
+    mpt.mpt_destroy(ctx)
