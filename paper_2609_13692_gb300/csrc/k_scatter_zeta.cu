@@ -12,6 +12,19 @@
 // recurrence g is indexed in its rotated order (rot_index): the superset
 // relation does not depend on the order of the index bits, so the same
 // transform then yields w(I(S)) at the rotated position of S.
+//
+// Private chunks (blocked paths).  A chunk x with S_x = {i} is one maximal
+// cluster of S_x in every hierarchy (t_x(H) = 1 in Thm 1), so it adds w(x)
+// to F(S) for every S containing i whatever the splits: with
+// pi_i = sum of w(x) over x with N_x = {i} and pi(S) = sum_{i in S} pi_i,
+//     F(S) = F'(S) + pi(S),   F'({i}) = w(R_i) - pi_i,
+//     F'(S) = min over splits of F'(A) + F'(B) - w(I(S))   (|S| >= 2),
+// since pi(A) + pi(B) = pi(S) and w(I(S)) does not involve private chunks
+// for |S| >= 2.  The argmin is the same.  For the blocked paths K1 adds such
+// chunks to pi_i instead of to g, so the transform yields w(I(S)) for
+// |S| >= 2 and w(R_i) - pi_i for S = {i}; the recurrence then runs on F',
+// whose candidates stay below the shared weight sum_i (w(R_i) - pi_i), the
+// quantity the packed keys must hold.
 #include "mpt_internal.cuh"
 
 namespace mpt {
@@ -20,11 +33,12 @@ namespace {
 constexpr int kScatterThreads = 256;
 
 // g is uint64 (int64 tables) or uint32 (lean tables, sum_i w(R_i) < 2^31).
+// priv: pi_i of the private chunks (blocked paths), or nullptr.
 template <typename G>
 __global__ void __launch_bounds__(kScatterThreads)
 k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m, int64_t words,
-          G* __restrict__ g, uint32_t* __restrict__ used_N, int32_t* __restrict__ used_x,
-          int32_t* __restrict__ counters, int64_t slots, bool rotated, int L, int b) {
+          G* __restrict__ g, unsigned long long* __restrict__ priv, uint32_t* __restrict__ used_N,
+          int32_t* __restrict__ used_x, int32_t* __restrict__ counters, int64_t slots, bool rotated, int L, int b) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
     const int64_t word = x >> 6;
@@ -32,7 +46,10 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
     uint32_t N = 0;
     for (int i = 0; i < m; ++i) N |= (uint32_t)((__ldg(&bits[(int64_t)i * words + word]) >> sh) & 1ull) << i;
     if (N) {
-      atomicAdd(&g[rotated ? rot_index(N, L, b) : (size_t)N], (G)w[x]);
+      if (priv && (N & (N - 1)) == 0)
+        atomicAdd(&priv[__ffs(N) - 1], (unsigned long long)w[x]);
+      else
+        atomicAdd(&g[rotated ? rot_index(N, L, b) : (size_t)N], (G)w[x]);
       const int k = atomicAdd(&counters[0], 1);
       if (k < slots) {
         used_N[k] = N;
@@ -217,12 +234,12 @@ cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t str
   void* g = g_table(s, ws);
   if (s.lean)
     k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
-        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned int*>(g), ws.used_N, ws.used_x, ws.counters,
-        s.slots, s.blocked, s.L, s.b);
+        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned int*>(g), s.blocked ? ws.priv : nullptr,
+        ws.used_N, ws.used_x, ws.counters, s.slots, s.blocked, s.L, s.b);
   else
     k_scatter<<<(unsigned)blocks, kScatterThreads, 0, stream>>>(
-        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned long long*>(g), ws.used_N, ws.used_x,
-        ws.counters, s.slots, s.blocked, s.L, s.b);
+        ws.weights, ws.bits, s.n, s.m, s.words, static_cast<unsigned long long*>(g), s.blocked ? ws.priv : nullptr,
+        ws.used_N, ws.used_x, ws.counters, s.slots, s.blocked, s.L, s.b);
   ++*launches;
   return cudaGetLastError();
 }

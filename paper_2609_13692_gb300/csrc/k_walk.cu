@@ -8,9 +8,10 @@
 // request set of x), and request i's permutation is R_i sorted by
 // (depth of that node, chunk id).  The left-to-right leaf order is the trie
 // DFS order that Thm 7 (Sec. 8) serves requests in.  After a blocked solve
-// split is read at the rotated position of each node and OPT = F(full) from
-// Gp = F << b (uint32, or uint64 on the wide path); after a general one both
-// are in natural order.
+// split is read at the rotated position of each node and OPT = F(full) =
+// F'(full) + sum_i pi_i from Gp = F' << b (uint32, or uint64 on the wide
+// path) and the private weights pi (k_scatter_zeta.cu); after a general one
+// both are in natural order.
 //
 // Trie cost: a string's node at depth p is new exactly when no earlier
 // string shares its first p+1 symbols, so the trie weight is
@@ -25,8 +26,8 @@ constexpr int kMaxM = 32;
 
 __global__ void __launch_bounds__(kWalkThreads)
 k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F, const int32_t* __restrict__ F32,
-       const uint32_t* __restrict__ Gp, const unsigned long long* __restrict__ Gp64, int L, int b,
-       const uint32_t* __restrict__ used_N,
+       const uint32_t* __restrict__ Gp, const unsigned long long* __restrict__ Gp64,
+       const unsigned long long* __restrict__ priv, int L, int b, const uint32_t* __restrict__ used_N,
        const int32_t* __restrict__ used_x, int32_t* __restrict__ counters, int64_t slots,
        unsigned long long* __restrict__ keys, int64_t* __restrict__ perm_offsets, int64_t* __restrict__ perm_chunks,
        int32_t* __restrict__ dfs, int64_t* __restrict__ opt) {
@@ -77,8 +78,11 @@ k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F,
       ++sp;
     }
     if (bad) atomicOr(&counters[1], kErrBadSplit);
-    *opt = Gp64 ? (int64_t)(Gp64[rot_index(full, L, b)] >> b)
-           : Gp ? (int64_t)(Gp[rot_index(full, L, b)] >> b)
+    int64_t pi_all = 0;
+    if (priv)
+      for (int i = 0; i < m; ++i) pi_all += (int64_t)priv[i];
+    *opt = Gp64 ? (int64_t)(Gp64[rot_index(full, L, b)] >> b) + pi_all
+           : Gp ? (int64_t)(Gp[rot_index(full, L, b)] >> b) + pi_all
                 : (F ? F[full] : (int64_t)F32[full]);
   }
   __syncthreads();
@@ -161,7 +165,8 @@ k_trie_cost(int m, const int64_t* __restrict__ w, const int64_t* __restrict__ of
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
   k_walk<<<1, kWalkThreads, 0, stream>>>(s.m, s.blocked ? ws.split_rot : ws.split, s.lean ? nullptr : ws.F,
                                          s.lean ? ws.fw : nullptr, s.blocked && !s.wide ? ws.Gp : nullptr,
-                                         s.blocked && s.wide ? ws.Gp64 : nullptr, s.L, s.b, ws.used_N,
+                                         s.blocked && s.wide ? ws.Gp64 : nullptr, s.blocked ? ws.priv : nullptr,
+                                         s.L, s.b, ws.used_N,
                                          ws.used_x, ws.counters, s.slots, ws.keys,
                                          ws.perm_offsets, ws.perm_chunks, ws.dfs, ws.opt);
   ++*launches;

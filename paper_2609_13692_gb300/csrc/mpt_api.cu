@@ -16,7 +16,8 @@ struct mpt_ctx {
   mpt::Shape shape{};
   std::vector<int64_t> w;
   std::vector<uint64_t> bits;
-  int64_t sum_w = 0;  // sum_i w(R_i)
+  int64_t sum_w = 0;     // sum_i w(R_i)
+  int64_t shared_w = 0;  // the same less the chunks only one request needs
   int32_t mode = MPT_DP_AUTO;
   int32_t tables = MPT_TABLES_INT64;
   void* own_ws = nullptr;
@@ -49,12 +50,14 @@ constexpr int64_t kSumLimit = (int64_t)1 << 62;
 
 constexpr int64_t kWideLimit = (int64_t)1 << 51;  // 64-bit keys: F(A) + F(B) < 2^52
 
+// The blocked recurrence runs on F' = F - pi(S) (k_scatter_zeta.cu), whose
+// candidates F'(A) + F'(B) stay at most the shared weight.
 bool blocked_feasible(const mpt_ctx* c) {
   const int b = mpt::blocked_tile_bits(c->shape.m);
-  return c->sum_w < ((int64_t)1 << (32 - b));
+  return c->shared_w < ((int64_t)1 << (32 - b));
 }
 
-bool wide_feasible(const mpt_ctx* c) { return c->sum_w < kWideLimit; }
+bool wide_feasible(const mpt_ctx* c) { return c->shared_w < kWideLimit; }
 
 bool use_blocked(const mpt_ctx* c) {
   if (c->mode == MPT_DP_GENERAL) return false;
@@ -133,6 +136,7 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws) {
     ws->Gc = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->partial = reinterpret_cast<unsigned long long*>(take((size_t)(s.partial_entries > 0 ? s.partial_entries : 1) * 8));
   }
+  ws->priv = s.blocked ? reinterpret_cast<unsigned long long*>(take(32 * 8)) : nullptr;
   if (s.blocked) {
     // The rotated tables share the buffers of the natural ones: w(I) sits in
     // the F table (int64) or in fw (lean), split in the split table.  The
@@ -200,6 +204,18 @@ mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* 
       }
     }
   }
+  // weight of the chunks exactly one request needs: per word, the bits seen
+  // once (s1) but not twice (s2) over all requests
+  int64_t private_w = 0;
+  for (int64_t j = 0; j < words; ++j) {
+    uint64_t s1 = 0, s2 = 0;
+    for (int i = 0; i < m; ++i) {
+      const uint64_t v = req_bits[(size_t)i * (size_t)words + (size_t)j];
+      s2 |= s1 & v;
+      s1 |= v;
+    }
+    for (uint64_t v = s1 & ~s2; v; v &= v - 1) private_w += weights[j * 64 + __builtin_ctzll(v)];
+  }
   mpt_ctx* c = new (std::nothrow) mpt_ctx();
   if (!c) return MPT_ERR_OUT_OF_MEMORY;
   try {
@@ -214,6 +230,7 @@ mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* 
   c->shape.words = words;
   c->shape.slots = slots;
   c->sum_w = sum;
+  c->shared_w = sum - private_w;
   refresh_shape(c);
   *out = c;
   return MPT_OK;
@@ -309,6 +326,7 @@ mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStrea
     MPT_CK(cudaMemcpyAsync(ws.bits, c->bits.data(), c->bits.size() * 8, cudaMemcpyHostToDevice, stream), "copy bits");
   }
   MPT_CK(cudaMemsetAsync(ws.counters, 0, 8 * 4, stream), "memset counters");
+  if (ws.priv) MPT_CK(cudaMemsetAsync(ws.priv, 0, 32 * 8, stream), "memset private weights");
   MPT_CK(cudaMemsetAsync(mpt::g_table(s, ws), 0, N * (s.lean ? 4 : 8), stream), "memset g");
   mark(1);
   MPT_CK(mpt::launch_scatter(s, ws, stream, launches), "scatter kernel");
@@ -558,10 +576,10 @@ mpt_status ensure_natural(mpt_ctx* c) {
   if (e == cudaSuccess && s.wide)
     e = mpt::unrotate_tables_wide(s, ws.split_rot, reinterpret_cast<uint32_t*>(ws.Gc64), ws.wI_rot,
                                   s.lean ? nullptr : ws.wI, ws.Gp64, s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr,
-                                  c->conv_stream);
+                                  ws.priv, c->conv_stream);
   else if (e == cudaSuccess)
     e = mpt::unrotate_tables(s, ws.split_rot, ws.Gc, ws.wI_rot, s.lean ? nullptr : ws.wI, ws.Gp,
-                             s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr, c->conv_stream);
+                             s.lean ? nullptr : ws.F, s.lean ? ws.fw : nullptr, ws.priv, c->conv_stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->conv_stream);
   if (e != cudaSuccess) st = cuda_fail(c, e, "natural-order tables");
   cudaSetDevice(prev);

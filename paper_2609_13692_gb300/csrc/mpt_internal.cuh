@@ -100,8 +100,8 @@ struct Workspace {
   uint32_t* split;    // [2^m]
   // blocked DP working tables, rotated order idx(S) = (T << b) | U with
   // T = S mod 2^L and U = S >> L (see k_dp_blocked.cu)
-  uint32_t* Gp;       // [2^m]  F << b
-  uint32_t* Gc;       // [2^m]  (F << b) | (~u & (2^b - 1))
+  uint32_t* Gp;       // [2^m]  F' << b, F'(S) = F(S) - sum_{i in S} pi_i
+  uint32_t* Gc;       // [2^m]  (F' << b) | (~u & (2^b - 1))
   unsigned long long* partial;  // [max tiles of one layer << b]
   // wide blocked path (64-bit keys): Gp and Gc hold uint64 entries, and the
   // pair kernel leaves one (key, Ta) slot of 2^b entries per block
@@ -111,6 +111,10 @@ struct Workspace {
   int64_t* wI_rot;    // [2^m] w(I(S)) at idx(S) (int64 tables), or nullptr
   int32_t* fw_rot;    // [2^m] w(I(S)) at idx(S) (lean tables), or nullptr
   uint32_t* split_rot;  // [2^m] split[S] at idx(S)
+  // blocked paths: pi_i = w of the chunks that request i alone needs, which
+  // K1 adds here instead of to g; the rotated tables then hold w(I) and F
+  // less those weights (see scatter in k_scatter_zeta.cu)
+  unsigned long long* priv;  // [32] or nullptr
   // layout
   unsigned long long* keys;  // [slots]
   int64_t* perm_offsets;     // [m + 1]
@@ -125,7 +129,7 @@ struct Shape {
   int64_t words;
   int64_t slots;    // sum_i |R_i|
   bool blocked;     // blocked DP tables present
-  bool wide;        // blocked path with 64-bit keys (sum_i w(R_i) >= 2^(32-b))
+  bool wide;        // blocked path with 64-bit keys (shared weight >= 2^(32-b))
   bool lean;        // one int32 table for w(I(S)) then F(S)
   int b;            // tile bits (blocked)
   int L;            // m - b
@@ -178,8 +182,9 @@ int blocked_tile_bits(int m);
 void choose_items(unsigned long long tiles, uint32_t P, int sms, unsigned long long max_items,
                   unsigned long long* items, uint32_t* ppi);
 
-// Wide blocked path (k_dp_wide.cu): 64-bit keys, valid when
-// sum_i w(R_i) < 2^51.  Partial slots: blocks of one pair layer, at most.
+// Wide blocked path (k_dp_wide.cu): 64-bit keys, valid when the shared
+// weight sum_i (w(R_i) - pi_i) is below 2^51.  Partial slots: blocks of one
+// pair layer, at most.
 int64_t wide_partial_slots(int m, int b);
 cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
                            BlockedTiming* timing, int step_begin = 0, int step_end = -1);
@@ -187,17 +192,19 @@ cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t str
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
 
 // Natural-order tables from the blocked path's rotated ones (k_tables.cu):
-// split_nat[S] = split_rot[idx(S)]; wI_nat[S] = wI_rot[idx(S)] (int64
-// tables); F_nat[S] or F32_nat[S] = Gp[idx(S)] >> b.  Null destinations are
-// skipped; they run in this order, so a destination may be the source of an
-// earlier conversion.
+// split_nat[S] = split_rot[idx(S)]; wI_nat[S] = wI_rot[idx(S)] plus pi_i for
+// S = {i} and sum_i pi_i for S = {} (int64 tables); F_nat[S] or F32_nat[S] =
+// (Gp[idx(S)] >> b) + sum_{i in S} pi_i.  priv (pi, m entries on the device)
+// may be null: no private weights.  Null destinations are skipped; they run
+// in this order, so a destination may be the source of an earlier conversion.
 cudaError_t unrotate_tables(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat, const int64_t* wI_rot,
                             int64_t* wI_nat, const uint32_t* Gp, int64_t* F_nat, int32_t* F32_nat,
-                            cudaStream_t stream);
+                            const unsigned long long* priv, cudaStream_t stream);
 // The same for the wide path (F from the uint64 Gp table).
 cudaError_t unrotate_tables_wide(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat,
                                  const int64_t* wI_rot, int64_t* wI_nat, const unsigned long long* Gp64,
-                                 int64_t* F_nat, int32_t* F32_nat, cudaStream_t stream);
+                                 int64_t* F_nat, int32_t* F32_nat, const unsigned long long* priv,
+                                 cudaStream_t stream);
 // eq. (1) for any number of strings by lexicographic sorting (k_sched.cu)
 mpt_status trie_cost_lex(const int64_t* weights, int64_t n_chunks, int64_t m, const int64_t* offsets,
                          const int64_t* chunks, cudaStream_t st, int64_t* cost);

@@ -39,7 +39,9 @@ constexpr size_t kOffGp = align_up(kOffUsedX + kNoAllocMaxSlots * sizeof(int32_t
 constexpr size_t kOffGc = align_up(kOffGp + (sizeof(uint32_t) << kNoAllocMaxM));
 constexpr size_t kOffPartial = align_up(kOffGc + (sizeof(uint32_t) << kNoAllocMaxM));
 constexpr size_t kOffCheck = align_up(kOffPartial + max_partial_entries() * sizeof(unsigned long long));
-constexpr size_t kScratchBytes = align_up(kOffCheck + 4 * sizeof(unsigned long long));
+constexpr int kChecks = 6;
+constexpr size_t kOffPriv = align_up(kOffCheck + kChecks * sizeof(unsigned long long));
+constexpr size_t kScratchBytes = align_up(kOffPriv + 32 * sizeof(unsigned long long));
 
 // The scratch: about 10.7 MiB per device.  In host code `g_noalloc_scratch`
 // is only a host-side stand-in for the symbol; kernels receive the device
@@ -69,12 +71,15 @@ cudaError_t scratch_for_current_device(char** out) {
 }
 
 // Argument checks that need the device-resident inputs: every weight >= 1,
-// no request bit at a chunk >= n, the number of chunk occurrences, and
-// sum_i w(R_i).  Each term w(x) * |S_x| is capped at 2^62 (beyond which the
-// instance is rejected anyway) and added as two 32-bit halves into separate
-// 64-bit counters, which cannot wrap for n < 2^31.
+// no request bit at a chunk >= n, the number of chunk occurrences,
+// sum_i w(R_i), and the weight of the chunks that one request alone needs
+// (left out of the blocked recurrence's keys, see k_scatter_zeta.cu).  Each
+// term w(x) * |S_x| is capped at 2^62 (beyond which the instance is rejected
+// anyway) and added as two 32-bit halves into separate 64-bit counters, which
+// cannot wrap for n < 2^31.
 //   check[0] = bad weight or stray bit, check[1] = occurrences,
-//   check[2] = sum of the low halves, check[3] = sum of the high halves
+//   check[2] / check[3] = sums of the low / high halves of the terms,
+//   check[4] / check[5] = the same for the private chunks' terms
 __global__ void k_noalloc_check(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m,
                                 int64_t words, unsigned long long* __restrict__ check) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -99,6 +104,10 @@ __global__ void k_noalloc_check(const int64_t* __restrict__ w, const uint64_t* _
           (unsigned long long)wx > cap / (unsigned long long)cnt ? cap : (unsigned long long)wx * (unsigned long long)cnt;
       atomicAdd(&check[2], term & 0xFFFFFFFFull);
       atomicAdd(&check[3], term >> 32);
+      if (cnt == 1) {
+        atomicAdd(&check[4], term & 0xFFFFFFFFull);
+        atomicAdd(&check[5], term >> 32);
+      }
     }
   }
 }
@@ -118,14 +127,14 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
 
   const int64_t words = (n_chunks + 63) / 64;
   unsigned long long* check = reinterpret_cast<unsigned long long*>(base + kOffCheck);
-  if (cudaMemsetAsync(check, 0, 4 * sizeof(unsigned long long), stream) != cudaSuccess) return MPT_ERR_CUDA;
+  if (cudaMemsetAsync(check, 0, kChecks * sizeof(unsigned long long), stream) != cudaSuccess) return MPT_ERR_CUDA;
   {
     int64_t blocks = (words * 64 + 255) / 256;
     if (blocks > 152 * 16) blocks = 152 * 16;
     k_noalloc_check<<<(unsigned)blocks, 256, 0, stream>>>(d_weights, d_req_bits, n_chunks, m, words, check);
     if (cudaGetLastError() != cudaSuccess) return MPT_ERR_CUDA;
   }
-  unsigned long long h_check[4] = {0, 0, 0, 0};
+  unsigned long long h_check[kChecks] = {0, 0, 0, 0, 0, 0};
   if (cudaMemcpyAsync(h_check, check, sizeof(h_check), cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
       cudaStreamSynchronize(stream) != cudaSuccess)
     return MPT_ERR_CUDA;
@@ -133,6 +142,7 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   if (h_check[1] > (unsigned long long)kNoAllocMaxSlots) return MPT_ERR_TOO_LARGE;
   const unsigned __int128 sum_w = ((unsigned __int128)h_check[3] << 32) + h_check[2];
   if (sum_w >= ((unsigned __int128)1 << 62)) return MPT_ERR_OVERFLOW;
+  const unsigned __int128 private_w = ((unsigned __int128)h_check[5] << 32) + h_check[4];
 
   mpt::Shape s{};
   s.m = m;
@@ -141,7 +151,7 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   s.slots = (int64_t)h_check[1];
   s.b = mpt::blocked_tile_bits(m);
   s.L = m - s.b;
-  s.blocked = sum_w < ((unsigned __int128)1 << (32 - s.b));
+  s.blocked = sum_w - private_w < ((unsigned __int128)1 << (32 - s.b));
   s.partial_entries = s.blocked ? mpt::blocked_partial_entries(m, s.b) : 0;
 
   mpt::Workspace ws{};
@@ -156,6 +166,7 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   ws.Gp = reinterpret_cast<uint32_t*>(base + kOffGp);
   ws.Gc = reinterpret_cast<uint32_t*>(base + kOffGc);
   ws.partial = reinterpret_cast<unsigned long long*>(base + kOffPartial);
+  ws.priv = s.blocked ? reinterpret_cast<unsigned long long*>(base + kOffPriv) : nullptr;
   // The blocked recurrence works on rotated tables: w(I) in the caller's F
   // table, split in its wI table; the natural outputs are written from them
   // at the end (split, then wI, then F from Gp).
@@ -168,7 +179,8 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   // the blocked launcher before each layer; Gp and Gc are fully rewritten).
   int launches = 0;
   if (cudaMemsetAsync(ws.counters, 0, 8 * sizeof(int32_t), stream) != cudaSuccess ||
-      cudaMemsetAsync(mpt::g_table(s, ws), 0, sizeof(int64_t) << m, stream) != cudaSuccess)
+      cudaMemsetAsync(mpt::g_table(s, ws), 0, sizeof(int64_t) << m, stream) != cudaSuccess ||
+      (ws.priv && cudaMemsetAsync(ws.priv, 0, 32 * sizeof(unsigned long long), stream) != cudaSuccess))
     return MPT_ERR_CUDA;
   if (mpt::launch_scatter(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;
   if (mpt::launch_zeta(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;
@@ -176,7 +188,8 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
                             : mpt::launch_dp_general(s, ws, stream, &launches);
   if (e != cudaSuccess) return MPT_ERR_CUDA;
   if (s.blocked &&
-      mpt::unrotate_tables(s, ws.split_rot, d_split, ws.wI_rot, d_wI, ws.Gp, d_F, nullptr, stream) != cudaSuccess)
+      mpt::unrotate_tables(s, ws.split_rot, d_split, ws.wI_rot, d_wI, ws.Gp, d_F, nullptr, ws.priv, stream) !=
+          cudaSuccess)
     return MPT_ERR_CUDA;
   const size_t full = ((size_t)1 << m) - 1;
   if (cudaMemcpyAsync(d_opt, d_F + full, sizeof(int64_t), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)

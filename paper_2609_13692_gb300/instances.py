@@ -40,6 +40,7 @@ __all__ = [
     "config",
     "CONFIGS",
     "random_instance",
+    "with_query_chunks",
     "k4_3",
     "open_problem_k4",
     "tightness_witness",
@@ -252,6 +253,21 @@ def random_instance(m: int, n: int, k: int | tuple[int, int], seed: int, wmin: i
             kk = 1
         reqs.append(rng.choice(n, size=kk, replace=False).tolist())
     return Instance(weights, pack_requests(reqs, n), f"random m={m} n={n} k={k} seed={seed}")
+
+
+def with_query_chunks(inst: Instance, wmin: int, wmax: int, seed: int, every: int = 1) -> Instance:
+    """``inst`` with one new chunk appended to every ``every``-th request: a
+    per-request suffix (its own question or document) that no other request
+    holds, of weight uniform in [wmin, wmax]."""
+    rng = np.random.default_rng(seed)
+    reqs = inst.requests()
+    owners = list(range(0, inst.m, every))
+    extra = rng.integers(wmin, wmax + 1, size=len(owners), dtype=np.int64)
+    n = inst.n + len(owners)
+    for j, i in enumerate(owners):
+        reqs[i] = list(reqs[i]) + [inst.n + j]
+    weights = np.concatenate([inst.weights, extra])
+    return Instance(weights, pack_requests(reqs, n), f"{inst.name} + query chunks [{wmin}, {wmax}]")
 
 
 def k4_3() -> Instance:

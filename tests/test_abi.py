@@ -9,6 +9,7 @@ import pytest
 
 from paper_2609_13692_gb300 import build as B
 from paper_2609_13692_gb300 import instances as I
+from tests import weights as W
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -302,3 +303,28 @@ def test_caller_workspace_checks(mpt):
         mpt.mpt_layout(ctx)
     assert e.value.status == 7
     mpt.mpt_destroy(ctx)
+
+
+def test_key_width_follows_shared_weight(mpt):
+    """The packed-key limits apply to the shared weight: private suffixes of
+    2^40 tokens keep the 32-bit keys (BLOCKED accepted, the narrow
+    workspace); a shared chunk of 2^20 tokens does not."""
+    base = I.config(1)  # m = 12
+    heavy_private = I.with_query_chunks(base, 1 << 40, 1 << 40, seed=1)
+    narrow = mpt.mpt_create(base.weights, base.bits)
+    ctx = mpt.mpt_create(heavy_private.weights, heavy_private.bits)
+    assert mpt.mpt_workspace_bytes(ctx) - mpt.mpt_workspace_bytes(narrow) < 4096  # the inputs grow by 12 chunks
+    mpt.mpt_set_dp_mode(ctx, "blocked")
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_set_tables(ctx, "lean")  # the int32 tables still need sum_i w(R_i) < 2^31
+    assert e.value.status == 3
+    shared = I.Instance(base.weights.copy(), base.bits)
+    x = int(np.flatnonzero(np.unpackbits(base.bits[0].view(np.uint8), bitorder="little"))[0])
+    assert W.request_counts(base)[x] >= 2
+    shared.weights[x] = 1 << 20  # a chunk of request 0 that other requests hold too
+    ctx2 = mpt.mpt_create(shared.weights, shared.bits)
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_set_dp_mode(ctx2, "blocked")
+    assert e.value.status == 3
+    for c in (narrow, ctx, ctx2):
+        mpt.mpt_destroy(c)

@@ -30,7 +30,7 @@ def _instances():
         I.Instance(np.array([3, 4, 5], dtype=np.int64), I.pack_requests([[], [0, 1], [], [0, 1], [2]], 3),
                    "empty and identical requests"),
         I.rag_pools(20, 5000, 6, 40, 8, 1.1, seed=11),
-        I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000),  # sum > 2^20: 64-bit keys
+        I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000),  # shared weight > 2^20: 64-bit keys
     ]
     rng = np.random.default_rng(61)
     for m in (2, 5, 9, 12, 13, 16, 18):

@@ -98,3 +98,36 @@ def test_config1_and_config2_full(C):
     perms, dfs = O.layout(inst.weights, inst.bits, split)
     assert O.trie_cost(inst.weights, perms) == opt
     assert O.spanning_tree_bound(inst.weights, inst.bits) <= opt <= O.global_order_cost(inst.weights, inst.bits)
+
+
+def test_private_chunks_shift_F_by_a_constant():
+    """Thm 1: a chunk that one request alone holds is one maximal cluster in
+    every hierarchy (t_x(H) = 1), so appending one to request i adds its
+    weight to F(S) for every S holding i, to w(I(S)) only at S = {i} and
+    S = {}, and changes no split.  The tiled kernels rely on this to leave
+    such weights out of their packed keys."""
+    rng = np.random.default_rng(123)
+    for t in range(8):
+        m = int(rng.integers(2, 11))
+        base = I.random_instance(m, 30, (0, 7), seed=int(rng.integers(1 << 30)), wmin=1, wmax=50, allow_empty=True)
+        inst = I.with_query_chunks(base, 1, 10 ** 6, seed=t, every=1 + t % 2)
+        q = np.zeros(m, dtype=np.int64)
+        owners = list(range(0, m, 1 + t % 2))
+        q[owners] = inst.weights[base.n:]
+        opt0, F0, wI0, s0 = O.solve(base.weights, base.bits)
+        opt1, F1, wI1, s1 = O.solve(inst.weights, inst.bits)
+        S = np.arange(1 << m, dtype=np.int64)
+        pi_S = sum(((S >> i) & 1) * q[i] for i in range(m))
+        assert np.array_equal(F1, F0 + pi_S)
+        expect_wI = wI0.copy()
+        expect_wI[[1 << i for i in range(m)]] += q
+        expect_wI[0] += int(q.sum())
+        assert np.array_equal(wI1, expect_wI)
+        assert np.array_equal(s1, s0)
+        assert opt1 == opt0 + int(q.sum())
+    # the same shift by brute force over all chunk orders (no recurrence)
+    base = I.Instance(np.array([2, 3, 1, 4], dtype=np.int64), I.pack_requests([[0, 1], [1, 2], [0, 2, 3]], 4))
+    inst = I.with_query_chunks(base, 5, 9, seed=1)
+    extra = int(inst.weights[base.n:].sum())
+    assert O.brute_force_permutations(inst.weights, inst.bits) == O.brute_force_permutations(base.weights,
+                                                                                            base.bits) + extra

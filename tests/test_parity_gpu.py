@@ -12,6 +12,7 @@ import pytest
 
 import oracle as O
 from paper_2609_13692_gb300 import instances as I
+from tests import weights as W
 
 pytestmark = pytest.mark.gpu
 
@@ -138,17 +139,19 @@ def test_edge_cases(mpt):
 
 
 def test_large_weights_use_wide_then_general(mpt):
-    """sum_i w(R_i) >= 2^20: the packed 32-bit keys would overflow, AUTO picks the 64-bit keys;
+    """Shared weight >= 2^20: the packed 32-bit keys would overflow, AUTO picks the 64-bit keys;
     from 2^51 on those would overflow too, and AUTO picks the int64 kernels."""
     inst = I.random_instance(14, 50, (3, 12), seed=9, wmin=10 ** 9, wmax=10 ** 12)
+    assert W.shared_weight(inst) >= 1 << 20
     assert_full_parity(mpt, inst, "auto", expect_mode=3)
     huge = I.random_instance(14, 50, (3, 12), seed=9, wmin=1 << 46, wmax=1 << 47)
-    assert sum(int(huge.weights[x]) for i in range(huge.m) for x in range(50) if (int(huge.bits[i, x >> 6]) >> (x & 63)) & 1) >= 1 << 51
+    assert W.shared_weight(huge) >= 1 << 51
     assert_full_parity(mpt, huge, "auto", expect_mode=2)
 
 
 def test_sum_just_below_blocked_limit(mpt):
-    """Largest weights the blocked kernels accept: sum_i w(R_i) = 2^20 - 1."""
+    """sum_i w(R_i) = 2^20 - 1 (chunks 16..19 private, the shared weight
+    955,371), BLOCKED forced."""
     m = 15
     reqs = [[i, (i + 1) % 20, (i + 7) % 20] for i in range(m)]
     w = np.full(20, 1, dtype=np.int64)

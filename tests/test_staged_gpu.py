@@ -25,7 +25,7 @@ def mpt():
 
 
 def _cases():
-    big = I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000)  # sum_i w(R_i) > 2^20
+    big = I.random_instance(14, 60, (2, 8), seed=5, wmin=100_000, wmax=400_000)  # shared weight > 2^20
     return [
         ("blocked m=20", I.rag_pools(20, 5000, 6, 40, 8, 1.1, seed=3), "auto"),
         ("blocked m=12 (one step)", I.config(1), "auto"),

@@ -1,5 +1,6 @@
 """The blocked recurrence with 64-bit packed keys (MPT_DP_WIDE, chosen by AUTO
-when 2^20 <= sum_i w(R_i) < 2^51) against the oracle and against the 32-bit
+when the shared weight -- sum_i w(R_i) less the chunks one request alone
+holds -- lies in [2^20, 2^51)) against the oracle and against the 32-bit
 path, through the C ABI.  Integer results: bit-exact.
 
 Scaling every chunk weight by c scales w(I(S)), F(S) and OPT by c and keeps
@@ -14,6 +15,7 @@ import pytest
 
 import oracle as O
 from paper_2609_13692_gb300 import instances as I
+from tests import weights as W
 
 pytestmark = [pytest.mark.gpu, pytest.mark.timeout(1500)]
 
@@ -27,11 +29,6 @@ def mpt():
 
     M.load()
     return M
-
-
-def _req_sum(inst):
-    return sum(int(inst.weights[x]) for i in range(inst.m) for x in range(inst.weights.shape[0])
-               if (int(inst.bits[i, x >> 6]) >> (x & 63)) & 1)
 
 
 def _solve(mpt, inst, mode="auto"):
@@ -56,12 +53,14 @@ def _parity(mpt, inst, mode="auto", expect_mode=3):
 
 @pytest.mark.parametrize("m", list(range(1, 19)))
 def test_wide_sweep_heavy_weights(mpt, m):
-    """Random instances with weights up to 2^40: AUTO takes the 64-bit keys."""
+    """Random instances with weights up to 2^40: AUTO takes the 64-bit keys
+    (the 32-bit ones where no chunk is shared, e.g. m = 1)."""
     rng = np.random.default_rng(5000 + m)
     n = int(rng.integers(8, 120))
     inst = I.random_instance(m, n, (1, min(n, 12)), seed=int(rng.integers(1 << 30)), wmin=1 << 20, wmax=1 << 40)
-    assert (1 << 20) <= _req_sum(inst) < (1 << 51)
-    _parity(mpt, inst)
+    shared = W.shared_weight(inst)
+    assert shared < (1 << 51) and W.request_weight_sum(inst) >= 1 << 20
+    _parity(mpt, inst, expect_mode=3 if shared >= 1 << 20 else 1)
 
 
 @pytest.mark.parametrize("m", [13, 15, 17, 18])
@@ -96,7 +95,7 @@ def _scaled_equal(mpt, inst, c):
     narrow = mpt.solve(inst.weights, inst.bits, profile=True)
     assert mpt.mpt_get_profile(narrow.ctx)["dp_mode"] == 1
     heavy = I.Instance(inst.weights * c, inst.bits)
-    assert _req_sum(heavy) >= 1 << 20
+    assert W.shared_weight(heavy) >= 1 << 20
     wide = mpt.solve(heavy.weights, heavy.bits, profile=True)
     assert mpt.mpt_get_profile(wide.ctx)["dp_mode"] == 3
     assert wide.opt == c * narrow.opt
@@ -127,11 +126,13 @@ def test_wide_lean_tables(mpt):
     import torch
 
     inst = I.random_instance(16, 60, (2, 8), seed=21, wmin=50_000, wmax=200_000)
-    assert (1 << 20) <= _req_sum(inst) < (1 << 31)
+    assert W.shared_weight(inst) >= 1 << 20 and W.request_weight_sum(inst) < 1 << 31
     ctx1 = mpt.mpt_create(inst.weights, inst.bits)
     o1 = mpt.mpt_solve(ctx1)
+    assert mpt.mpt_get_profile(ctx1)["dp_mode"] == 3
     F1, _, s1 = mpt.mpt_tables(ctx1)
     ctx2 = mpt.mpt_create(inst.weights, inst.bits)
+    mpt.mpt_set_dp_mode(ctx2, "wide")
     mpt.mpt_set_tables(ctx2, "lean")
     assert mpt.mpt_solve(ctx2) == o1
     F2, s2 = mpt.mpt_tables32(ctx2)

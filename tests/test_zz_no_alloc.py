@@ -59,6 +59,8 @@ def test_noalloc_matches_solve_on_consecutive_calls(mpt):
         I.random_instance(14, 60, (2, 10), seed=3, wmin=10 ** 9, wmax=10 ** 11),  # int64 kernels
         I.config(2),                                                         # the first instance again
         I.config(1),                                                         # m = 12, one tile
+        I.with_query_chunks(I.config(2), 1 << 30, 1 << 38, seed=2),          # private suffixes, blocked kernels
+        I.with_query_chunks(I.rag_pools(16, 5000, 4, 60, 8, 1.1, seed=11), 1 << 30, 1 << 38, seed=3),
     ]
     for inst in cases:
         ref = _reference(mpt, inst)
