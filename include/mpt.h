@@ -53,13 +53,15 @@ typedef enum mpt_status {
 typedef struct mpt_ctx mpt_ctx;
 
 /* DP kernels mpt_solve may use.  Their limits are on the shared weight
- * W = sum_i w(R_i) - sum_i pi_i, where pi_i is the weight of the chunks that
- * request i alone needs: such a chunk adds w(x) to F(S) for every S holding
- * i, whatever the hierarchy (t_x(H) = 1 in Thm 1), so the tiled kernels
- * run the recurrence on F(S) - sum_{i in S} pi_i and add it back in every
- * output.  AUTO picks BLOCKED whenever W < 2^20 (its 32-bit packed keys are
- * then exact), else WIDE while W < 2^51 (64-bit packed keys), else GENERAL.
- * All of them return the same tables, OPT and layout. */
+ * W = sum_i w(R_i) - sum_i pi_i - m u, where pi_i is the weight of the
+ * chunks that request i alone needs and u (m >= 2) that of the chunks every
+ * request needs.  Such a chunk is one cluster in every hierarchy (t_x(H) = 1
+ * in Thm 1): it adds w(x) to F(S) for every non-empty S holding its
+ * requests, whatever the splits.  The tiled kernels therefore run the
+ * recurrence on F(S) - sum_{i in S} pi_i - u and add it back in every output.
+ * AUTO picks BLOCKED whenever W < 2^20 (its 32-bit packed keys are then
+ * exact), else WIDE while W < 2^51 (64-bit packed keys), else GENERAL.  All
+ * of them return the same tables, OPT and layout. */
 typedef enum mpt_dp_mode {
   MPT_DP_AUTO = 0,
   MPT_DP_BLOCKED = 1, /* shared-memory tiled min-plus; needs W < 2^20 */

@@ -20,10 +20,14 @@
 //     F(S) = F'(S) + pi(S),   F'({i}) = w(R_i) - pi_i,
 //     F'(S) = min over splits of F'(A) + F'(B) - w(I(S))   (|S| >= 2),
 // since pi(A) + pi(B) = pi(S) and w(I(S)) does not involve private chunks
-// for |S| >= 2.  The argmin is the same.  For the blocked paths K1 adds such
-// chunks to pi_i instead of to g, so the transform yields w(I(S)) for
-// |S| >= 2 and w(R_i) - pi_i for S = {i}; the recurrence then runs on F',
-// whose candidates stay below the shared weight sum_i (w(R_i) - pi_i), the
+// for |S| >= 2.  The argmin is the same.  Likewise a chunk that all m >= 2
+// requests hold has S_x = the root, one cluster in every hierarchy: with u
+// the weight of such chunks, F(S) = F'(S) + pi(S) + u for non-empty S, and
+// the recurrence on F' sees w(I(S)) - u (u + u - u = u per split).  For the
+// blocked paths K1 adds private chunks to pi_i and universal ones to u
+// instead of to g, so the transform yields w(I(S)) - u for |S| >= 2 and
+// w(R_i) - pi_i - u for S = {i}; the recurrence then runs on F', whose
+// candidates stay below the shared weight sum_i (w(R_i) - pi_i - u), the
 // quantity the packed keys must hold.
 #include "mpt_internal.cuh"
 
@@ -33,13 +37,15 @@ namespace {
 constexpr int kScatterThreads = 256;
 
 // g is uint64 (int64 tables) or uint32 (lean tables, sum_i w(R_i) < 2^31).
-// priv: pi_i of the private chunks (blocked paths), or nullptr.
+// priv: pi_i of the private chunks and u of the universal ones (blocked
+// paths, kOffsetSlots entries), or nullptr.
 template <typename G>
 __global__ void __launch_bounds__(kScatterThreads)
 k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m, int64_t words,
           G* __restrict__ g, unsigned long long* __restrict__ priv, uint32_t* __restrict__ used_N,
           int32_t* __restrict__ used_x, int32_t* __restrict__ counters, int64_t slots, bool rotated, int L, int b) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const uint32_t full = m >= 32 ? 0xFFFFFFFFu : (1u << m) - 1u;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
     const int64_t word = x >> 6;
     const int sh = (int)(x & 63);
@@ -48,6 +54,8 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
     if (N) {
       if (priv && (N & (N - 1)) == 0)
         atomicAdd(&priv[__ffs(N) - 1], (unsigned long long)w[x]);
+      else if (priv && N == full)  // m >= 2 here: for m = 1 the full set is a singleton
+        atomicAdd(&priv[kUniversalSlot], (unsigned long long)w[x]);
       else
         atomicAdd(&g[rotated ? rot_index(N, L, b) : (size_t)N], (G)w[x]);
       const int k = atomicAdd(&counters[0], 1);

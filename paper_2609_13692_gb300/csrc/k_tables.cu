@@ -6,9 +6,10 @@
 // is the transpose of that 2^L x 2^b matrix; it is produced only when the
 // tables themselves are asked for, by a shared-memory tiled transpose (32 x 32
 // tiles: reads coalesced along U, writes along T).  The same pass adds back
-// the private weights pi_i that the blocked recurrence leaves out
-// (k_scatter_zeta.cu): sum_{i in S} pi_i to F(S), pi_i to w(I({i})) and
-// sum_i pi_i to w(I({})), the weight of the union of all requests.
+// the weights that the blocked recurrence leaves out (k_scatter_zeta.cu):
+// the private pi_i and the universal u, i.e. sum_{i in S} pi_i + u to F(S)
+// for non-empty S, u to every w(I(S)), plus pi_i at S = {i} and sum_i pi_i at
+// S = {}, the weight of the union of all requests.
 #include "mpt_internal.cuh"
 
 namespace mpt {
@@ -31,14 +32,15 @@ struct Gp64ToF {
 enum Offset { kNone, kPiOfS, kPiOfSingletons };
 
 // dst[(U << L) | T] = Op(src[(T << b) | U]) + offset(S) for T < 2^L, U < 2^b,
-// S = (U << L) | T: offset pi(S) (F), or pi_i at S = {i} and sum_i pi_i at
-// S = {} (w(I)), or none; priv null means pi = 0.
+// S = (U << L) | T: offset pi(S) + u for S non-empty (F), or u plus pi_i at
+// S = {i} and sum_i pi_i at S = {} (w(I)), or none; priv null means no
+// offsets.
 template <typename Src, typename Dst, typename Op, Offset Off>
 __global__ void __launch_bounds__(kTile * kRowsPerPass)
 k_unrotate(const Src* __restrict__ src, Dst* __restrict__ dst, int L, int b,
            const unsigned long long* __restrict__ priv, int m) {
   __shared__ Dst t[kTile][kTile + 1];
-  __shared__ long long piT[kTile], piU[kTile], pi_all;
+  __shared__ long long piT[kTile], piU[kTile], pi_all, univ;
   const size_t nT = (size_t)1 << L, nU = (size_t)1 << b;
   const size_t T0 = (size_t)blockIdx.x * kTile, U0 = (size_t)blockIdx.y * kTile;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -57,6 +59,7 @@ k_unrotate(const Src* __restrict__ src, Dst* __restrict__ dst, int L, int b,
       if (priv)
         for (int i = 0; i < m; ++i) v += (long long)priv[i];
       pi_all = v;
+      univ = priv ? (long long)priv[kUniversalSlot] : 0;
     }
   }
 #pragma unroll
@@ -70,10 +73,11 @@ k_unrotate(const Src* __restrict__ src, Dst* __restrict__ dst, int L, int b,
     const size_t U = U0 + ty + j, T = T0 + tx;
     if (T < nT && U < nU) {
       Dst v = t[tx][ty + j];
+      const uint32_t S = ((uint32_t)U << L) | (uint32_t)T;
       if (Off == kPiOfS) {
-        v += (Dst)(piT[tx] + piU[ty + j]);
+        if (S != 0) v += (Dst)(piT[tx] + piU[ty + j] + univ);
       } else if (Off == kPiOfSingletons) {
-        const uint32_t S = ((uint32_t)U << L) | (uint32_t)T;
+        v += (Dst)univ;
         if (S == 0)
           v += (Dst)pi_all;
         else if ((S & (S - 1)) == 0)

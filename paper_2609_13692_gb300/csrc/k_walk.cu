@@ -9,9 +9,9 @@
 // (depth of that node, chunk id).  The left-to-right leaf order is the trie
 // DFS order that Thm 7 (Sec. 8) serves requests in.  After a blocked solve
 // split is read at the rotated position of each node and OPT = F(full) =
-// F'(full) + sum_i pi_i from Gp = F' << b (uint32, or uint64 on the wide
-// path) and the private weights pi (k_scatter_zeta.cu); after a general one
-// both are in natural order.
+// F'(full) + sum_i pi_i + u from Gp = F' << b (uint32, or uint64 on the wide
+// path) and the offsets pi, u (k_scatter_zeta.cu); after a general one both
+// are in natural order.
 //
 // Trie cost: a string's node at depth p is new exactly when no earlier
 // string shares its first p+1 symbols, so the trie weight is
@@ -79,8 +79,10 @@ k_walk(int m, const uint32_t* __restrict__ split, const int64_t* __restrict__ F,
     }
     if (bad) atomicOr(&counters[1], kErrBadSplit);
     int64_t pi_all = 0;
-    if (priv)
+    if (priv) {
       for (int i = 0; i < m; ++i) pi_all += (int64_t)priv[i];
+      pi_all += (int64_t)priv[kUniversalSlot];
+    }
     *opt = Gp64 ? (int64_t)(Gp64[rot_index(full, L, b)] >> b) + pi_all
            : Gp ? (int64_t)(Gp[rot_index(full, L, b)] >> b) + pi_all
                 : (F ? F[full] : (int64_t)F32[full]);

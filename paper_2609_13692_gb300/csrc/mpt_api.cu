@@ -17,7 +17,7 @@ struct mpt_ctx {
   std::vector<int64_t> w;
   std::vector<uint64_t> bits;
   int64_t sum_w = 0;     // sum_i w(R_i)
-  int64_t shared_w = 0;  // the same less the chunks only one request needs
+  int64_t shared_w = 0;  // the same less the chunks one or every request needs
   int32_t mode = MPT_DP_AUTO;
   int32_t tables = MPT_TABLES_INT64;
   void* own_ws = nullptr;
@@ -136,7 +136,7 @@ size_t carve_workspace(const Shape& s, char* base, Workspace* ws) {
     ws->Gc = reinterpret_cast<uint32_t*>(take(N * 4));
     ws->partial = reinterpret_cast<unsigned long long*>(take((size_t)(s.partial_entries > 0 ? s.partial_entries : 1) * 8));
   }
-  ws->priv = s.blocked ? reinterpret_cast<unsigned long long*>(take(32 * 8)) : nullptr;
+  ws->priv = s.blocked ? reinterpret_cast<unsigned long long*>(take(mpt::kOffsetSlots * 8)) : nullptr;
   if (s.blocked) {
     // The rotated tables share the buffers of the natural ones: w(I) sits in
     // the F table (int64) or in fw (lean), split in the split table.  The
@@ -204,17 +204,21 @@ mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* 
       }
     }
   }
-  // weight of the chunks exactly one request needs: per word, the bits seen
-  // once (s1) but not twice (s2) over all requests
+  // request weight the packed keys leave out (k_scatter_zeta.cu): the chunks
+  // exactly one request needs (per word, the bits seen once, s1, but not
+  // twice, s2) and, for m >= 2, m times those that every request needs
   int64_t private_w = 0;
   for (int64_t j = 0; j < words; ++j) {
-    uint64_t s1 = 0, s2 = 0;
+    uint64_t s1 = 0, s2 = 0, all = ~0ull;
     for (int i = 0; i < m; ++i) {
       const uint64_t v = req_bits[(size_t)i * (size_t)words + (size_t)j];
       s2 |= s1 & v;
       s1 |= v;
+      all &= v;
     }
     for (uint64_t v = s1 & ~s2; v; v &= v - 1) private_w += weights[j * 64 + __builtin_ctzll(v)];
+    if (m >= 2)
+      for (uint64_t v = all; v; v &= v - 1) private_w += (int64_t)m * weights[j * 64 + __builtin_ctzll(v)];
   }
   mpt_ctx* c = new (std::nothrow) mpt_ctx();
   if (!c) return MPT_ERR_OUT_OF_MEMORY;
@@ -326,7 +330,7 @@ mpt_status run_front(mpt_ctx* c, const mpt::Workspace& ws, char* base, cudaStrea
     MPT_CK(cudaMemcpyAsync(ws.bits, c->bits.data(), c->bits.size() * 8, cudaMemcpyHostToDevice, stream), "copy bits");
   }
   MPT_CK(cudaMemsetAsync(ws.counters, 0, 8 * 4, stream), "memset counters");
-  if (ws.priv) MPT_CK(cudaMemsetAsync(ws.priv, 0, 32 * 8, stream), "memset private weights");
+  if (ws.priv) MPT_CK(cudaMemsetAsync(ws.priv, 0, mpt::kOffsetSlots * 8, stream), "memset offsets");
   MPT_CK(cudaMemsetAsync(mpt::g_table(s, ws), 0, N * (s.lean ? 4 : 8), stream), "memset g");
   mark(1);
   MPT_CK(mpt::launch_scatter(s, ws, stream, launches), "scatter kernel");

@@ -82,6 +82,9 @@ enum DeviceError : int {
 // ---------------------------------------------------------------------------
 // Workspace carve-up (all offsets 256-byte aligned).
 // ---------------------------------------------------------------------------
+constexpr int kOffsetSlots = 33;
+constexpr int kUniversalSlot = 32;
+
 struct Workspace {
   // inputs
   int64_t* weights;   // [n]
@@ -100,7 +103,7 @@ struct Workspace {
   uint32_t* split;    // [2^m]
   // blocked DP working tables, rotated order idx(S) = (T << b) | U with
   // T = S mod 2^L and U = S >> L (see k_dp_blocked.cu)
-  uint32_t* Gp;       // [2^m]  F' << b, F'(S) = F(S) - sum_{i in S} pi_i
+  uint32_t* Gp;       // [2^m]  F' << b, F'(S) = F(S) - sum_{i in S} pi_i - u
   uint32_t* Gc;       // [2^m]  (F' << b) | (~u & (2^b - 1))
   unsigned long long* partial;  // [max tiles of one layer << b]
   // wide blocked path (64-bit keys): Gp and Gc hold uint64 entries, and the
@@ -111,10 +114,12 @@ struct Workspace {
   int64_t* wI_rot;    // [2^m] w(I(S)) at idx(S) (int64 tables), or nullptr
   int32_t* fw_rot;    // [2^m] w(I(S)) at idx(S) (lean tables), or nullptr
   uint32_t* split_rot;  // [2^m] split[S] at idx(S)
-  // blocked paths: pi_i = w of the chunks that request i alone needs, which
-  // K1 adds here instead of to g; the rotated tables then hold w(I) and F
-  // less those weights (see scatter in k_scatter_zeta.cu)
-  unsigned long long* priv;  // [32] or nullptr
+  // blocked paths: slot i < 32 holds pi_i, the weight of the chunks that
+  // request i alone needs, and slot kUniversalSlot the weight u of the
+  // chunks that every request needs (m >= 2); K1 adds those chunks here
+  // instead of to g, and the rotated tables hold w(I) and F less them (see
+  // the scatter in k_scatter_zeta.cu)
+  unsigned long long* priv;  // [kOffsetSlots] or nullptr
   // layout
   unsigned long long* keys;  // [slots]
   int64_t* perm_offsets;     // [m + 1]
@@ -192,10 +197,10 @@ cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t str
 cudaError_t launch_walk(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches);
 
 // Natural-order tables from the blocked path's rotated ones (k_tables.cu):
-// split_nat[S] = split_rot[idx(S)]; wI_nat[S] = wI_rot[idx(S)] plus pi_i for
-// S = {i} and sum_i pi_i for S = {} (int64 tables); F_nat[S] or F32_nat[S] =
-// (Gp[idx(S)] >> b) + sum_{i in S} pi_i.  priv (pi, m entries on the device)
-// may be null: no private weights.  Null destinations are skipped; they run
+// split_nat[S] = split_rot[idx(S)]; wI_nat[S] = wI_rot[idx(S)] + u plus
+// pi_i for S = {i} and sum_i pi_i for S = {} (int64 tables); F_nat[S] or
+// F32_nat[S] = (Gp[idx(S)] >> b) + sum_{i in S} pi_i + u (S non-empty).
+// priv (the kOffsetSlots offsets on the device) may be null: no offsets.  Null destinations are skipped; they run
 // in this order, so a destination may be the source of an earlier conversion.
 cudaError_t unrotate_tables(const Shape& s, const uint32_t* split_rot, uint32_t* split_nat, const int64_t* wI_rot,
                             int64_t* wI_nat, const uint32_t* Gp, int64_t* F_nat, int32_t* F32_nat,

@@ -39,9 +39,9 @@ constexpr size_t kOffGp = align_up(kOffUsedX + kNoAllocMaxSlots * sizeof(int32_t
 constexpr size_t kOffGc = align_up(kOffGp + (sizeof(uint32_t) << kNoAllocMaxM));
 constexpr size_t kOffPartial = align_up(kOffGc + (sizeof(uint32_t) << kNoAllocMaxM));
 constexpr size_t kOffCheck = align_up(kOffPartial + max_partial_entries() * sizeof(unsigned long long));
-constexpr int kChecks = 6;
+constexpr int kChecks = 8;
 constexpr size_t kOffPriv = align_up(kOffCheck + kChecks * sizeof(unsigned long long));
-constexpr size_t kScratchBytes = align_up(kOffPriv + 32 * sizeof(unsigned long long));
+constexpr size_t kScratchBytes = align_up(kOffPriv + mpt::kOffsetSlots * sizeof(unsigned long long));
 
 // The scratch: about 10.7 MiB per device.  In host code `g_noalloc_scratch`
 // is only a host-side stand-in for the symbol; kernels receive the device
@@ -72,14 +72,16 @@ cudaError_t scratch_for_current_device(char** out) {
 
 // Argument checks that need the device-resident inputs: every weight >= 1,
 // no request bit at a chunk >= n, the number of chunk occurrences,
-// sum_i w(R_i), and the weight of the chunks that one request alone needs
-// (left out of the blocked recurrence's keys, see k_scatter_zeta.cu).  Each
+// sum_i w(R_i), and the request weight of the chunks that one request alone
+// or (m >= 2) every request needs (left out of the blocked recurrence's keys,
+// see k_scatter_zeta.cu).  Each
 // term w(x) * |S_x| is capped at 2^62 (beyond which the instance is rejected
 // anyway) and added as two 32-bit halves into separate 64-bit counters, which
 // cannot wrap for n < 2^31.
 //   check[0] = bad weight or stray bit, check[1] = occurrences,
 //   check[2] / check[3] = sums of the low / high halves of the terms,
-//   check[4] / check[5] = the same for the private chunks' terms
+//   check[4] / check[5] = the same for the private chunks' terms,
+//   check[6] / check[7] = the same for the universal chunks' terms
 __global__ void k_noalloc_check(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int64_t n, int m,
                                 int64_t words, unsigned long long* __restrict__ check) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -107,6 +109,9 @@ __global__ void k_noalloc_check(const int64_t* __restrict__ w, const uint64_t* _
       if (cnt == 1) {
         atomicAdd(&check[4], term & 0xFFFFFFFFull);
         atomicAdd(&check[5], term >> 32);
+      } else if (cnt == m) {
+        atomicAdd(&check[6], term & 0xFFFFFFFFull);
+        atomicAdd(&check[7], term >> 32);
       }
     }
   }
@@ -134,7 +139,7 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
     k_noalloc_check<<<(unsigned)blocks, 256, 0, stream>>>(d_weights, d_req_bits, n_chunks, m, words, check);
     if (cudaGetLastError() != cudaSuccess) return MPT_ERR_CUDA;
   }
-  unsigned long long h_check[kChecks] = {0, 0, 0, 0, 0, 0};
+  unsigned long long h_check[kChecks] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (cudaMemcpyAsync(h_check, check, sizeof(h_check), cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
       cudaStreamSynchronize(stream) != cudaSuccess)
     return MPT_ERR_CUDA;
@@ -142,7 +147,8 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   if (h_check[1] > (unsigned long long)kNoAllocMaxSlots) return MPT_ERR_TOO_LARGE;
   const unsigned __int128 sum_w = ((unsigned __int128)h_check[3] << 32) + h_check[2];
   if (sum_w >= ((unsigned __int128)1 << 62)) return MPT_ERR_OVERFLOW;
-  const unsigned __int128 private_w = ((unsigned __int128)h_check[5] << 32) + h_check[4];
+  const unsigned __int128 private_w = ((unsigned __int128)h_check[5] << 32) + h_check[4] +
+                                      ((unsigned __int128)h_check[7] << 32) + h_check[6];
 
   mpt::Shape s{};
   s.m = m;
@@ -180,7 +186,8 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   int launches = 0;
   if (cudaMemsetAsync(ws.counters, 0, 8 * sizeof(int32_t), stream) != cudaSuccess ||
       cudaMemsetAsync(mpt::g_table(s, ws), 0, sizeof(int64_t) << m, stream) != cudaSuccess ||
-      (ws.priv && cudaMemsetAsync(ws.priv, 0, 32 * sizeof(unsigned long long), stream) != cudaSuccess))
+      (ws.priv && cudaMemsetAsync(ws.priv, 0, mpt::kOffsetSlots * sizeof(unsigned long long), stream) !=
+                      cudaSuccess))
     return MPT_ERR_CUDA;
   if (mpt::launch_scatter(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;
   if (mpt::launch_zeta(s, ws, stream, &launches) != cudaSuccess) return MPT_ERR_CUDA;

@@ -41,6 +41,7 @@ __all__ = [
     "CONFIGS",
     "random_instance",
     "with_query_chunks",
+    "with_common_prefix",
     "k4_3",
     "open_problem_k4",
     "tightness_witness",
@@ -268,6 +269,14 @@ def with_query_chunks(inst: Instance, wmin: int, wmax: int, seed: int, every: in
         reqs[i] = list(reqs[i]) + [inst.n + j]
     weights = np.concatenate([inst.weights, extra])
     return Instance(weights, pack_requests(reqs, n), f"{inst.name} + query chunks [{wmin}, {wmax}]")
+
+
+def with_common_prefix(inst: Instance, weight: int) -> Instance:
+    """``inst`` with one new chunk of the given weight in every request: a
+    system prompt or tool catalogue that all requests share."""
+    reqs = [list(r) + [inst.n] for r in inst.requests()]
+    weights = np.concatenate([inst.weights, np.array([weight], dtype=np.int64)])
+    return Instance(weights, pack_requests(reqs, inst.n + 1), f"{inst.name} + common prefix {weight}")
 
 
 def k4_3() -> Instance:

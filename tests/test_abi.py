@@ -306,9 +306,10 @@ def test_caller_workspace_checks(mpt):
 
 
 def test_key_width_follows_shared_weight(mpt):
-    """The packed-key limits apply to the shared weight: private suffixes of
-    2^40 tokens keep the 32-bit keys (BLOCKED accepted, the narrow
-    workspace); a shared chunk of 2^20 tokens does not."""
+    """The packed-key limits apply to the shared weight: private suffixes and
+    a common prefix of 2^40 tokens keep the 32-bit keys (BLOCKED accepted,
+    the narrow workspace); a chunk of 2^20 tokens that some but not all
+    requests share does not."""
     base = I.config(1)  # m = 12
     heavy_private = I.with_query_chunks(base, 1 << 40, 1 << 40, seed=1)
     narrow = mpt.mpt_create(base.weights, base.bits)
@@ -318,6 +319,10 @@ def test_key_width_follows_shared_weight(mpt):
     with pytest.raises(mpt.MPTError) as e:
         mpt.mpt_set_tables(ctx, "lean")  # the int32 tables still need sum_i w(R_i) < 2^31
     assert e.value.status == 3
+    prefix = I.with_common_prefix(heavy_private, 1 << 40)  # plus 2^40 tokens in every request
+    ctx_p = mpt.mpt_create(prefix.weights, prefix.bits)
+    mpt.mpt_set_dp_mode(ctx_p, "blocked")
+    mpt.mpt_destroy(ctx_p)
     shared = I.Instance(base.weights.copy(), base.bits)
     x = int(np.flatnonzero(np.unpackbits(base.bits[0].view(np.uint8), bitorder="little"))[0])
     assert W.request_counts(base)[x] >= 2

@@ -131,3 +131,26 @@ def test_private_chunks_shift_F_by_a_constant():
     extra = int(inst.weights[base.n:].sum())
     assert O.brute_force_permutations(inst.weights, inst.bits) == O.brute_force_permutations(base.weights,
                                                                                             base.bits) + extra
+
+
+def test_universal_chunks_shift_F_by_a_constant():
+    """Thm 1: a chunk that all m >= 2 requests hold has the root as its one
+    maximal cluster in every hierarchy, so it adds its weight u to F(S) for
+    every non-empty S and to every w(I(S)), and changes no split."""
+    rng = np.random.default_rng(321)
+    for t in range(8):
+        m = int(rng.integers(2, 11))
+        base = I.random_instance(m, 30, (0, 7), seed=int(rng.integers(1 << 30)), wmin=1, wmax=50, allow_empty=True)
+        u = int(rng.integers(1, 10 ** 6))
+        inst = I.with_common_prefix(base, u)
+        opt0, F0, wI0, s0 = O.solve(base.weights, base.bits)
+        opt1, F1, wI1, s1 = O.solve(inst.weights, inst.bits)
+        nonempty = (np.arange(1 << m) != 0).astype(np.int64)
+        assert np.array_equal(F1, F0 + u * nonempty)
+        assert np.array_equal(wI1, wI0 + u)
+        assert np.array_equal(s1, s0)
+        assert opt1 == opt0 + u
+    base = I.Instance(np.array([2, 3, 1, 4], dtype=np.int64), I.pack_requests([[0, 1], [1, 2], [0, 2, 3]], 4))
+    inst = I.with_common_prefix(base, 7)
+    assert O.brute_force_permutations(inst.weights, inst.bits) == O.brute_force_permutations(base.weights,
+                                                                                            base.bits) + 7

@@ -1,11 +1,12 @@
-"""Heavy private chunks on the tiled kernels, through the C ABI.
+"""Heavy private and universal chunks on the tiled kernels, through the C ABI.
 
-A chunk that one request alone holds is one maximal cluster of its request
-set in every hierarchy (Thm 1: t_x(H) = 1), so it adds its weight to F(S) for
-every S holding that request and never changes a split.  The tiled kernels
-therefore run the recurrence without those weights and add them back; their
-key width depends only on the shared weight.  Here every request gets a
-suffix of its own (a question or a document) weighing up to 2^40 tokens,
+A chunk that one request alone holds, or that every request holds, is one
+maximal cluster of its request set in every hierarchy (Thm 1: t_x(H) = 1),
+so it adds its weight to F(S) for every S holding its requests and never
+changes a split.  The tiled kernels therefore run the recurrence without
+those weights and add them back; their key width depends only on the shared
+weight.  Here requests get a suffix of their own (a question or a document)
+of up to 2^40 tokens and a common prefix (a system prompt) of up to 2^34,
 which keeps sum_i w(R_i) far beyond the 32-bit keys while the shared weight
 stays below 2^20: AUTO must still take the 32-bit keys, and every table must
 equal the oracle's bit for bit."""
@@ -73,6 +74,20 @@ def test_query_chunks_sweep(mpt, m):
     _parity(mpt, inst)
 
 
+@pytest.mark.parametrize("m", [1, 2, 3, 5, 8, 11, 13, 16, 18])
+def test_common_prefix_sweep(mpt, m):
+    """A common prefix of 2^34 tokens in every request, with and without
+    private suffixes: the 32-bit keys, every table bit-exact."""
+    rng = np.random.default_rng(8000 + m)
+    n = int(rng.integers(8, 90))
+    base = I.random_instance(m, n, (0, min(n, 10)), seed=int(rng.integers(1 << 30)), wmin=1, wmax=400,
+                             allow_empty=True)
+    inst = I.with_common_prefix(base, 1 << 34)
+    assert W.shared_weight(inst) < 1 << 20
+    _parity(mpt, inst)
+    _parity(mpt, _with_queries(inst, seed=m, every=2))
+
+
 def test_query_chunks_paper_examples(mpt):
     """The paper's examples and the edge cases with heavy private suffixes:
     one request, empty requests, identical requests, all-private requests."""
@@ -124,6 +139,7 @@ def test_shared_weight_limit(mpt):
     assert W.shared_weight(inst) == 2 ** 20 - 1
     _parity(mpt, inst, expect_mode=1)
     _parity(mpt, inst, mode="blocked", expect_mode=1)
+    _parity(mpt, I.with_common_prefix(inst, 1 << 34), expect_mode=1)
     heavier = I.Instance(inst.weights.copy(), inst.bits)
     heavier.weights[m] += 1  # chunk m is shared: the shared weight reaches 2^20 + 2
     assert W.shared_weight(heavier) >= 1 << 20
@@ -211,5 +227,37 @@ def test_query_chunks_rag_workloads(mpt, workload):
     pa, pb = a.permutations(), b.permutations()
     for i in range(m):
         assert pb[i] == pa[i] + [base.n + i]  # the suffix is emitted last, at the leaf
+    assert b.dfs_order.tolist() == a.dfs_order.tolist()
+    assert mpt.mpt_trie_cost(inst.weights, b.perm_offsets, b.perm_chunks) == b.opt
+
+
+def test_common_prefix_rag_workload(mpt):
+    """The m = 28 workload behind a common prefix of 2^30 tokens and with
+    private suffixes: F shifts by sum_{i in S} pi_i + u for non-empty S, every
+    w(I(S)) by u, the splits stay and every permutation starts with the
+    prefix, all on the 32-bit keys."""
+    import torch
+
+    base = I.config(4)
+    u = 1 << 30
+    inst = _with_queries(I.with_common_prefix(base, u), seed=11, wmin=1 << 26, wmax=1 << 30)
+    assert W.shared_weight(inst) == W.shared_weight(base) and W.universal_weight(inst) == u
+    a = mpt.solve(base.weights, base.bits)
+    b = mpt.solve(inst.weights, inst.bits, profile=True)
+    assert mpt.mpt_get_profile(b.ctx)["dp_mode"] == 1
+    m = base.m
+    q = inst.weights[base.n + 1:]  # request i's suffix is chunk base.n + 1 + i
+    assert b.opt == a.opt + u + int(q.sum())
+    Fa, wIa, sa = mpt.mpt_tables(a.ctx)
+    Fb, wIb, sb = mpt.mpt_tables(b.ctx)
+    assert torch.equal(sa, sb)
+    nonempty = (torch.arange(1 << m, device="cuda") != 0).to(torch.int64)
+    assert torch.equal(Fb, Fa + _pi_of_subsets(m, q) + u * nonempty)
+    expect = wIa + u
+    expect[torch.tensor([1 << i for i in range(m)], device="cuda")] += torch.from_numpy(q.copy()).cuda()
+    expect[0] += int(q.sum())
+    assert torch.equal(wIb, expect)
+    for i, (pa, pb) in enumerate(zip(a.permutations(), b.permutations())):
+        assert pb == [base.n] + pa + [base.n + 1 + i]
     assert b.dfs_order.tolist() == a.dfs_order.tolist()
     assert mpt.mpt_trie_cost(inst.weights, b.perm_offsets, b.perm_chunks) == b.opt

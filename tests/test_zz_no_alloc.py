@@ -61,6 +61,7 @@ def test_noalloc_matches_solve_on_consecutive_calls(mpt):
         I.config(1),                                                         # m = 12, one tile
         I.with_query_chunks(I.config(2), 1 << 30, 1 << 38, seed=2),          # private suffixes, blocked kernels
         I.with_query_chunks(I.rag_pools(16, 5000, 4, 60, 8, 1.1, seed=11), 1 << 30, 1 << 38, seed=3),
+        I.with_common_prefix(I.with_query_chunks(I.config(1), 1 << 30, 1 << 38, seed=4), 1 << 36),
     ]
     for inst in cases:
         ref = _reference(mpt, inst)

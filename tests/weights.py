@@ -1,6 +1,7 @@
 """Weight totals of an instance that decide which key width the tiled
 kernels use: sum_i w(R_i), and the shared weight, the same sum less the
-chunks that exactly one request needs."""
+chunks that exactly one request needs and (for m >= 2) those that every
+request needs."""
 
 from __future__ import annotations
 
@@ -19,7 +20,15 @@ def request_weight_sum(inst) -> int:
 
 
 def shared_weight(inst) -> int:
-    return int(sum(int(w) * int(c) for w, c in zip(inst.weights, request_counts(inst)) if c >= 2))
+    m = inst.m
+    return int(sum(int(w) * int(c) for w, c in zip(inst.weights, request_counts(inst)) if 2 <= c < m))
+
+
+def universal_weight(inst) -> int:
+    """u: the weight of the chunks that every one of m >= 2 requests holds."""
+    if inst.m < 2:
+        return 0
+    return int(sum(int(w) for w, c in zip(inst.weights, request_counts(inst)) if c == inst.m))
 
 
 def private_weights(inst) -> list[int]:
