@@ -22,9 +22,11 @@
 // For T = 0 the tile kernel runs the recurrence on the b inner bits alone.
 // Tiles with |T| = k depend only on tiles with |T| < k: one launch pair per k.
 //
-// Packed keys.  With sum_i w(R_i) < 2^(32-b) every candidate F(A) + F(B) fits
-// in 32 - b bits, so the working tables hold G = F << b and the key of a
-// candidate is
+// Packed keys.  The tables hold F less the weight of the chunks that one or
+// every request needs (F' of k_scatter_zeta.cu; written F below).  With the
+// shared weight sum_i w(R_i) - sum_i pi_i - m u below 2^(32-b) every
+// candidate F(A) + F(B) fits in 32 - b bits, so the working tables hold
+// G = F << b and the key of a candidate is
 //     key = Gp[A] + Gc[B] = ((F(A) + F(B)) << b) | (2^b - 1 - U + Ua),
 // Gp = F << b and Gc = (F << b) | (~u & (2^b - 1)) (u = the entry's U part).
 // An unsigned min over keys picks the least value and, among equal values,

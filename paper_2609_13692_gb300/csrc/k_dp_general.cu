@@ -7,7 +7,7 @@
 // This form reads F(A) and F(S \ A) straight from the 2^m table in HBM/L2 for
 // every split (16 bytes per split), so it is bound by random gathers.  It is
 // exact for any weights below the int64 limit and is used when the blocked
-// kernels' 32-bit packed keys could overflow (sum_i w(R_i) >= 2^20), or on
+// kernels' packed keys could overflow (shared weight >= 2^51), or on
 // request.  T is the table type: int64 (separate w(I) and F tables), or int32
 // for the lean table, where wI and F are the same array -- the thread that
 // finishes S reads w(I(S)) and writes F(S) over it, and F is read only at

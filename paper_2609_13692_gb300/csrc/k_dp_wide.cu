@@ -3,7 +3,8 @@
 // with the tiling of k_dp_blocked.cu (rotated tables, tile T and inner U,
 // proper pairs per window pair, the self pair inside the tile) and 64-bit
 // packed keys, for instances whose candidate sums do not fit the 32-bit keys
-// (sum_i w(R_i) >= 2^(32-b)) but stay below 2^51:
+// (shared weight sum_i w(R_i) - sum_i pi_i - m u >= 2^(32-b), F and w(I) less
+// the offsets of k_scatter_zeta.cu) but stay below 2^51:
 //     key = Gp[A] + Gc[B] = ((F(A) + F(B)) << b) | (2^b - 1 - U + Ua),
 // Gp = F << b and Gc = Gp | (~u & (2^b - 1)) as uint64.  The candidates and
 // the tie order (value, Ua, Ta) are those of the 32-bit path, so the argmin is
