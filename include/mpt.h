@@ -233,7 +233,9 @@ typedef struct mpt_batch mpt_batch;
  *   chunk_ids: int64[req_offsets[last]] in [0, n_chunks), no repeat inside a
  *   request.
  * Limits per instance: 1 <= m <= 13 and at most 2048 chunk occurrences
- * (MPT_ERR_TOO_LARGE beyond), sum_i w(R_i) < 2^31 (MPT_ERR_OVERFLOW).
+ * (MPT_ERR_TOO_LARGE beyond); sum_i w(R_i) < 2^62 and a shared weight
+ * (sum_i w(R_i) less the chunks that one request alone or all m >= 2
+ * requests hold, see MPT_DP_AUTO) below 2^31 (MPT_ERR_OVERFLOW).
  * Errors: INVALID_ARG, TOO_LARGE, OVERFLOW, OUT_OF_MEMORY.  No CUDA call. */
 mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t batch, const int64_t* inst_requests,
                             const int64_t* req_offsets, const int64_t* chunk_ids, mpt_batch** out);

@@ -18,9 +18,17 @@
 //   4. the hierarchy walk of the Thm 1 proof: request i's chunks ordered by
 //      (depth of the highest node on its path inside N_x, chunk id), and the
 //      left-to-right leaf order (Thm 7).
-// Values are kept in 32 bits: the host accepts an instance only when
-// sum_i w(R_i) < 2^31, so every F and every split sum fits.  When also
-// sum_i w(R_i) < 2^(32-m) (the common case), the F table holds F << m and the
+// Offsets: a chunk that one request alone holds, or that all m >= 2 hold, is
+// one cluster in every hierarchy (Thm 1), so for instances whose
+// sum_i w(R_i) would not fit the packed keys (flag kFlagOffsets) step 2 adds
+// it to a per-request sum pi_i or a universal sum u instead of to g, step 3
+// runs on F'(S) = F(S) - sum_{i in S} pi_i - u, and the outputs add those
+// back (the same reduction as the single-instance scatter,
+// k_scatter_zeta.cu).  Lighter instances keep the plain form (F' = F).
+// Values are kept in 32 bits: the host accepts an instance only when its
+// shared weight W = sum_i w(R_i) - sum_i pi_i - m u is below 2^31, so every
+// F' and every split sum fits.  When also W < 2^(32-m) (the common case),
+// the F table holds F' << m and the
 // key of split A is F[A] + F[S \ A] + A = ((F(A) + F(S \ A)) << m) + A: one
 // 32-bit minimum picks the least value and, among equal values, the least A.
 // Otherwise keys are (value << 16 | A) in 64 bits.
@@ -32,6 +40,40 @@ namespace mpt {
 namespace {
 
 constexpr int kBatchThreads = 256;
+constexpr int kBatchOffsets = 17;  // pi_i in slots 0..12, u in slot kBatchUniv
+constexpr int kBatchUniv = 16;
+
+// Step 2's scatter: chunk u of the instance goes to pi_i (N_x = {i}), to u
+// (N_x = all m >= 2 requests) or to g(N_x), the last through g_at(N_x); with
+// off null, every chunk goes to g.
+template <int TPI, typename GAt>
+__device__ void batch_scatter(int m, int nd, const int64_t* __restrict__ weights, const int32_t* cx,
+                              const uint32_t* cN, unsigned long long* off, GAt g_at) {
+  for (int u = threadIdx.x; u < nd; u += TPI) {
+    const uint32_t Nx = cN[u];
+    const unsigned long long wx = (unsigned long long)weights[cx[u]];
+    if (off && (Nx & (Nx - 1)) == 0)
+      atomicAdd(&off[__ffs(Nx) - 1], wx);
+    else if (off && __popc(Nx) == m)  // all m requests (written this way, ptxas keeps k_batch_rows spill-free)
+      atomicAdd(&off[kBatchUniv], wx);
+    else
+      atomicAdd(g_at(Nx), (uint32_t)wx);
+  }
+}
+
+// What step 3 left out of F(S): sum_{i in S} pi_i + u for S non-empty.  A
+// thread writes the entries S = t, t + TPI, t + 2 TPI, ..., so the requests
+// below TPI are its own (summed once, lo) and only the others are summed per
+// entry.
+__device__ __forceinline__ int64_t batch_pi(uint32_t S, const unsigned long long* off) {
+  int64_t v = 0;
+  for (uint32_t r = S; r; r &= r - 1) v += (int64_t)off[__ffs(r) - 1];
+  return v;
+}
+template <int TPI>
+__device__ __forceinline__ int64_t batch_offset(uint32_t S, int64_t lo, const long long* hi) {
+  return S == 0 ? 0 : lo + hi[S / TPI];
+}
 
 
 // Step 1: the instance's distinct chunks cx[0..nd) (in no particular order)
@@ -168,12 +210,13 @@ __global__ void __launch_bounds__(kBatchThreads)
 k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
               const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
               const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list,
-              const uint8_t* __restrict__ packed_ok, int occ_cap, int max_m, int64_t* __restrict__ opt_out,
+              const uint8_t* __restrict__ flags, int occ_cap, int max_m, int64_t* __restrict__ opt_out,
               int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out, int64_t* __restrict__ perm_out,
               int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int inst = inst_list[blockIdx.x];
-  const bool packed = packed_ok[inst] != 0;
+  const bool packed = (flags[inst] & kFlagPacked) != 0;
+  const bool use_off = (flags[inst] & kFlagOffsets) != 0;
   const int64_t r0 = inst_req[inst], r1 = inst_req[inst + 1];
   const int m = (int)(r1 - r0);
   const int64_t o0 = req_off[r0], o1 = req_off[r1];
@@ -190,14 +233,17 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   uint32_t* tmask = cN + occ_cap;                                                // [2 * occ_cap] hash-table masks
   __shared__ int ndistinct;
   __shared__ int roff[16];  // request offsets relative to o0
+  __shared__ unsigned long long off[kBatchOffsets];
   const int t = threadIdx.x;
   const int nd = batch_gather<kBatchThreads>(m, r0, o0, occ, occ_cap, req_off, chunks,
                                              reinterpret_cast<int32_t*>(keys), tmask, cx, cN, roff, &ndistinct);
   for (int S = t; S < N; S += kBatchThreads) wI[S] = 0;
+  if (t < kBatchOffsets) off[t] = 0;
   __syncthreads();
 
-  // 2. g(T), then superset sums over the m request bits
-  for (int u = t; u < nd; u += kBatchThreads) atomicAdd(&wI[cN[u]], (uint32_t)weights[cx[u]]);
+  // 2. g(T) and the offsets, then superset sums over the m request bits
+  batch_scatter<kBatchThreads>(m, nd, weights, cx, cN, use_off ? off : nullptr,
+                               [&](uint32_t Nx) { return &wI[Nx]; });
   __syncthreads();
   for (int j = 0; j < m; ++j) {
     for (int p = t; p < (N >> 1); p += kBatchThreads) {
@@ -308,11 +354,24 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 
   // outputs: tables and OPT
   const int64_t tb = tab_off[inst];
-  for (int S = t; S < N; S += kBatchThreads) {
-    F_out[tb + S] = (int64_t)(F[S] >> vshift);
-    split_out[tb + S] = split[S];
+  if (use_off) {
+    __shared__ long long hi_off[32];
+    if (t < 32) hi_off[t] = batch_pi((uint32_t)t * kBatchThreads, off) + (long long)off[kBatchUniv];
+    __syncthreads();
+    const int64_t lo = batch_pi((uint32_t)t & (kBatchThreads - 1), off);
+    for (int S = t; S < N; S += kBatchThreads) {
+      F_out[tb + S] = (int64_t)(F[S] >> vshift) + batch_offset<kBatchThreads>((uint32_t)S, lo, hi_off);
+      split_out[tb + S] = split[S];
+    }
+    if (t == 0)
+      opt_out[inst] = (int64_t)(F[N - 1] >> vshift) + batch_pi((uint32_t)N - 1u, off) + (int64_t)off[kBatchUniv];
+  } else {
+    for (int S = t; S < N; S += kBatchThreads) {
+      F_out[tb + S] = (int64_t)(F[S] >> vshift);
+      split_out[tb + S] = split[S];
+    }
+    if (t == 0) opt_out[inst] = (int64_t)(F[N - 1] >> vshift);
   }
-  if (t == 0) opt_out[inst] = (int64_t)(F[N - 1] >> vshift);
 
   // 4. hierarchy walk
   __syncthreads();
@@ -418,9 +477,10 @@ template <int TPI>
 __global__ void __launch_bounds__(TPI, TPI >= 256 ? 3 : (TPI == 128 ? 6 : 12))  // 12 warps or more per SM
 k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
              const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
-             const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list, int occ_cap, int mm,
-             int64_t* __restrict__ opt_out, int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out,
-             int64_t* __restrict__ perm_out, int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
+             const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list,
+             const uint8_t* __restrict__ flags, int occ_cap, int mm, int64_t* __restrict__ opt_out,
+             int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out, int64_t* __restrict__ perm_out,
+             int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int inst = inst_list[blockIdx.x];
   const int64_t r0 = inst_req[inst], r1 = inst_req[inst + 1];
@@ -447,14 +507,17 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   const int t = threadIdx.x;
 
   __shared__ int roff[16];  // request offsets relative to o0
+  __shared__ unsigned long long off[kBatchOffsets];
   const int nd = batch_gather<TPI>(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask,
                                    cx, cN, roff, &ndistinct);
 
-  // g and the superset sums, in the padded row layout: the five in-row bits
-  // per row in registers, then one row-pair pass per row bit
+  // g, the offsets and the superset sums, in the padded row layout: the five
+  // in-row bits per row in registers, then one row-pair pass per row bit
   for (int i = t; i < R * kBRowStride; i += TPI) Gp[i] = 0;
+  if (t < kBatchOffsets) off[t] = 0;
   __syncthreads();
-  for (int u = t; u < nd; u += TPI) atomicAdd(&Gp[bidx(cN[u])], (uint32_t)weights[cx[u]]);
+  const bool use_off = (flags[inst] & kFlagOffsets) != 0;
+  batch_scatter<TPI>(m, nd, weights, cx, cN, use_off ? off : nullptr, [&](uint32_t Nx) { return &Gp[bidx(Nx)]; });
   __syncthreads();
   for (int r = t; r < R; r += TPI) {
     uint32_t v[kBRow];
@@ -614,11 +677,23 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   }
 
   // outputs: tables and OPT
-  for (int U = t; U < N; U += TPI) {
-    F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m);
-    split_out[tb + U] = split[U];
+  if (use_off) {
+    __shared__ long long hi_off[32];
+    if (t < 32) hi_off[t] = batch_pi((uint32_t)t * TPI, off) + (long long)off[kBatchUniv];
+    __syncthreads();
+    const int64_t lo = batch_pi((uint32_t)t & (TPI - 1), off);
+    for (int U = t; U < N; U += TPI) {
+      F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m) + batch_offset<TPI>((uint32_t)U, lo, hi_off);
+      split_out[tb + U] = split[U];
+    }
+    if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m) + batch_pi(mask, off) + (int64_t)off[kBatchUniv];
+  } else {
+    for (int U = t; U < N; U += TPI) {
+      F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m);
+      split_out[tb + U] = split[U];
+    }
+    if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   }
-  if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   __syncthreads();
   batch_walk<TPI>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
@@ -633,13 +708,13 @@ size_t batch_smem_bytes(int max_m, int occ_cap) {
 // One grid over `count` instances of size m (ids inst_list[0..count)).
 cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                          const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
-                         const int32_t* inst_list, const uint8_t* packed_ok, int64_t* opt, int64_t* F,
+                         const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
                          uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream) {
   const size_t smem = batch_smem_bytes(m, occ_cap);
   cudaError_t e = cudaFuncSetAttribute(k_batch_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_batch_solve<<<(unsigned)count, kBatchThreads, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off,
-                                                                  inst_list, packed_ok, occ_cap, m, opt, F, split,
+                                                                  inst_list, flags, occ_cap, m, opt, F, split,
                                                                   perm, dfs, status);
   return cudaGetLastError();
 }
@@ -654,8 +729,8 @@ size_t batch_rows_smem_bytes(int m, int occ_cap) {
 // whose request weights allow packed keys.
 cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                               const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
-                              const int32_t* inst_list, int64_t* opt, int64_t* F, uint32_t* split, int64_t* perm,
-                              int32_t* dfs, int32_t* status, cudaStream_t stream) {
+                              const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
+                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream) {
   if (m < 6 || m > 13) return cudaErrorInvalidValue;
   const size_t smem = batch_rows_smem_bytes(m, occ_cap);
   const int tpi = batch_rows_threads(m);
@@ -663,8 +738,8 @@ cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weig
   auto go = [&](auto kernel) {
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess)
-      kernel<<<(unsigned)count, tpi, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off, inst_list, occ_cap, m,
-                                                      opt, F, split, perm, dfs, status);
+      kernel<<<(unsigned)count, tpi, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off, inst_list, flags,
+                                                      occ_cap, m, opt, F, split, perm, dfs, status);
   };
   if (tpi == 64)
     go(k_batch_rows<64>);

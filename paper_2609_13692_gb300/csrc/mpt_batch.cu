@@ -15,12 +15,12 @@ namespace mpt {
 size_t batch_smem_bytes(int max_m, int occ_cap);
 cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                          const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
-                         const int32_t* inst_list, const uint8_t* packed_ok, int64_t* opt, int64_t* F,
+                         const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
                          uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream);
 cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                               const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
-                              const int32_t* inst_list, int64_t* opt, int64_t* F, uint32_t* split, int64_t* perm,
-                              int32_t* dfs, int32_t* status, cudaStream_t stream);
+                              const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
+                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream);
 }  // namespace mpt
 
 struct mpt_batch {
@@ -34,7 +34,10 @@ struct mpt_batch {
   std::vector<int32_t> inst_list;
   std::vector<int64_t> group_start, group_rows_end;
   std::vector<int> group_occ_cap;
-  std::vector<uint8_t> packed_ok;  // sum_i w(R_i) < 2^(32 - m): 32-bit keys
+  // per instance: kFlagPacked when the shared weight is below 2^(32 - m)
+  // (32-bit keys), kFlagOffsets when sum_i w(R_i) is not (private and
+  // universal chunks kept out of the kernels' values, k_batch.cu)
+  std::vector<uint8_t> flags;
   // results of the last solve
   bool solved = false;
   std::vector<int64_t> opt, perm;
@@ -49,12 +52,13 @@ namespace {
 
 constexpr int kBatchMaxM = 13;
 constexpr int kBatchMaxOcc = 2048;
+constexpr int64_t kBatchSumLimit = (int64_t)1 << 62;
 
 struct BatchCarve {
   int64_t *weights, *inst_req, *req_off, *chunks, *tab_off, *opt, *F, *perm;
   uint32_t* split;
   int32_t *dfs, *status, *inst_list;
-  uint8_t* packed_ok;
+  uint8_t* flags;
 };
 
 size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
@@ -76,7 +80,7 @@ size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
   c->dfs = reinterpret_cast<int32_t*>(take((size_t)b->requests * 4));
   c->status = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
   c->inst_list = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
-  c->packed_ok = reinterpret_cast<uint8_t*>(take((size_t)b->batch));
+  c->flags = reinterpret_cast<uint8_t*>(take((size_t)b->batch));
   return off;
 }
 
@@ -106,7 +110,7 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
   if (!c) return MPT_ERR_OUT_OF_MEMORY;
   try {
     c->tab_off.resize((size_t)batch + 1);
-    c->packed_ok.assign((size_t)batch, 0);
+    c->flags.assign((size_t)batch, 0);
     std::vector<int> inst_occ((size_t)batch);
     int64_t tab = 0;
     std::vector<int64_t> ids;
@@ -118,7 +122,6 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
         delete c;
         return MPT_ERR_TOO_LARGE;
       }
-      int64_t sum = 0;
       for (int64_t r = r0; r < r1; ++r) {
         ids.assign(chunk_ids + req_offsets[r], chunk_ids + req_offsets[r + 1]);
         std::sort(ids.begin(), ids.end());
@@ -127,18 +130,38 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
             delete c;
             return MPT_ERR_INVALID_ARG;
           }
-          sum += weights[ids[j]];
-          if (sum >= ((int64_t)1 << 31)) {
+        }
+      }
+      // sum_i w(R_i) (below 2^62) and the shared weight W (below 2^31): the
+      // request weight less the chunks that one or all m >= 2 requests hold,
+      // which the kernels keep out of their 32-bit values (k_batch.cu)
+      ids.assign(chunk_ids + req_offsets[r0], chunk_ids + req_offsets[r1]);
+      std::sort(ids.begin(), ids.end());
+      int64_t sum = 0, shared = 0;
+      for (size_t j = 0; j < ids.size();) {
+        size_t k = j;
+        while (k < ids.size() && ids[k] == ids[j]) ++k;
+        const int64_t cnt = (int64_t)(k - j), wx = weights[ids[j]];
+        if (wx > (kBatchSumLimit - 1 - sum) / cnt) {
+          delete c;
+          return MPT_ERR_OVERFLOW;
+        }
+        sum += cnt * wx;
+        if (cnt >= 2 && cnt < m) {
+          shared += cnt * wx;
+          if (shared >= ((int64_t)1 << 31)) {
             delete c;
             return MPT_ERR_OVERFLOW;
           }
         }
+        j = k;
       }
       c->tab_off[(size_t)b] = tab;
       tab += (int64_t)1 << m;
       c->max_m = std::max(c->max_m, m);
       while (c->occ_cap < occ) c->occ_cap <<= 1;
-      c->packed_ok[(size_t)b] = sum < ((int64_t)1 << (32 - m)) ? 1 : 0;
+      c->flags[(size_t)b] = (uint8_t)((shared < ((int64_t)1 << (32 - m)) ? mpt::kFlagPacked : 0) |
+                                      (sum >= ((int64_t)1 << (32 - m)) ? mpt::kFlagOffsets : 0));
       inst_occ[(size_t)b] = (int)occ;
     }
     c->tab_off[(size_t)batch] = tab;
@@ -152,7 +175,7 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
     for (int pass = 0; pass < 2; ++pass) {
       for (int32_t b = 0; b < batch; ++b) {
         const int m = (int)(inst_requests[b + 1] - inst_requests[b]);
-        const bool rows = m >= 6 && c->packed_ok[(size_t)b];
+        const bool rows = m >= 6 && (c->flags[(size_t)b] & mpt::kFlagPacked);
         if (rows != (pass == 0)) continue;
         c->inst_list[(size_t)fill[(size_t)m]++] = b;
         int& cap = c->group_occ_cap[(size_t)m];
@@ -228,17 +251,17 @@ mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_byt
   h2d(c.chunks, b->chunks.data(), (size_t)b->occurrences * 8);
   h2d(c.tab_off, b->tab_off.data(), (B + 1) * 8);
   h2d(c.inst_list, b->inst_list.data(), B * 4);
-  h2d(c.packed_ok, b->packed_ok.data(), B);
+  h2d(c.flags, b->flags.data(), B);
   for (int m = 1; m <= kBatchMaxM && e == cudaSuccess; ++m) {
     const int64_t g0 = b->group_start[(size_t)m], gr = b->group_rows_end[(size_t)m],
                   g1 = b->group_start[(size_t)m + 1];
     const int cap = b->group_occ_cap[(size_t)m];
     if (gr > g0)
       e = mpt::launch_batch_rows((int)(gr - g0), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                                 c.inst_list + g0, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+                                 c.inst_list + g0, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
     if (e == cudaSuccess && g1 > gr)
       e = mpt::launch_batch((int)(g1 - gr), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                            c.inst_list + gr, c.packed_ok, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+                            c.inst_list + gr, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
   }
   d2h(b->opt.data(), c.opt, B * 8);
   d2h(b->status.data(), c.status, B * 4);

@@ -83,6 +83,11 @@ enum DeviceError : int {
 // Workspace carve-up (all offsets 256-byte aligned).
 // ---------------------------------------------------------------------------
 constexpr int kOffsetSlots = 33;
+
+// Per-instance flags of a batch (mpt_batch.cu, k_batch.cu): packed 32-bit keys,
+// and private / universal chunks kept out of the keys.
+constexpr uint8_t kFlagPacked = 1;
+constexpr uint8_t kFlagOffsets = 2;
 constexpr int kUniversalSlot = 32;
 
 struct Workspace {

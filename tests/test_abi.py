@@ -133,7 +133,10 @@ def test_batch_create_validation(mpt):
     assert _batch_status(mpt, w, [[[50]]]) == 1                             # chunk id >= n
     assert _batch_status(mpt, w, [[]]) == 1                                 # an instance with no request
     heavy = np.full(50, 1 << 30, dtype=np.int64)
-    assert _batch_status(mpt, heavy, [[[0, 1]]]) == 3                       # sum of w(R_i) >= 2^31
+    assert _batch_status(mpt, heavy, [[[0, 1], [0, 1], [2]]]) == 3          # shared weight >= 2^31
+    assert _batch_status(mpt, heavy, [[[0, 1]], [[0, 3], [0, 4]]]) == 0     # private and common chunks only
+    huge = np.full(50, 1 << 61, dtype=np.int64)
+    assert _batch_status(mpt, huge, [[[0, 1], [0, 1]]]) == 3                # sum of w(R_i) >= 2^62
     big = [[list(range(0, 2049))]]
     assert _batch_status(mpt, np.ones(3000, dtype=np.int64), big) == 2      # > 2048 occurrences
 

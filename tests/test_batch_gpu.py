@@ -94,19 +94,52 @@ def test_batch_large_requests(mpt):
     check_batch(mpt, weights, batch)
 
 
+def _shared_weight(weights, reqs):
+    """sum_i w(R_i) less the chunks that one or all m >= 2 requests hold."""
+    cnt = {}
+    for r in reqs:
+        for x in r:
+            cnt[x] = cnt.get(x, 0) + 1
+    return sum(int(weights[x]) * c for x, c in cnt.items() if 2 <= c < len(reqs))
+
+
 def test_batch_mixed_key_widths(mpt):
-    """Instances whose request weights need the 64-bit keys (sum_i w(R_i) >=
-    2^(32 - m)) next to ones that use the packed 32-bit keys, sizes shuffled
-    so the per-size launches must map results back to their instances."""
+    """Instances whose shared weight needs the 64-bit keys (>= 2^(32 - m))
+    next to ones that use the packed 32-bit keys, sizes shuffled so the
+    per-size launches must map results back to their instances."""
     rng = np.random.default_rng(71)
     n = 400
     heavy = rng.integers(60_000, 120_000, size=n, dtype=np.int64)
     batch = []
     for _ in range(60):
         m = int(rng.integers(2, 14))
-        batch.append([sorted(set(int(x) for x in rng.choice(n, size=int(rng.integers(1, 12)), replace=False)))
+        pool = rng.choice(n, size=30, replace=False)
+        batch.append([sorted(set(int(x) for x in rng.choice(pool, size=int(rng.integers(1, 12)), replace=False)))
                       for _ in range(m)])
-    sums = [sum(int(heavy[x]) for r in reqs for x in r) for reqs in batch]
-    assert any(s >= 1 << (32 - len(reqs)) for s, reqs in zip(sums, batch))
-    assert any(s < 1 << (32 - len(reqs)) for s, reqs in zip(sums, batch))
+    shared = [_shared_weight(heavy, reqs) for reqs in batch]
+    assert any(s >= 1 << (32 - len(reqs)) for s, reqs in zip(shared, batch))
+    assert any(s < 1 << (32 - len(reqs)) for s, reqs in zip(shared, batch))
     check_batch(mpt, heavy, batch)
+
+
+def test_batch_private_and_common_weights(mpt):
+    """Groups whose requests carry a private suffix of up to 2^40 tokens and a
+    common prefix of up to 2^36 (sum_i w(R_i) far beyond 2^31) over small
+    shared passages: the shared weight keeps them on the 32-bit keys, and
+    every OPT, table entry and order equals the oracle's."""
+    weights, batch = rag_batch(200, 3000, seed=5, m_range=(1, 13))
+    rng = np.random.default_rng(6)
+    extra = []
+    for g, reqs in enumerate(batch):
+        prefix = len(weights) + len(extra)
+        extra.append(int(rng.integers(1 << 30, 1 << 36)))
+        for i in range(len(reqs)):
+            if rng.random() < 0.7:
+                reqs[i] = reqs[i] + [len(weights) + len(extra)]
+                extra.append(int(rng.integers(1 << 20, 1 << 40)))
+            if g % 2 == 0:
+                reqs[i] = [prefix] + reqs[i]
+    w = np.concatenate([weights, np.array(extra, dtype=np.int64)])
+    assert all(_shared_weight(w, reqs) < 1 << (32 - len(reqs)) for reqs in batch)
+    assert max(sum(int(w[x]) for r in reqs for x in r) for reqs in batch) >= 1 << 40
+    check_batch(mpt, w, batch)
