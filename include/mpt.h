@@ -59,12 +59,13 @@ typedef struct mpt_ctx mpt_ctx;
  * in Thm 1): it adds w(x) to F(S) for every non-empty S holding its
  * requests, whatever the splits.  The tiled kernels therefore run the
  * recurrence on F(S) - sum_{i in S} pi_i - u and add it back in every output.
- * AUTO picks BLOCKED whenever W < 2^20 (its 32-bit packed keys are then
- * exact), else WIDE while W < 2^51 (64-bit packed keys), else GENERAL.  All
- * of them return the same tables, OPT and layout. */
+ * AUTO picks BLOCKED whenever W < 2^(32 - b), b = min(m, 12) tile bits
+ * (2^20 from m = 12 on; its 32-bit packed keys are then exact), else WIDE
+ * while W < 2^51 (64-bit packed keys), else GENERAL.  All of them return the
+ * same tables, OPT and layout. */
 typedef enum mpt_dp_mode {
   MPT_DP_AUTO = 0,
-  MPT_DP_BLOCKED = 1, /* shared-memory tiled min-plus; needs W < 2^20 */
+  MPT_DP_BLOCKED = 1, /* shared-memory tiled min-plus; needs W < 2^(32 - min(m, 12)) */
   MPT_DP_GENERAL = 2, /* one subset per thread or warp, int64 gathers from HBM/L2 */
   MPT_DP_WIDE = 3     /* the tiled min-plus with 64-bit keys; needs W < 2^51 */
 } mpt_dp_mode;
@@ -84,8 +85,8 @@ mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* 
 mpt_status mpt_workspace_bytes(const mpt_ctx* ctx, size_t* bytes);
 
 /* Choose the DP kernels (default MPT_DP_AUTO).  BLOCKED is refused with
- * OVERFLOW when the shared weight W (above) is >= 2^20, WIDE when
- * W >= 2^51. */
+ * OVERFLOW when the shared weight W (above) is >= 2^(32 - min(m, 12)), WIDE
+ * when W >= 2^51. */
 mpt_status mpt_set_dp_mode(mpt_ctx* ctx, int32_t mode);
 
 /* Solve exactly (Sec. 3.1): scatter chunk weights by request set, superset

@@ -336,3 +336,38 @@ def test_key_width_follows_shared_weight(mpt):
     assert e.value.status == 3
     for c in (narrow, ctx, ctx2):
         mpt.mpt_destroy(c)
+
+
+def test_blocked_limit_on_shared_weight_property(mpt):
+    """Host logic of the key-width choice on random instances: BLOCKED is
+    accepted exactly when the shared weight (sum_i w(R_i) less the chunks
+    one request alone or all m >= 2 requests hold) is below 2^(32 - b),
+    b = min(m, 12) tile bits (2^20 from m = 12 on), and WIDE exactly when it
+    is below 2^51."""
+    rng = np.random.default_rng(404)
+    for t in range(60):
+        m = int(rng.integers(1, 15))
+        n = int(rng.integers(1, 40))
+        base = I.random_instance(m, n, (0, n), seed=int(rng.integers(1 << 30)), wmin=1, wmax=9, allow_empty=True)
+        if t % 3 == 0:
+            base = I.with_common_prefix(base, int(rng.integers(1, 1 << 40)))
+        shared = W.shared_weight(base)
+        for limit, mode in ((1 << (32 - min(m, 12)), "blocked"), (1 << 51, "wide")):
+            # scale so that the shared weight lands just below or at the limit when it is positive
+            for target in (limit - 1, limit):
+                scale = max(1, target // shared) if shared > 0 else 1
+                if max(int(x) for x in base.weights) * scale * max(m, 1) >= 1 << 62:
+                    continue  # beyond the int64 sums the ABI accepts
+                inst = I.Instance(base.weights * scale, base.bits)
+                if W.request_weight_sum(inst) >= 1 << 62:
+                    continue
+                ctx = mpt.mpt_create(inst.weights, inst.bits)
+                ok = W.shared_weight(inst) < limit
+                try:
+                    mpt.mpt_set_dp_mode(ctx, mode)
+                    accepted = True
+                except mpt.MPTError as e:
+                    assert e.status == 3
+                    accepted = False
+                assert accepted == ok, (t, mode, W.shared_weight(inst))
+                mpt.mpt_destroy(ctx)
