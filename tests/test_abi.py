@@ -371,3 +371,26 @@ def test_blocked_limit_on_shared_weight_property(mpt):
                     accepted = False
                 assert accepted == ok, (t, mode, W.shared_weight(inst))
                 mpt.mpt_destroy(ctx)
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    """No fallback: with the CUDA library absent, the binding refuses to load
+    instead of computing anything elsewhere."""
+    import subprocess
+    import sys
+
+    code = (
+        "import pathlib, sys\n"
+        "from paper_2609_13692_gb300 import build as B, mpt\n"
+        f"B.LIB = pathlib.Path({str(tmp_path / 'absent' / 'libmpt.so')!r})\n"
+        "mpt._LIB = None\n"
+        "try:\n"
+        "    mpt.solve([3, 4], [[1], [3]])\n"
+        "except RuntimeError as e:\n"
+        "    print('refused:', e)\n"
+        "    sys.exit(0)\n"
+        "sys.exit(1)\n"
+    )
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True, timeout=120)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert "is missing" in r.stdout
