@@ -185,6 +185,41 @@ def pin_recompute_local(C):
         assert (f, a, w) == (F[S], split[S], wI[S])
 
 
+def _balanced_t(lo, hi, a, b):
+    """Maximal clusters of a balanced binary tree over the requests lo..hi
+    (split at the midpoint) that lie inside the interval [a, b]."""
+    if b < lo or hi < a:
+        return 0
+    if a <= lo and hi <= b:
+        return 1
+    mid = (lo + hi) // 2
+    return _balanced_t(lo, mid, a, b) + _balanced_t(mid + 1, hi, a, b)
+
+
+def pin_c1p_bound(C):
+    """Consecutive-ones instances (Sec. 3, "a tractable special case"): each
+    chunk is wanted by a contiguous run of requests, so in a balanced tree
+    over that line every S_x splits into at most 2 ceil(log2 m) clusters, and
+    by Thm 1 (eq. 1) OPT_free <= sum_x w(x) t_x(balanced) <=
+    sum_x w(x) min(|S_x|, 2 ceil(log2 m))."""
+    rng = np.random.default_rng(97)
+    for _ in range(12):
+        m = int(rng.integers(2, 12))
+        n = int(rng.integers(3, 30))
+        runs = []
+        for _x in range(n):
+            a = int(rng.integers(0, m))
+            runs.append((a, int(rng.integers(a, m))))
+        reqs = [[x for x, (a, b) in enumerate(runs) if a <= i <= b] for i in range(m)]
+        w = rng.integers(1, 50, size=n, dtype=np.int64)
+        inst = I.Instance(w, I.pack_requests(reqs, n))
+        opt = _opt(C, inst)
+        depth = 2 * int(np.ceil(np.log2(m)))
+        balanced = sum(int(w[x]) * _balanced_t(0, m - 1, a, b) for x, (a, b) in enumerate(runs))
+        bound = sum(int(w[x]) * min(b - a + 1, depth) for x, (a, b) in enumerate(runs))
+        assert opt <= balanced <= bound, (m, n, opt, balanced, bound)
+
+
 ALL_PINS = [
     pin_k4_3,
     pin_open_problem,
@@ -198,5 +233,6 @@ ALL_PINS = [
     pin_bounds,
     pin_split_rule,
     pin_recompute,
+    pin_c1p_bound,
     pin_recompute_local,
 ]
