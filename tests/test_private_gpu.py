@@ -261,3 +261,17 @@ def test_common_prefix_rag_workload(mpt):
         assert pb == [base.n] + pa + [base.n + 1 + i]
     assert b.dfs_order.tolist() == a.dfs_order.tolist()
     assert mpt.mpt_trie_cost(inst.weights, b.perm_offsets, b.perm_chunks) == b.opt
+
+
+def test_common_prefix_on_every_kernel_family(mpt):
+    """A common prefix and private suffixes under the 64-bit keys (chosen by
+    AUTO for heavy shared weights, and forced) and the int64 kernels: every
+    table bit-exact against the oracle."""
+    heavy_shared = I.random_instance(14, 40, (2, 8), seed=31, wmin=1 << 20, wmax=1 << 24)
+    inst = _with_queries(I.with_common_prefix(heavy_shared, 1 << 40), seed=32, every=2)
+    assert (1 << 20) <= W.shared_weight(inst) < 1 << 51 and W.universal_weight(inst) == 1 << 40
+    _parity(mpt, inst, expect_mode=3)
+    _parity(mpt, inst, mode="general", expect_mode=2)
+    light = _with_queries(I.with_common_prefix(I.rag_pools(15, 3000, 5, 40, 8, 1.1, seed=8), 1 << 34), seed=33)
+    _parity(mpt, light, mode="wide", expect_mode=3)
+    _parity(mpt, light, mode="general", expect_mode=2)
