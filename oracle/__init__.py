@@ -8,9 +8,10 @@ It shares no code with the CUDA library and never imports it.
 Everything here follows "Prefix Sharing Is a Sorting Problem" (arxiv
 2609.13692):
 
-* ``intersection_weights`` / ``dp`` / ``recompute``: the C half
+* ``intersection_weights`` / ``dp`` / ``recompute`` / ``dp_at``: the C half
   (``oracle.c``): w(I(S)) by direct intersection (Thm 1 proof) and the
-  O(3^m) subset recurrence of Sec. 3.1 in cost form.
+  O(3^m) subset recurrence of Sec. 3.1 in cost form (``dp_at``: its step at
+  listed subsets, for timing samples of layers too large to finish).
 * ``layout``: the constructive direction of Thm 1 -- walk the hierarchy
   top-down, at node B emit I(B) minus I(parent(B)), then recurse.
 * ``trie_cost``: eq. (1), the weight of the non-root nodes of the trie of the
@@ -78,6 +79,8 @@ def _bind(lib):
     lib.oracle_recompute.restype = ctypes.c_int
     lib.oracle_recompute.argtypes = [ctypes.c_int32, ctypes.c_int64, i64p, u64p, i64p, u64p, ctypes.c_int64,
                                      i64p, u32p, i64p, ctypes.c_int32]
+    lib.oracle_dp_at.restype = ctypes.c_int
+    lib.oracle_dp_at.argtypes = [ctypes.c_int32, i64p, i64p, u64p, ctypes.c_int64, i64p, u32p, ctypes.c_int32]
     lib.oracle_max_threads.restype = ctypes.c_int
     lib.oracle_max_threads.argtypes = []
     return lib
@@ -132,6 +135,22 @@ class COracle:
         if rc != 0:
             raise RuntimeError(f"oracle_dp failed ({rc})")
         return F, split
+
+    def dp_at(self, wI: np.ndarray, F: np.ndarray, m: int, subsets, threads: int = 0):
+        """The recurrence's step at the listed subsets, from the tables wI and
+        F (int64[2^m]): returns (F int64[count], split uint32[count])."""
+        wI = np.ascontiguousarray(wI, dtype=np.int64)
+        F = np.ascontiguousarray(F, dtype=np.int64)
+        S = np.ascontiguousarray(subsets, dtype=np.uint64)
+        if wI.shape[0] != (1 << m) or F.shape[0] != (1 << m) or (S.size and int(S.max()) >= (1 << m)):
+            raise ValueError("tables must hold 2^m entries and subsets lie below 2^m")
+        Fo = np.zeros(S.shape[0], dtype=np.int64)
+        so = np.zeros(S.shape[0], dtype=np.uint32)
+        rc = self.lib.oracle_dp_at(m, _p(wI, ctypes.c_int64), _p(F, ctypes.c_int64), _p(S, ctypes.c_uint64),
+                                   int(S.shape[0]), _p(Fo, ctypes.c_int64), _p(so, ctypes.c_uint32), threads)
+        if rc != 0:
+            raise RuntimeError(f"oracle_dp_at failed ({rc})")
+        return Fo, so
 
     def solve(self, weights, bits, threads: int = 0):
         """(OPT, F, wI, split) for a whole instance."""
@@ -191,6 +210,10 @@ def solve(weights, bits, threads: int = 0):
 
 def recompute(weights, bits, F_table: np.ndarray, subsets, threads: int = 0):
     return _default().recompute(weights, bits, F_table, subsets, threads)
+
+
+def dp_at(wI: np.ndarray, F: np.ndarray, m: int, subsets, threads: int = 0):
+    return _default().dp_at(wI, F, m, subsets, threads)
 
 
 # ---------------------------------------------------------------------------

@@ -202,6 +202,39 @@ int oracle_dp(int32_t m, const int64_t* wI, int64_t* F, uint32_t* split, int32_t
   return 0;
 }
 
+/* The recurrence's step (Sec. 3.1) at listed subsets only: for each S with
+ * |S| >= 2, F(S) and split(S) from the tables F (its proper subsets) and wI,
+ * by the same best_split as oracle_dp; subsets with |S| <= 1 get F = wI[S]
+ * (0 for S = 0) and split 0.  With the oracle's own tables it reproduces
+ * oracle_dp's entries; its use is timing the recurrence on samples of
+ * layers too large to finish (each S costs 2^(|S|-1) - 1 splits whatever
+ * the table values). */
+int oracle_dp_at(int32_t m, const int64_t* wI, const int64_t* F, const uint64_t* subsets, int64_t count,
+                 int64_t* F_out, uint32_t* split_out, int32_t nthreads) {
+  if (m < 1 || m > 32 || count < 0) return -1;
+#ifdef _OPENMP
+  if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+  (void)nthreads;
+#endif
+  int64_t t;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (t = 0; t < count; ++t) {
+    uint64_t S = subsets[t];
+    if (popcount64(S) <= 1) {
+      F_out[t] = (S == 0) ? 0 : wI[S];
+      split_out[t] = 0;
+      continue;
+    }
+    int64_t best;
+    uint64_t arg;
+    best_split(S, F, &best, &arg);
+    F_out[t] = best - wI[S];
+    split_out[t] = (uint32_t)arg;
+  }
+  return 0;
+}
+
 /* Recompute F(S) and split(S) for a list of subsets from a supplied table
  * (e.g. one produced elsewhere), with w(I(S)) recomputed from scratch.  Used
  * to check sampled entries of tables too large for oracle_dp. */

@@ -154,3 +154,25 @@ def test_universal_chunks_shift_F_by_a_constant():
     inst = I.with_common_prefix(base, 7)
     assert O.brute_force_permutations(inst.weights, inst.bits) == O.brute_force_permutations(base.weights,
                                                                                             base.bits) + 7
+
+
+def test_dp_at_reproduces_the_full_table(C):
+    """The recurrence's step at listed subsets (used to time samples of layers
+    too large to finish) gives oracle_dp's F and split at every subset when it
+    reads the oracle's own tables, including singletons and the empty set;
+    and F(S) = F(split) + F(S \\ split) - w(I(S)) at the full set (Sec. 3.1)."""
+    inst = I.config(1)
+    opt, F, wI, split = C.solve(inst.weights, inst.bits)
+    m = inst.m
+    subsets = np.arange(1 << m, dtype=np.uint64)
+    Fa, sa = C.dp_at(wI, F, m, subsets, threads=2)
+    assert np.array_equal(Fa, F) and np.array_equal(sa, split)
+    full = (1 << m) - 1
+    A = int(split[full])
+    assert Fa[full] == F[A] + F[full ^ A] - wI[full] == opt
+    rng = np.random.default_rng(3)
+    pick = rng.integers(0, 1 << m, size=200).astype(np.uint64)
+    Fb, sb = C.dp_at(wI, F, m, pick, threads=1)
+    assert np.array_equal(Fb, F[pick.astype(np.int64)]) and np.array_equal(sb, split[pick.astype(np.int64)])
+    with pytest.raises(ValueError):
+        C.dp_at(wI, F, m, np.array([1 << m], dtype=np.uint64))
