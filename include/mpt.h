@@ -374,12 +374,16 @@ mpt_status mpt_layout_pinned(const int64_t* weights, int64_t n_chunks, int32_t m
  * (MPT_ERR_OVERFLOW).  The scratch -- the blocked recurrence's working tables
  * and per-layer minima -- is one file-scope device array of 10.7 MiB that
  * every GPU loading this library holds until the process exits.  The first
- * call on a device looks up that array's device address, so make it before
- * any stream capture.  The call synchronises `stream` once, to read the
+ * call on a device looks up that array's device address (and the device's
+ * SM count) and keeps it for the life of the process, so make it before any
+ * stream capture, and do not reset the device (cudaDeviceReset) while the
+ * library is loaded.  Every call synchronises `stream` once, to read the
  * input check, then enqueues the solve and returns: the outputs are ready
- * when the stream reaches that point.  Every call shares the one array and
- * finds the previous call's contents in it; calls whose work overlaps on the
- * GPU (other streams, other host threads) race and must be serialised. */
+ * when the stream reaches that point.  The device-side consistency flags
+ * that mpt_solve reports as MPT_ERR_INTERNAL are not read back by this call.
+ * Every call shares the one array and finds the previous call's contents in
+ * it; calls whose work overlaps on the GPU (other streams, other host
+ * threads) race and must be serialised. */
 mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chunks, const uint64_t* d_req_bits, int32_t m,
                              int64_t* d_F, int64_t* d_wI, uint32_t* d_split, int64_t* d_opt, void* stream);
 
@@ -392,6 +396,18 @@ mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chunks, const u
  * current device.  gbps: 8 bytes per load / elapsed seconds / 1e9.
  * 10 <= log2_entries <= 32.  Errors: INVALID_ARG, OUT_OF_MEMORY, CUDA. */
 mpt_status mpt_gather_bandwidth(int32_t log2_entries, int64_t loads, void* stream, double* gbps);
+
+/* Measurement helper, not part of the method: the measured peak rate of the
+ * one instruction the blocked Sec. 3.1 recurrence issues per split -- a
+ * 32-bit add fused with an unsigned min, acc = min(acc, x + y), on the
+ * integer ALU pipe -- with every SM busy (16 warps each, 32 independent
+ * minima per thread, no memory traffic in the loop).  About `ops` add-mins
+ * are timed with CUDA events on `stream` after a short warm-up launch.
+ * ops_per_s: add-mins per second at whatever SM clock the GPU ran (the
+ * caller samples it); the nominal figure is SMs x 64 lanes x clock.
+ * 1 <= ops < ~2^28 x SMs x 2^19.  Errors: INVALID_ARG, OUT_OF_MEMORY (an
+ * 8-byte sink), CUDA. */
+mpt_status mpt_alu_addmin_peak(int64_t ops, void* stream, double* ops_per_s);
 
 /* Free the context and any workspace the library allocated.  NULL is a no-op. */
 void mpt_destroy(mpt_ctx* ctx);

@@ -44,6 +44,7 @@ EXPORTED = [
     "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
     "mpt_cache_costs", "mpt_layout_pinned", "mpt_solve_steps", "mpt_solve_begin", "mpt_solve_layers",
     "mpt_solve_end", "mpt_solve_resume", "mpt_set_tables", "mpt_tables32", "mpt_gather_bandwidth",
+    "mpt_alu_addmin_peak",
 ]
 
 
@@ -130,6 +131,7 @@ def load() -> ctypes.CDLL:
         "mpt_set_tables": ([vp, i32], ctypes.c_int),
         "mpt_tables32": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp)], ctypes.c_int),
         "mpt_gather_bandwidth": ([i32, i64, vp, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+        "mpt_alu_addmin_peak": ([i64, vp, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -678,4 +680,12 @@ def mpt_gather_bandwidth(log2_entries: int, loads: int = 1 << 28, stream: Option
     s = 0 if stream is None else int(stream)
     _check(load().mpt_gather_bandwidth(int(log2_entries), int(loads), ctypes.c_void_p(s), ctypes.byref(out)),
            "mpt_gather_bandwidth")
+    return float(out.value)
+
+
+def mpt_alu_addmin_peak(ops: int = 1 << 42, stream: Optional[int] = None) -> float:
+    """Measured add-min instructions per second of the integer ALU pipe, all SMs busy."""
+    out = ctypes.c_double()
+    s = 0 if stream is None else int(stream)
+    _check(load().mpt_alu_addmin_peak(int(ops), ctypes.c_void_p(s), ctypes.byref(out)), "mpt_alu_addmin_peak")
     return float(out.value)

@@ -246,8 +246,9 @@ def test_lean_tables_host_checks(mpt):
 
 
 def test_helper_argument_checks(mpt):
-    """Host-side checks of mpt_trie_cost, mpt_solve_noalloc and
-    mpt_gather_bandwidth, all returned before any CUDA call."""
+    """Host-side checks of mpt_trie_cost, mpt_solve_noalloc,
+    mpt_gather_bandwidth and mpt_alu_addmin_peak, all returned before any CUDA
+    call."""
     import ctypes
 
     lib = mpt.load()
@@ -278,6 +279,10 @@ def test_helper_argument_checks(mpt):
     assert lib.mpt_gather_bandwidth(33, 1000, None, ctypes.byref(gbps)) == 1
     assert lib.mpt_gather_bandwidth(20, 0, None, ctypes.byref(gbps)) == 1
     assert lib.mpt_gather_bandwidth(20, 1000, None, None) == 1
+    # mpt_alu_addmin_peak: operation count and output
+    rate = ctypes.c_double()
+    assert lib.mpt_alu_addmin_peak(0, None, ctypes.byref(rate)) == 1
+    assert lib.mpt_alu_addmin_peak(1000, None, None) == 1
 
 
 def test_caller_workspace_checks(mpt):
