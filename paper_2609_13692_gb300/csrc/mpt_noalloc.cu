@@ -51,22 +51,29 @@ __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
 char* g_scratch_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
 
-// Per-device set-up: the device address of the scratch array for the current
-// device, looked up once and cached.
-cudaError_t scratch_for_current_device(char** out) {
+// Per-device set-up: the device address of the scratch array and the SM
+// count of the current device, looked up once and cached (so a
+// cudaDeviceReset while the library is loaded leaves a stale address).
+cudaError_t scratch_for_current_device(char** out, int* sms) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
   if (!g_scratch_ptr[dev]) {
+    int count = 0;
+    e = cudaDeviceGetAttribute(&count, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
+    g_sm_count[dev] = count > 0 ? count : 1;
     g_scratch_ptr[dev] = static_cast<char*>(p);
   }
   *out = g_scratch_ptr[dev];
+  *sms = g_sm_count[dev];
   return cudaSuccess;
 }
 
@@ -128,14 +135,15 @@ extern "C" mpt_status mpt_solve_noalloc(const int64_t* d_weights, int64_t n_chun
   if (m > kNoAllocMaxM) return MPT_ERR_TOO_LARGE;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_ptr);
   char* base = nullptr;
-  if (scratch_for_current_device(&base) != cudaSuccess) return MPT_ERR_CUDA;
+  int sms = 1;
+  if (scratch_for_current_device(&base, &sms) != cudaSuccess) return MPT_ERR_CUDA;
 
   const int64_t words = (n_chunks + 63) / 64;
   unsigned long long* check = reinterpret_cast<unsigned long long*>(base + kOffCheck);
   if (cudaMemsetAsync(check, 0, kChecks * sizeof(unsigned long long), stream) != cudaSuccess) return MPT_ERR_CUDA;
   {
     int64_t blocks = (words * 64 + 255) / 256;
-    if (blocks > 152 * 16) blocks = 152 * 16;
+    if (blocks > (int64_t)sms * 16) blocks = (int64_t)sms * 16;
     k_noalloc_check<<<(unsigned)blocks, 256, 0, stream>>>(d_weights, d_req_bits, n_chunks, m, words, check);
     if (cudaGetLastError() != cudaSuccess) return MPT_ERR_CUDA;
   }
