@@ -1,10 +1,11 @@
 """CUDA path vs the CPU oracle, through the C ABI.
 
 Integer results must be bit-exact: OPT, every F(S), every w(I(S)), every
-split(S), the per-request permutations and the DFS order.  Where the oracle
-cannot run the whole recurrence (m >= 24), sampled subsets are recomputed by
-the oracle from the GPU's own table of smaller subsets, w(I(S)) is recomputed
-from scratch, and the trie cost of the returned layout must equal OPT.
+split(S), the per-request permutations and the DFS order -- in full up to
+m = 24, where the oracle still finishes the whole recurrence.  Where it
+cannot (m >= 28), at least 10^5 sampled subsets are recomputed by the oracle
+from the GPU's own table of smaller subsets, w(I(S)) is recomputed from
+scratch, and the trie cost of the returned layout must equal OPT.
 """
 
 import numpy as np
@@ -205,12 +206,11 @@ def assert_sampled_parity(mpt, inst, seed, uniform=20000):
 
 
 def test_config3_m24(mpt):
-    """RAG-shaped m = 24: every w(I(S)) bit-exact; sampled F and split."""
-    inst = I.config(3)
-    res, prof, count = assert_sampled_parity(mpt, inst, seed=24)
-    wI = mpt.mpt_tables(res.ctx)[1].cpu().numpy()
-    assert np.array_equal(wI, O.intersection_weights(inst.weights, inst.bits))
-    assert prof["dp_mode"] == 1 and count > 20000
+    """RAG-shaped m = 24 (1.4e11 splits): the oracle runs the whole recurrence
+    (about half a minute on the host cores), and OPT, every F(S), every
+    w(I(S)), every split(S), the permutations and the DFS order are bit-exact."""
+    res, prof = assert_full_parity(mpt, I.config(3), expect_mode=1)
+    assert prof["dp_mode"] == 1
 
 
 def test_config4_m28(mpt):
@@ -220,9 +220,10 @@ def test_config4_m28(mpt):
 
 
 def test_config5_m30(mpt):
-    """RAG-shaped m = 30, k = 40, 1M-passage corpus."""
-    res, prof, count = assert_sampled_parity(mpt, I.config(5), seed=30, uniform=20000)
-    assert prof["dp_mode"] == 1
+    """RAG-shaped m = 30, k = 40, 1M-passage corpus: at least 10^5 sampled
+    subsets recomputed (uniform plus per-size strata, the full set included)."""
+    res, prof, count = assert_sampled_parity(mpt, I.config(5), seed=30, uniform=100000)
+    assert prof["dp_mode"] == 1 and count >= 100000
 
 
 def _submask_index(S):
