@@ -37,12 +37,11 @@ if ROOT not in sys.path:
 
 METRIC = "subset-splits evaluated/sec (≈3^m/2 per solve) and exact-MPT solve time at m=28"
 WORKLOAD = 4
-ORACLE_SAMPLE_REQUESTS = 22  # reference arm: full oracle recurrence on the first 22 requests per step
-CPU_BASELINE_REQUESTS = 23  # cpu_baseline: one run on the first 23 requests (10-30 s of CPU work)
+FULL_RUN_REQUESTS = 22  # context: the oracle's whole recurrence on the first 22 requests
 # Each split is one 32-bit add and min, which the pair kernel issues as one
 # instruction on the integer ALU pipe (ncu: its arithmetic runs on that pipe).
-# The pipe peak (SMs x 4 sub-partitions x 16 lanes per clock at the maximum SM
-# clock) is computed from the device where the roofline is reported.
+# The roofline peak is that instruction's rate measured on this GPU
+# (mpt_alu_addmin_peak: every SM busy, nothing else in the loop).
 OPS_PER_SPLIT = 1
 
 
@@ -163,16 +162,116 @@ class ClockSampler:
 # CPU oracle legs
 # ---------------------------------------------------------------------------
 
+_HOST_CORES = None
+
+
+def host_cores() -> int:
+    """OpenMP threads the oracle has on this host, read before any call
+    that sets a smaller count (the setting persists in the process)."""
+    global _HOST_CORES
+    if _HOST_CORES is None:
+        import oracle
+
+        _HOST_CORES = oracle.max_threads()
+    return _HOST_CORES
+
+
 def oracle_sample(inst, m_sub: int, threads: int = 0):
     """The oracle's full recurrence on the first ``m_sub`` requests of the
     instance (all host cores, or ``threads`` of them)."""
     import oracle
 
+    P = threads or host_cores()
     bits = np.ascontiguousarray(inst.bits[:m_sub])
     t0 = time.perf_counter()
-    opt, F, wI, split = oracle.solve(inst.weights, bits, threads=threads)
+    opt, F, wI, split = oracle.solve(inst.weights, bits, threads=P)
     dt = time.perf_counter() - t0
-    return splits_per_solve(m_sub), dt, (threads or oracle.max_threads())
+    return splits_per_solve(m_sub), dt, P
+
+
+RUNS_PER_LAYER = 16
+
+
+def next_same_size(S: int) -> int:
+    """The next larger integer with the same number of set bits (Gosper)."""
+    c = S & -S
+    r = S + c
+    return (((r ^ S) >> 2) // c) | r
+
+
+def oracle_extrapolated(m: int, threads: int = 0, seed: int = 0, layer_splits: float = 4e8,
+                        measure_cost: float = 3e9, wi_requests: int = 22, inst=None) -> dict:
+    """The oracle's whole solve time for an m-request instance, extrapolated
+    from samples of every layer of its recurrence (labelled as such).
+
+    Layer k of the oracle's loop holds C(m, k) subsets of 2^(k-1) - 1 splits
+    each (the table values only decide rare strict improvements, not the
+    work), run in parallel over the subsets of the layer.  Each layer's
+    sample -- runs of 8 consecutive k-subsets in the increasing order the
+    oracle visits them, from seeded random starts, at least 4 per thread --
+    goes through the oracle's own step (``oracle.dp_at``) on a table of the
+    full 2^m size, and its measured splits/s prices the layer; a layer of at
+    most 4 subsets per thread is run whole.  Layers whose sample would cost
+    more than ``measure_cost`` splits are priced from the per-thread split
+    time of the largest measured layer, in rounds of one subset per thread.
+    The direct-intersection table w(I) (a single-threaded walk over all 2^m
+    subsets) is timed on the first ``wi_requests`` requests and scaled by
+    2^(m - wi_requests)."""
+    import oracle
+
+    P = threads or host_cores()
+    table = np.ones(1 << m, dtype=np.int64)  # stands in for F and w(I)
+    rng = np.random.default_rng(seed)
+    total, measured, modelled, tau = 0.0, [], [], None
+    for k in range(2, m + 1):
+        per = (1 << (k - 1)) - 1
+        count = math.comb(m, k)
+        want = min(count, max(4 * P, math.ceil(layer_splits / per)), 4096)
+        if want * per <= measure_cost or tau is None:
+            if want == count:
+                S = (1 << k) - 1
+                sample = []
+                while S < (1 << m):
+                    sample.append(S)
+                    S = next_same_size(S)
+            else:
+                sample = []
+                run = max(8, want // RUNS_PER_LAYER)
+                while len(sample) < want:
+                    S = int(sum(1 << int(i) for i in rng.choice(m, size=k, replace=False)))
+                    for _ in range(run):
+                        if S >= (1 << m) or len(sample) >= want:
+                            break
+                        sample.append(S)
+                        S = next_same_size(S)
+            subsets = np.array(sample, dtype=np.uint64)
+            t0 = time.perf_counter()
+            oracle.dp_at(table, table, m, subsets, threads=P)
+            dt = time.perf_counter() - t0
+            layer = dt if len(sample) == count else count * dt / len(sample)
+            tau = dt * min(P, len(sample)) / (len(sample) * per)
+            measured.append(k)
+        else:
+            layer = math.ceil(count / P) * per * tau
+            modelled.append(k)
+        total += layer
+    wi = None
+    if inst is not None:
+        sub = min(wi_requests, m)
+        bits = np.ascontiguousarray(inst.bits[:sub])
+        t0 = time.perf_counter()
+        oracle.intersection_weights(inst.weights, bits)
+        wi = (time.perf_counter() - t0) * 2.0 ** (m - sub)
+        total += wi
+    del table
+    return {"m": m, "extrapolated_solve_s": total, "splits_per_s": splits_per_solve(m) / total, "threads": P,
+            "layers_sampled": measured, "layers_priced_from_largest_sampled": modelled,
+            "wI_walk_s": wi,
+            "sample": (f"every layer k = 2..{m} of the oracle's recurrence sampled (>= 4 subsets per thread, "
+                       f"runs of 8 consecutive k-subsets from seeded starts, ~{layer_splits:.0e} splits per "
+                       "layer, small layers whole) through oracle.dp_at on a 2^m table; layer time = "
+                       "C(m,k)(2^(k-1)-1) / sampled splits/s; w(I) walk timed on the first "
+                       f"{min(wi_requests, m)} requests x 2^{m - min(wi_requests, m)}; EXTRAPOLATED, not a full run")}
 
 
 def cpu_model() -> str:
@@ -198,25 +297,39 @@ def run_reference(args):
             return
     from paper_2609_13692_gb300 import instances
 
-    inst = instances.config(WORKLOAD, seed=0)
-    m_sub = args.ref_requests
-    for _ in range(args.warmup):
-        oracle_sample(inst, m_sub)
-    total_splits, total_t, cores = 0, 0.0, 1
-    for _ in range(args.steps):
-        s, dt, cores = oracle_sample(inst, m_sub)
-        total_splits += s
-        total_t += dt
-    rate = total_splits / total_t
-    sample = (f"oracle recurrence (C, OpenMP over the subsets of each size) on the first {m_sub} of the "
-              f"{inst.m} requests of workload {WORKLOAD}: {splits_per_solve(m_sub)} splits per step")
+    inst = instances.config(args.workload, seed=0)
+    m = inst.m
+    for w in range(args.warmup):
+        oracle_extrapolated(m, seed=1000 + w)
+    total_t, cores, last = 0.0, 1, None
+    t_wall = 0.0
+    for step in range(args.steps):
+        t0 = time.perf_counter()
+        last = oracle_extrapolated(m, seed=step, inst=inst if step == 0 else None)
+        t_wall += time.perf_counter() - t0
+        if step == 0:
+            wi_s = last["wI_walk_s"]
+        else:
+            last["extrapolated_solve_s"] += wi_s
+        total_t += last["extrapolated_solve_s"]
+        cores = last["threads"]
+    solve_s = total_t / args.steps
+    rate = splits_per_solve(m) / solve_s
+    full_m = min(FULL_RUN_REQUESTS, m)
+    full_s, full_dt, _ = oracle_sample(inst, full_m)
+    sample = (f"workload {args.workload} (m = {m}) per step: " + last["sample"] +
+              f"; {1000 * t_wall / args.steps:.0f} ms of host time per step")
     line = {
         "impl": "reference", "metric": METRIC, "value": rate, "unit": "splits/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total_t / args.steps,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * solve_s,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-        "config": {"workload": instances.CONFIG_NAMES[WORKLOAD], "m": inst.m, "n": inst.n, "sample_requests": m_sub,
-                   "parallelism": "host cores"},
-        "cpu_baseline": {"value": rate, "unit": "splits/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "solve_time_s": solve_s, "solve_time_kind": "extrapolated from per-layer samples",
+        "config": {"workload": instances.CONFIG_NAMES[args.workload], "m": m, "n": inst.n,
+                   "splits_per_solve": splits_per_solve(m), "parallelism": "host cores"},
+        "cpu_baseline": {"value": rate, "unit": "splits/s", "cores": cores, "kind": "oracle", "sample": sample,
+                         "cpu": cpu_model(),
+                         "full_run": {"value": full_s / full_dt, "sample": f"whole recurrence on the first "
+                                      f"{full_m} requests ({full_s} splits, {full_dt:.1f} s)"}},
         "e2e": {"value": rate, "unit": "splits/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -228,14 +341,37 @@ def run_reference(args):
 # GPU leg
 # ---------------------------------------------------------------------------
 
+def source_digest(rel: str) -> str:
+    import hashlib
+
+    with open(os.path.join(ROOT, rel), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
 def load_traffic_profile():
-    """DRAM bytes per pair-kernel launch from a committed ncu summary (or None)."""
+    """DRAM bytes per pair-kernel launch from a committed ncu summary, or None
+    when the kernel source has changed since those counters were taken."""
     path = os.path.join(ROOT, "profiles", "k_dp_pairs_traffic.json")
     try:
         with open(path) as f:
-            return json.load(f)
+            tr = json.load(f)
     except OSError:
         return None
+    src = tr.get("source")
+    if not src or tr.get("source_sha256_16") != source_digest(src):
+        return None
+    return tr
+
+
+def measure_alu_peak(mpt, stream, device_index: int, tries: int = 3) -> dict:
+    """The add-min peak of the integer ALU pipe measured on this GPU
+    (mpt_alu_addmin_peak, best of ``tries``), with the SM clock sampled
+    while it ran."""
+    sampler = ClockSampler(device_index)
+    sampler.start()
+    rates = [mpt.mpt_alu_addmin_peak(1 << 43, stream) for _ in range(tries)]
+    clocks = sampler.stop()
+    return {"ops_per_s": max(rates), "runs": rates, "clocks": clocks}
 
 
 def run_ours(args):
@@ -257,6 +393,10 @@ def run_ours(args):
     mpt.load()
 
     inst = instances.config(args.workload, seed=replica_seed(rank))
+    if args.requests:
+        # profiling a smaller case of the same workload: its first requests
+        inst = instances.Instance(inst.weights, np.ascontiguousarray(inst.bits[:args.requests]),
+                                  f"{inst.name}, first {args.requests} requests")
     m = inst.m
     splits = splits_per_solve(m)
 
@@ -302,7 +442,7 @@ def run_ours(args):
     h2d = int(inst.weights.nbytes + inst.bits.nbytes)
     slots = int(sum(int(x).bit_count() for x in inst.bits.ravel()))
     d2h = 8 + 32 + 8 * (m + 1) + 8 * slots + 4 * m
-    e2e_steps = max(1, min(args.steps, 3))
+    e2e_steps = max(1, args.steps)
     barrier(world)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
@@ -330,20 +470,33 @@ def run_ours(args):
         ops_per_launch = OPS_PER_SPLIT * prof_sum["splits_pairs"] / launches
         achieved = ops_per_launch / (avg_ms / 1000.0) / 1e12
         tr = load_traffic_profile()
-        # integer ALU pipe: SMs (from the device) x 4 sub-partitions x 16 lanes
-        # per clock at the maximum SM clock nvidia-smi reports (2,070 MHz if
-        # it reports none)
+        # the pipe's add-min rate measured on this GPU, next to the nominal
+        # SMs x 4 sub-partitions x 16 lanes per clock at the maximum SM clock
+        alu = measure_alu_peak(mpt, stream.cuda_stream, torch.cuda.current_device())
+        alu_peak = alu["ops_per_s"] / 1e12
         sms = torch.cuda.get_device_properties(device).multi_processor_count
         max_mhz = (clock_info or {}).get("sm_max_mhz") or 2070.0
-        alu_peak = sms * 64 * max_mhz * 1e6 / 1e12
+        nominal = sms * 64 * max_mhz * 1e6 / 1e12
+        run_mhz = (clock_info or {}).get("sm_mhz")
+        probe_mhz = alu["clocks"].get("sm_mhz")
         wide = dp_mode == "wide"
         roofline = {"bound": "alu", "kernel": "k_dp_pairs_w" if wide else "k_dp_pairs", "achieved": achieved,
                     "peak": alu_peak, "unit": "Tops/s", "frac": achieved / alu_peak,
-                    "traffic": None if wide else (tr or {}).get("dram_bytes_per_launch"),
+                    "traffic": None if wide or tr is None else tr.get("dram_bytes_per_launch"),
+                    "traffic_source": None if wide or tr is None else
+                    f"ncu capture summarised in profiles/k_dp_pairs_traffic.json ({tr.get('workload', '')}), "
+                    "scaled to this workload's average launch; not measured by this run",
                     "ops_per_split": OPS_PER_SPLIT,
-                    "peak_basis": f"{sms} SMs x 64 integer-ALU-pipe lanes x {max_mhz / 1000:.3f} GHz "
-                                  "(one add-min per split" + ("; 64-bit keys take several ALU instructions "
-                                                              "per split" if wide else "") + ")",
+                    "peak_basis": "measured: mpt_alu_addmin_peak, independent add-min chains on every SM, "
+                                  f"best of {len(alu['runs'])} ({', '.join(f'{r / 1e12:.2f}' for r in alu['runs'])} "
+                                  f"Tops/s) at a median SM clock of {probe_mhz} MHz"
+                                  + ("; 64-bit keys take several ALU instructions per split" if wide else ""),
+                    "nominal_peak": nominal, "frac_of_nominal": achieved / nominal,
+                    "nominal_basis": f"{sms} SMs x 64 integer-ALU-pipe lanes x {max_mhz / 1000:.3f} GHz",
+                    "per_sm_clock": {"kernel_ops": achieved * 1e12 / (sms * run_mhz * 1e6) if run_mhz else None,
+                                     "kernel_mhz": run_mhz,
+                                     "peak_ops": alu["ops_per_s"] / (sms * probe_mhz * 1e6) if probe_mhz else None,
+                                     "peak_mhz": probe_mhz, "nominal_ops": 64},
                     "share_of_step": prof_sum["ms_dp_pairs"] / (local_ms if local_ms > 0 else 1)}
     else:
         hbm = float(peaks.get("hbm_gbs", 6800.0))
@@ -356,16 +509,40 @@ def run_ours(args):
     gather_gbs = mpt.mpt_gather_bandwidth(min(m, 30), 1 << 28, stream.cuda_stream)
     gather_frac = (16.0 * value / world) / (gather_gbs * 1e9)
 
-    # CPU baseline: the oracle, timed on this host, bounded sample
+    # CPU baseline: the oracle, timed on this host on bounded samples of the
+    # same workload (every layer of its recurrence), extrapolated to a whole
+    # solve; beside it the m = 30 workload and one whole run at 22 requests
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        s_sub, dt, cores = oracle_sample(inst, CPU_BASELINE_REQUESTS)
-        s1, dt1, _ = oracle_sample(inst, 19, threads=1)
-        cpu = {"value": s_sub / dt, "unit": "splits/s", "cores": cores, "kind": "oracle",
-               "sample": f"full oracle recurrence on the first {CPU_BASELINE_REQUESTS} of the {m} requests "
-                         f"({s_sub} splits, {dt:.1f} s)",
-               "single_thread": {"value": s1 / dt1, "sample": f"first 19 requests ({s1} splits, {dt1:.1f} s)"},
+        t_cpu = time.perf_counter()
+        ext = oracle_extrapolated(m, inst=inst)
+        ext1 = oracle_extrapolated(m, threads=1, layer_splits=1e7, measure_cost=4e7)
+        ext1["extrapolated_solve_s"] += ext["wI_walk_s"]
+        ext1["splits_per_s"] = splits / ext1["extrapolated_solve_s"]
+        cpu = {"value": ext["splits_per_s"], "unit": "splits/s", "cores": ext["threads"], "kind": "oracle",
+               "sample": f"workload {args.workload} (m = {m}): " + ext["sample"],
+               "extrapolated_solve_s": ext["extrapolated_solve_s"],
+               "single_thread": {"value": ext1["splits_per_s"], "extrapolated_solve_s": ext1["extrapolated_solve_s"],
+                                 "sample": "the same per-layer sampling with one thread (~1e7 splits per layer)"},
                "cpu": cpu_model()}
+        if args.workload == WORKLOAD:
+            inst30 = instances.config(5, seed=0)
+            e30 = oracle_extrapolated(30, inst=inst30)
+            e30_1 = oracle_extrapolated(30, threads=1, layer_splits=1e7, measure_cost=4e7)
+            e30_1["extrapolated_solve_s"] += e30["wI_walk_s"]
+            cpu["m30"] = {"workload": instances.CONFIG_NAMES[5], "extrapolated_solve_s": e30["extrapolated_solve_s"],
+                          "splits_per_s": e30["splits_per_s"], "threads": e30["threads"],
+                          "single_thread_extrapolated_solve_s": e30_1["extrapolated_solve_s"],
+                          "sample": "the same per-layer sampling on the m = 30 workload"}
+        s_sub, dt, _ = oracle_sample(inst, FULL_RUN_REQUESTS)
+        sub = instances.Instance(inst.weights, np.ascontiguousarray(inst.bits[:FULL_RUN_REQUESTS]))
+        e_sub = oracle_extrapolated(FULL_RUN_REQUESTS, inst=sub)
+        cpu["full_run"] = {"value": s_sub / dt, "solve_s": dt,
+                           "extrapolated_solve_s": e_sub["extrapolated_solve_s"],
+                           "sample": f"whole oracle recurrence on the first {FULL_RUN_REQUESTS} of the {m} requests "
+                                     f"({s_sub} splits, {dt:.1f} s), beside the per-layer extrapolation of the "
+                                     "same run as a check of the method"}
+        cpu["host_seconds"] = time.perf_counter() - t_cpu
 
     solve_s = max_ms / 1000.0 / args.steps
     line = {
@@ -380,9 +557,14 @@ def run_ours(args):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": {"blocked": "u32", "wide": "u64"}.get(dp_mode, "int64"),
+        "dtype_note": {"blocked": "exact: 32-bit packed integer keys, valid because the shared weight is below "
+                                  "2^(32 - tile bits) (checked at mpt_create); int64 tables and OPT",
+                       "wide": "exact: 64-bit packed integer keys (shared weight < 2^51); int64 tables and OPT"
+                       }.get(dp_mode, "exact int64 arithmetic"),
         "data": "synthetic",
         "solve_time_s": solve_s,
-        "config": {"workload": instances.CONFIG_NAMES[args.workload], "m": m, "n": inst.n,
+        "config": {"workload": instances.CONFIG_NAMES[args.workload]
+                   + (f" (first {args.requests} requests)" if args.requests else ""), "m": m, "n": inst.n,
                    "k": instances.CONFIGS[args.workload].get("k", m - 1), "seed": replica_seed(rank),
                    "splits_per_solve": splits, "dp_mode": dp_mode, "tables": args.tables,
                    "workspace_gib": round(ws.numel() / 2**30, 2),
@@ -532,10 +714,9 @@ def greedy_gap_small_groups(mpt):
 
 
 def run_cache(args):
-    """Finite-cache study (Sec. 8) on the NFCorpus-shaped stream: prefill cost
-    at many capacities per call, in arrival order, inside reorder windows and
-    in Thm 7's order, for the production (relevance-order), greedy and pinned
-    layouts."""
+    """Wall time of the Thm 7 serving order (mpt_serve_order) and of the
+    LRU radix-cache simulator (mpt_cache_costs, 10 capacities per call) on the
+    greedy layout of an NFCorpus-shaped request stream."""
     import torch
 
     from paper_2609_13692_gb300 import build as B
@@ -556,54 +737,28 @@ def run_cache(args):
         weights, ranked = instances.stream("nfcorpus-shaped", seed=0)
     n, m = len(weights), len(ranked)
     one = float(np.mean([sum(int(weights[x]) for x in q) for q in ranked]))
-    mult = [0.25, 0.5, 0.75, 0.9, 1, 4, 16, 64, 256, 1024]
-    caps = [int(round(f * one)) for f in mult]
-    layouts = {"production": [list(r) for r in ranked]}
-    if m <= 16384:  # the greedy hierarchy's limit
-        layouts["greedy"] = mpt.mpt_greedy(weights, ranked).perms
-        for t in (1, 2, 3):
-            layouts[f"pin_top{t}"] = mpt.mpt_layout_pinned(weights, ranked, t, "greedy").strings
-    total = int(sum(int(weights[x]) for q in ranked for x in q))
-    arrival = list(range(m))
-    g = layouts.get("greedy", layouts["production"])
-    # timed: the C ABI calls on a CSR built once (host arrays in and out)
-    g_csr = mpt.to_csr(g)
+    caps = [int(round(f * one)) for f in (0.25, 0.5, 0.75, 0.9, 1, 4, 16, 64, 256, 1024)]
+    layout = mpt.mpt_greedy(weights, ranked).perms if m <= 16384 else [list(r) for r in ranked]
+    csr = mpt.to_csr(layout)
     arr = np.arange(m, dtype=np.int32)
     for _ in range(args.warmup):
-        mpt.mpt_cache_costs(weights, g_csr, caps, arr)
+        mpt.mpt_cache_costs(weights, csr, caps, arr)
+        mpt.mpt_serve_order(n, csr)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        mpt.mpt_cache_costs(weights, g_csr, caps, arr)
+        mpt.mpt_cache_costs(weights, csr, caps, arr)
     dt = (time.perf_counter() - t0) / args.steps
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        thm7 = mpt.mpt_serve_order(n, g_csr)
+        mpt.mpt_serve_order(n, csr)
     dt_order = (time.perf_counter() - t0) / args.steps
-
-    table = {}
-    for name, strings in layouts.items():
-        unb = None
-        row = {}
-        for label, order in (("arrival", arrival), ("thm7", mpt.mpt_serve_order(n, strings).tolist())):
-            costs, unb = mpt.mpt_cache_costs(weights, strings, caps, order)
-            row[label] = {f"{f}x": int(c) for f, c in zip(mult, costs)}
-        row["unbounded"] = unb
-        row["saving_vs_no_sharing"] = 1 - unb / total
-        table[name] = row
-    windows = {}
-    for W in sorted({1, 128, 512, 2048, m}):
-        order = mpt.mpt_serve_order(n, g, arrival, W).tolist()
-        costs, unb = mpt.mpt_cache_costs(weights, g, caps[4:], order)
-        windows["all" if W == m else str(W)] = {f"{f}x": round(c / unb - 1, 4) for f, c in zip(mult[4:], costs)}
-    line = {"mode": "cache", "metric": "finite radix cache, prefill cost at 10 capacities per call",
-            "value": dt, "unit": "s", "higher_is_better": False, "steps": args.steps,
-            "timed_layout": "greedy" if "greedy" in layouts else "production",
-            "workload": f"nfcorpus-shaped stream: m = {m} requests, k = 8, one request = {one:.0f} tokens"
+    line = {"mode": "cache", "metric": "LRU radix-cache simulator, 10 capacities per call, wall time",
+            "value": dt, "unit": "s", "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+            "serve_order_s": dt_order,
+            "workload": f"nfcorpus-shaped stream: m = {m} requests, k = 8, greedy layout"
                         + (" (scaled)" if args.cache_m else ""),
-            "accesses": int(sum(len(q) for q in g)), "serve_order_s": dt_order,
-            "capacities_in_requests": mult, "no_sharing_cost": total, "layouts": table,
-            "window_excess_over_unbounded_greedy": windows,
+            "accesses": int(sum(len(q) for q in layout)),
             "note": "host arrays in and out, device buffers allocated inside each call"}
     print(json.dumps(line), flush=True)
 
@@ -624,14 +779,14 @@ def main():
     ap.add_argument("--workload", type=int, default=WORKLOAD, choices=[1, 2, 3, 4, 5, 6, 7],
                     help="benchmark workload (default 4: m = 28); others are for profiling")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--ref-requests", type=int, default=ORACLE_SAMPLE_REQUESTS,
-                    help="reference arm: requests of the workload in each step's oracle sample")
+    ap.add_argument("--requests", type=int, default=0,
+                    help="solve only the workload's first M requests (smaller cases for ncu captures)")
     ap.add_argument("--tables", choices=["int64", "lean"], default="int64",
                     help="table layout of the exact solve (lean: one int32 table, F over w(I))")
     ap.add_argument("--mode", choices=["solve", "batch", "greedy", "cache"], default="solve",
                     help="solve: the m = 28 exact solve (default); batch: many small request groups; "
                          "greedy: agglomerative hierarchy on a trace-sized request set; "
-                         "cache: finite-cache study on a request stream")
+                         "cache: serving order and radix-cache simulator timings on a request stream")
     ap.add_argument("--batch-size", type=int, default=20000)
     ap.add_argument("--greedy-m", type=int, default=3000)
     ap.add_argument("--cache-m", type=int, default=0,
