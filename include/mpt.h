@@ -46,7 +46,7 @@ typedef enum mpt_status {
   MPT_ERR_WORKSPACE_TOO_SMALL = 5, /* caller workspace below mpt_workspace_bytes() */
   MPT_ERR_CUDA = 6,                /* a CUDA call failed; mpt_last_error() has its text */
   MPT_ERR_NOT_SOLVED = 7,          /* results asked for before a successful mpt_solve */
-  MPT_ERR_TIMEOUT = 8,             /* reserved: a bounded device-side wait gave up */
+  MPT_ERR_TIMEOUT = 8,             /* a bounded wait on a shared-memory barrier inside a kernel gave up */
   MPT_ERR_INTERNAL = 9             /* a device-side consistency check failed */
 } mpt_status;
 
@@ -408,6 +408,14 @@ mpt_status mpt_gather_bandwidth(int32_t log2_entries, int64_t loads, void* strea
  * 1 <= ops < ~2^28 x SMs x 2^19.  Errors: INVALID_ARG, OUT_OF_MEMORY (an
  * 8-byte sink), CUDA. */
 mpt_status mpt_alu_addmin_peak(int64_t ops, void* stream, double* ops_per_s);
+
+/* How this copy of the library was built, as bits in *flags: bit 0 set
+ * means the bounds-checked variant (compiled with MPT_BOUNDS), whose kernels
+ * test table indices, window offsets and split entries, skip any access that
+ * fails and report MPT_ERR_INTERNAL from mpt_solve -- a stand-in for a
+ * device memory checker, slower than the default build.  Not part of the
+ * method.  Errors: INVALID_ARG (flags NULL). */
+mpt_status mpt_build_info(int32_t* flags);
 
 /* Free the context and any workspace the library allocated.  NULL is a no-op. */
 void mpt_destroy(mpt_ctx* ctx);

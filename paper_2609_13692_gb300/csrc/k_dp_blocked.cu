@@ -45,18 +45,26 @@ constexpr int kRow = 1 << kB2;             // 32 entries per row
 constexpr int kRowStride = kRow + 4;       // 36 words: consecutive rows start in different 16-byte bank groups
 constexpr int kRows = 1 << kB1;            // 128 rows per window
 constexpr int kWin = kRows * kRowStride;   // words per padded window
-constexpr int kPairThreads = 256;         // 8 warps: 2 per SM sub-partition, equal work each
+constexpr int kPairThreads = 256;         // 8 warps: 2 per SM sub-partition
+constexpr int kRing = 4;                   // window-pair slots per block
 constexpr int kSharedRows = 34;            // rows merged through shared memory every pair
 constexpr int kSharedOut = kSharedRows * kRow;
 constexpr int kSharedStride = kRow + 1;    // words per shared row in the per-pair minimum arrays
 constexpr int kSharedWords = kSharedRows * kSharedStride;
 constexpr int kSharedOwned = (kSharedOut + kPairThreads - 1) / kPairThreads;
-constexpr int kPairSmemBytes = (2 * 2 * kWin + 2 * kSharedWords + kRow * kPairThreads) * (int)sizeof(uint32_t);
+constexpr int kExtraUnits = 139;           // shared-row units of one pair
+constexpr int kExtraSlots = (kExtraUnits + 31) / 32;  // whole-warp slots per pair: 4 full, 1 of 11 lanes
+constexpr int kSlotCycle = 8;              // pairs after which the slot-to-warp rotation repeats
+constexpr int kPairSmemWords = kRing * 2 * kWin + kRing * kSharedWords + kRow * kPairThreads;
+constexpr int kPairSmemBytes = kPairSmemWords * (int)sizeof(uint32_t) + 3 * kRing * 8;
 constexpr int kMinPairsPerItem = 16;
 constexpr int kTileThreads = 512;
 constexpr int kMaxTileBits = 12;
 
-static_assert(kPairSmemBytes >= (1 << kB) * 8, "merge buffer must fit in the window buffers");
+static_assert(kRing * 2 * kWin * (int)sizeof(uint32_t) >= (1 << kB) * 8, "merge buffer must fit in the windows");
+static_assert((kRing * 2 * kWin + kRing * kSharedWords + kRow * kPairThreads) % 2 == 0, "8-byte aligned barriers");
+static_assert(kExtraSlots * 32 >= kExtraUnits && kExtraSlots <= kSlotCycle, "extra slots per pair");
+static_assert((kRowStride * 4) % 16 == 0, "padded rows start on 16-byte boundaries");
 
 // ---------------------------------------------------------------------------
 // Work split of the pair kernel.  The b inner bits are (s1, s2): s1 = the top
@@ -71,10 +79,13 @@ static_assert(kPairSmemBytes >= (1 << kB) * 8, "merge buffer must fit in the win
 // in registers across all pairs (running best key and Ta), merged with the
 // other tasks of the row once, at the end.
 // Shared rows: the 29 rows with <= 2 bits and those five -- 34 rows, 139
-// units.  Each unit is one extra unit of some thread (spread evenly over the
-// 8 warps); its 32 minima go to a per-pair shared array with atomicMin, and
-// owner threads fold that array into registers after every pair.
-// So every warp issues 8 units plus at most one extra unit per pair.
+// units per pair.  They run as whole-warp "slots" of 32 units (lane l takes
+// unit 32 i + l of slot i): 4 full slots and one of 11 lanes per pair.  The
+// slots of pair q go to warps (5 (q mod 8) + i) mod 8, so over 8 pairs every
+// warp runs exactly 5 slots, and each sub-partition 128 register units plus
+// 10 slots against 136.7 units of work (not 144, as one extra unit per warp
+// and pair would take).  A slot's 32 minima go to the pair's shared array
+// with atomicMin; owner threads fold that array into registers one pair later.
 // ---------------------------------------------------------------------------
 __host__ __device__ constexpr int popc_c(uint32_t v) {
   int c = 0;
@@ -97,9 +108,9 @@ constexpr uint32_t deposit_c(uint32_t q, uint32_t mask) {
 }
 
 struct PairPlan {
-  uint32_t task[kPairThreads];   // s1 | fixed << 8 | free << 16 (8 units)
-  uint32_t extra[kPairThreads];  // s1 | a1 << 8 | shared-row index << 16, or ~0u
-  uint32_t srow[kSharedRows];    // s1 of each shared row
+  uint32_t task[kPairThreads];            // s1 | fixed << 8 | free << 16 (8 units)
+  uint32_t extra[kExtraSlots * 32];       // s1 | a1 << 8 | shared-row index << 16, or ~0u
+  uint32_t srow[kSharedRows];             // s1 of each shared row
   int ntask, nextra, nsrow;
 };
 
@@ -131,13 +142,12 @@ constexpr PairPlan make_plan() {
     const uint32_t freem = s1 ^ lowbits;
     for (uint32_t v = 0; v < (1u << q); ++v) pl.task[n++] = s1 | (deposit_c(v, lowbits) << 8) | (freem << 16);
   }
-  for (int i = 0; i < kPairThreads; ++i) pl.extra[i] = 0xFFFFFFFFu;
+  for (int i = 0; i < kExtraSlots * 32; ++i) pl.extra[i] = 0xFFFFFFFFu;
   for (int ri = 0; ri < nr; ++ri) {
     const uint32_t s1 = pl.srow[ri];
     for (uint32_t k = 0; k < (1u << popc_c(s1)); ++k) {
       const uint32_t a1 = deposit_c(k, s1);
-      const int tid = (ne % 8) * 32 + ne / 8;  // extra unit ne -> warp ne % 8
-      pl.extra[tid] = s1 | (a1 << 8) | ((uint32_t)ri << 16);
+      pl.extra[ne] = s1 | (a1 << 8) | ((uint32_t)ri << 16);
       ++ne;
     }
   }
@@ -150,7 +160,7 @@ constexpr PairPlan make_plan() {
 constexpr PairPlan kPlanHost = make_plan();
 static_assert(kPlanHost.ntask == kPairThreads, "register tasks must fill the block");
 static_assert(kPlanHost.nsrow == kSharedRows, "shared row count");
-static_assert(kPlanHost.nextra == 139 && kPlanHost.nextra <= kPairThreads, "extra units");
+static_assert(kPlanHost.nextra == kExtraUnits, "extra units");
 static __constant__ PairPlan c_plan = make_plan();
 
 // Word of shared output j = (shared row, lane) in a per-pair minimum array:
@@ -165,34 +175,30 @@ __device__ __forceinline__ uint32_t sw_word(uint32_t j) { return j + (j >> kB2);
 __device__ __forceinline__ int row_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
 
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(gmem_src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(smem_u32(smem_dst)), "l"(gmem_src) : "memory");
 }
 
-// Issue the copies of the two windows of one pair into a buffer.  Thread t
-// copies the 16-byte chunks t + kThreads * j: rows (t >> 3) + (kThreads / 8) * j
-// (mod 128) of X (first 1024 chunks) and Y, always column t & 7.  row_pos is
-// linear, so each chunk's row position is one XOR away from row_pos(t >> 3).
-template <int kThreads>
-__device__ __forceinline__ void stage_pair(uint32_t* X, uint32_t* Y, const uint32_t* __restrict__ gx,
-                                           const uint32_t* __restrict__ gy) {
+// Every thread copies its share of the two windows of one pair into a ring
+// slot and arms the slot's "full" barrier to count one arrival once those
+// copies have landed (the barrier expects one arrival per thread).  Thread t
+// copies the 16-byte chunks t + kPairThreads * j: rows (t >> 3) + 32 j of X
+// (j < 4) and of Y, always column t & 7.  row_pos is linear, so each chunk's
+// padded row position is one XOR away from row_pos(t >> 3).
+__device__ __forceinline__ void copy_pair(uint32_t* X, uint32_t* Y, const uint32_t* __restrict__ gx,
+                                          const uint32_t* __restrict__ gy, unsigned long long* full) {
   constexpr int kChunks = kRows * kRow / 4;  // 1024 per window
-  static_assert(kChunks % kThreads == 0, "whole chunks per thread");
+  static_assert(kChunks % kPairThreads == 0, "whole chunks per thread");
   const uint32_t t = threadIdx.x;
   const uint32_t rp0 = (uint32_t)row_pos(t >> 3);
   const uint32_t col = (t & 7u) * 4u;
 #pragma unroll
-  for (int j = 0; j < kChunks / kThreads; ++j) {
-    const uint32_t rp = rp0 ^ (uint32_t)row_pos((uint32_t)(j * (kThreads / 8)));
+  for (int j = 0; j < kChunks / kPairThreads; ++j) {
+    const uint32_t rp = rp0 ^ (uint32_t)row_pos((uint32_t)(j * (kPairThreads / 8)));
     const uint32_t d = rp * kRowStride + col;
-    cp_async16(X + d, gx + 4 * (t + (uint32_t)(j * kThreads)));
-    cp_async16(Y + d, gy + 4 * (t + (uint32_t)(j * kThreads)));
+    cp_async16(X + d, gx + 4 * (t + (uint32_t)(j * kPairThreads)));
+    cp_async16(Y + d, gy + 4 * (t + (uint32_t)(j * kPairThreads)));
   }
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(full)) : "memory");
 }
 
 __device__ __forceinline__ void load_row(uint32_t (&v)[kRow], const uint32_t* p) {
@@ -208,8 +214,10 @@ __device__ __forceinline__ void load_row(uint32_t (&v)[kRow], const uint32_t* p)
 }
 
 // acc[s2] = min over a2 in s2 of x[a2] + y[s2 ^ a2]  (243 add/min pairs).
-// The a2-outer order puts independent accumulators next to each other.  With
-// kInit the a2 = 0 term initialises acc instead of being min-ed into it.
+// The a2-outer order puts independent accumulators next to each other (an
+// order that spreads each accumulator's updates evenly measured 1.7 % slower:
+// ptxas schedules this one better).  With kInit the a2 = 0 term initialises
+// acc instead of being min-ed into it.
 template <bool kInit = false>
 __device__ __forceinline__ void conv_rows(uint32_t (&acc)[kRow], const uint32_t (&x)[kRow], const uint32_t (&y)[kRow]) {
 #pragma unroll
@@ -226,19 +234,66 @@ __device__ __forceinline__ void conv_rows(uint32_t (&acc)[kRow], const uint32_t 
   }
 }
 
+// A bounded barrier wait that the whole (converged) warp leaves together:
+// true only if every lane saw the phase complete.
+__device__ __forceinline__ bool warp_wait(unsigned long long* bar, uint32_t parity) {
+  return __all_sync(0xFFFFFFFFu, mbar_wait(bar, parity));
+}
+
+// Fold pair jj's shared-row minima (ring slot jj mod kRing) into the running
+// bests of the shared outputs this thread owns (a strict improvement takes
+// the pair's Ta), reset them for the slot's next pair, and mark the slot
+// free.  False if the pair's "consumed" barrier did not complete in time.
+__device__ __forceinline__ bool fold_pair(uint32_t jj, uint32_t Ta_jj, uint32_t* smin, unsigned long long* consumed,
+                                          unsigned long long* folded, uint32_t (&sbk)[kSharedOwned],
+                                          uint32_t (&sbt)[kSharedOwned]) {
+  const uint32_t c = jj % kRing;
+  if (!warp_wait(&consumed[c], (jj / kRing) & 1u)) return false;
+  uint32_t* sm = smin + c * kSharedWords;
+#pragma unroll
+  for (int j = 0; j < kSharedOwned; ++j) {
+    const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
+    if (o < (uint32_t)kSharedOut) {
+      const uint32_t w = sw_word(o);
+      const uint32_t v = sm[w];
+      sm[w] = 0xFFFFFFFFu;
+      if (v < sbk[j]) {
+        sbk[j] = v;
+        sbt[j] = Ta_jj;
+      }
+    }
+  }
+  mbar_arrive(&folded[c]);
+  return true;
+}
+
 // Pair kernel for tiles with |T| = kh >= 2.  Block = (tile, range of pairs).
 // Writes, per inner subset U of the tile, the lexicographic minimum of
 // (key, Ta) over its pairs into partial[tile << kB | U] with atomicMin.
+//
+// The pairs of the range stream through a ring of kRing window slots with no
+// block-wide barrier.  Pair q lives in slot q mod kRing.  At the start of
+// step q every warp waits until all threads have folded pair q + 1 - kRing
+// ("folded"), and its threads start their copies of pair q + 1 into that
+// slot; then they wait for pair q's copies ("full"), run their units, arrive
+// on "consumed", fold the previous pair's shared-row minima into their
+// running bests (in pair order) and arrive on "folded".  Every wait is
+// bounded; one that gives up sets kErrTimeout in *flags and the thread stops
+// (after waiting, bounded again, for the copies it started), so the launch
+// ends with its results marked invalid.
 __global__ void __launch_bounds__(kPairThreads, 1)
 k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, unsigned long long* __restrict__ partial,
-           int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item) {
+           int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item,
+           int32_t* __restrict__ flags) {
   extern __shared__ __align__(16) uint32_t smem[];
-  // window buffer c: X at smem + 2c * kWin, Y right after it; then two
-  // per-pair minimum arrays of the shared rows
-  uint32_t* smin = smem + 4 * kWin;
-  // Ta of each register output's running best, [output][thread]: written only
-  // when a pair strictly improves the best, by a predicated store
-  uint32_t* sbest_t = smin + 2 * kSharedWords;
+  // ring slot c: X at smem + 2c * kWin, Y right after it; then one per-pair
+  // minimum array of the shared rows per slot; then the running-best Ta of
+  // every register output, [output][thread]; then the barriers
+  uint32_t* smin = smem + kRing * 2 * kWin;
+  uint32_t* sbest_t = smin + kRing * kSharedWords;
+  unsigned long long* full = reinterpret_cast<unsigned long long*>(sbest_t + kRow * kPairThreads);
+  unsigned long long* consumed = full + kRing;
+  unsigned long long* folded = consumed + kRing;
 
   const uint32_t tile = blockIdx.x / items_per_tile;
   const uint32_t item = blockIdx.x % items_per_tile;
@@ -247,6 +302,22 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t R = T ^ low;
   const uint32_t q0 = item * pairs_per_item;
   const uint32_t q1 = min(q0 + pairs_per_item, pairs_per_tile);
+  const uint32_t npairs = q1 > q0 ? q1 - q0 : 0u;
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31u;
+#ifdef MPT_BOUNDS
+  {
+    // the tile, and every pair's Ta: a part of T holding its lowest request,
+    // so both windows lie inside the 2^(L + kB)-entry tables
+    bool good = tile < c_binom.v[L][kh] && T < (1u << L) && __popc(T) == kh && q1 <= pairs_per_tile;
+    uint32_t sb = deposit_bits(q0, R);
+    for (uint32_t p = 0; p < npairs && good; ++p) {
+      const uint32_t Ta = low | sb;
+      good = (Ta & ~T) == 0 && Ta != T;
+      sb = (sb - R) & R;
+    }
+    if (MPT_BAD(flags, good)) return;  // the same decision in every thread
+  }
+#endif
 
   const uint32_t task = c_plan.task[threadIdx.x];
   const uint32_t s1 = task & 0xFFu;
@@ -257,11 +328,20 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t b2 = freem ^ b0 ^ b1;
   const uint32_t pos_fixed = (uint32_t)row_pos(fixed), pos_s1 = (uint32_t)row_pos(s1);
   const uint32_t pb0 = (uint32_t)row_pos(b0), pb1 = (uint32_t)row_pos(b1), pb2 = (uint32_t)row_pos(b2);
-  const uint32_t extra = c_plan.extra[threadIdx.x];
-  const bool has_extra = extra != 0xFFFFFFFFu;
-  const uint32_t es1 = extra & 0xFFu, ea1 = (extra >> 8) & 0xFFu, erow = (extra >> 16) & 0xFFu;
+  // this lane's unit in each of the kExtraSlots slots of a pair
+  uint32_t ext[kExtraSlots];
+#pragma unroll
+  for (int i = 0; i < kExtraSlots; ++i) ext[i] = c_plan.extra[32 * i + (int)lane];
 
-  for (int i = threadIdx.x; i < 2 * kSharedWords; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
+  if (threadIdx.x == 0) {
+    for (int c = 0; c < kRing; ++c) {
+      mbar_init(&full[c], kPairThreads);
+      mbar_init(&consumed[c], kPairThreads);
+      mbar_init(&folded[c], kPairThreads);
+    }
+    mbar_init_fence();
+  }
+  for (int i = threadIdx.x; i < kRing * kSharedWords; i += kPairThreads) smin[i] = 0xFFFFFFFFu;
   uint32_t bk[kRow], sbk[kSharedOwned], sbt[kSharedOwned];
 #pragma unroll
   for (int i = 0; i < kRow; ++i) {
@@ -273,30 +353,34 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
     sbk[j] = 0xFFFFFFFFu;
     sbt[j] = 0;
   }
+  __syncthreads();
 
+  // the first pair, into slot 0
   uint32_t sub = deposit_bits(q0, R);
-  {
-    const uint32_t Ta = low | sub;
-    stage_pair<kPairThreads>(smem, smem + kWin, Gp + ((size_t)Ta << kB), Gc + ((size_t)(T ^ Ta) << kB));
-    cp_async_commit();
-  }
-  for (uint32_t q = q0; q < q1; ++q) {
-    const int cur = (int)((q - q0) & 1u);
+  if (npairs >= 1) copy_pair(smem, smem + kWin, Gp + ((size_t)(low | sub) << kB), Gc + ((size_t)(R ^ sub) << kB), &full[0]);
+
+  bool ok = true;
+  uint32_t prev_Ta = 0;
+  for (uint32_t j = 0; j < npairs; ++j) {
+    const uint32_t c = j % kRing;
     const uint32_t Ta = low | sub;
     const uint32_t next = (sub - R) & R;
-    if (q + 1 < q1) {
-      const uint32_t Tn = low | next;
-      uint32_t* nb = smem + 2 * (cur ^ 1) * kWin;
-      stage_pair<kPairThreads>(nb, nb + kWin, Gp + ((size_t)Tn << kB), Gc + ((size_t)(T ^ Tn) << kB));
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
+    // copies of pair j + 1, into the slot pair j + 1 - kRing has left
+    if (j + 1 < npairs) {
+      const uint32_t cn = (j + 1) % kRing;
+      if (j + 1 >= (uint32_t)kRing && !warp_wait(&folded[cn], (((j + 1) / kRing) - 1u) & 1u)) {
+        ok = false;
+        break;
+      }
+      uint32_t* Xn = smem + 2 * cn * kWin;
+      copy_pair(Xn, Xn + kWin, Gp + ((size_t)(low | next) << kB), Gc + ((size_t)(R ^ next) << kB), &full[cn]);
     }
-    __syncthreads();
-    const uint32_t* X = smem + 2 * cur * kWin;
+    if (!warp_wait(&full[c], (j / kRing) & 1u)) {
+      ok = false;
+      break;
+    }
+    const uint32_t* X = smem + 2 * c * kWin;
     const uint32_t* Y = X + kWin;
-    uint32_t* sm = smin + cur * kSharedWords;
     {
       // The 8 units of the task visit a1 = fixed | sub with sub running over the
       // subsets of its 3 free bits in Gray-code order; row_pos is linear over
@@ -320,33 +404,38 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
         bk[i] = __vibmin_u32(bk[i], acc[i], &keep);
         if (!keep) sbest_t[i * kPairThreads + threadIdx.x] = Ta;
       }
-      if (has_extra) {
-        uint32_t x[kRow], y[kRow];
-        load_row(x, X + row_pos(ea1) * kRowStride);
-        load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
-        conv_rows<true>(acc, x, y);
-        uint32_t* row = sm + erow * kSharedStride;
+      // this warp's shared-row slot of the pair, if the rotation gives it one
+      const uint32_t slot = (warp + (uint32_t)kSlotCycle - (5u * (j % kSlotCycle)) % kSlotCycle) % kSlotCycle;
+      if (slot < (uint32_t)kExtraSlots) {
+        uint32_t e = ext[0];
 #pragma unroll
-        for (int i = 0; i < kRow; ++i) atomicMin(&row[i], acc[i]);
-      }
-    }
-    __syncthreads();
-    // fold this pair's shared-row minima into their owners' running best and
-    // reset the array for the pair after next
+        for (int i = 1; i < kExtraSlots; ++i)
+          if (slot == (uint32_t)i) e = ext[i];
+        if (e != 0xFFFFFFFFu) {
+          const uint32_t es1 = e & 0xFFu, ea1 = (e >> 8) & 0xFFu, erow = (e >> 16) & 0xFFu;
+          uint32_t x[kRow], y[kRow];
+          load_row(x, X + row_pos(ea1) * kRowStride);
+          load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
+          conv_rows<true>(acc, x, y);
+          uint32_t* row = smin + c * kSharedWords + erow * kSharedStride;
 #pragma unroll
-    for (int j = 0; j < kSharedOwned; ++j) {
-      const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
-      if (o < (uint32_t)kSharedOut) {
-        const uint32_t w = sw_word(o);
-        const uint32_t v = sm[w];
-        sm[w] = 0xFFFFFFFFu;
-        if (v < sbk[j]) {
-          sbk[j] = v;
-          sbt[j] = Ta;
+          for (int i = 0; i < kRow; ++i) atomicMin(&row[i], acc[i]);
         }
       }
     }
+    mbar_arrive(&consumed[c]);
+    if (j >= 1 && !fold_pair(j - 1, prev_Ta, smin, consumed, folded, sbk, sbt)) {
+      ok = false;
+      break;
+    }
+    prev_Ta = Ta;
     sub = next;
+  }
+  if (ok && npairs >= 1) ok = fold_pair(npairs - 1, prev_Ta, smin, consumed, folded, sbk, sbt);
+  if (!ok) {
+    if (lane == 0) atomicOr(flags, kErrTimeout);
+    // the copies this thread started must land before the block's memory goes away
+    asm volatile("cp.async.wait_all;" ::: "memory");
   }
 
   // Merge the threads that share a row, then the blocks that share the tile.
@@ -356,13 +445,14 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   __syncthreads();
 #pragma unroll
   for (int i = 0; i < kRow; ++i)
-    atomicMin(&merged[(s1 << kB2) | (uint32_t)i], ((unsigned long long)bk[i] << 32) | sbest_t[i * kPairThreads + threadIdx.x]);
+    atomicMin(&merged[(s1 << kB2) | (uint32_t)i],
+              ((unsigned long long)bk[i] << 32) | sbest_t[i * kPairThreads + threadIdx.x]);
 #pragma unroll
-  for (int j = 0; j < kSharedOwned; ++j) {
-    const uint32_t o = threadIdx.x + (uint32_t)(j * kPairThreads);
+  for (int jj = 0; jj < kSharedOwned; ++jj) {
+    const uint32_t o = threadIdx.x + (uint32_t)(jj * kPairThreads);
     if (o < (uint32_t)kSharedOut) {
       const uint32_t U = (c_plan.srow[o >> kB2] << kB2) | (o & (kRow - 1));
-      atomicMin(&merged[U], ((unsigned long long)sbk[j] << 32) | sbt[j]);
+      atomicMin(&merged[U], ((unsigned long long)sbk[jj] << 32) | sbt[jj]);
     }
   }
   __syncthreads();
@@ -385,7 +475,8 @@ __device__ __forceinline__ int64_t load_wI(const Tab* p) {
 template <typename Tab>
 __global__ void __launch_bounds__(kTileThreads)
 k_dp_tile(int L, int b, int kh, const Tab* __restrict__ wIr, const unsigned long long* __restrict__ partial,
-          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot) {
+          uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot,
+          int32_t* __restrict__ flags) {
   __shared__ uint32_t cur_p[1 << kMaxTileBits];   // this tile, F << b
   __shared__ uint32_t other_c[1 << kMaxTileBits]; // complement form: this tile (kh = 0) or tile 0 (kh >= 1)
   __shared__ uint16_t order[1 << kMaxTileBits];   // inner subsets sorted by size, then colex
@@ -476,9 +567,11 @@ k_dp_tile(int L, int b, int kh, const Tab* __restrict__ wIr, const unsigned long
         const uint32_t gc = gp | (~U & mask);
         cur_p[U] = gp;
         if (kh == 0) other_c[U] = gc;
-        Gp[idx] = gp;
-        Gc[idx] = gc;
-        split_rot[idx] = A;
+        if (!MPT_BAD(flags, idx < ((size_t)1 << (L + b)) && valid_split(T | (U << L), A))) {
+          Gp[idx] = gp;
+          Gc[idx] = gc;
+          split_rot[idx] = A;
+        }
       }
     }
     start += (uint32_t)cnt;
@@ -507,7 +600,8 @@ __device__ __forceinline__ uint32_t best_word(uint32_t U) { return U + (U >> kB2
 template <typename Tab>
 __global__ void __launch_bounds__(kRowsThreads)
 k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long long* __restrict__ partial,
-               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot) {
+               uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot,
+               int32_t* __restrict__ flags) {
   extern __shared__ __align__(16) uint32_t smem[];
   uint32_t* cur = smem;               // this tile, F << kB, padded rows
   uint32_t* zc = smem + kWin;         // tile 0, complement form, padded rows
@@ -518,6 +612,7 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
   const uint32_t tile = blockIdx.x;
   const uint32_t T = colex_unrank(tile, kh, L);
   const size_t tbase = (size_t)T << kB;
+  if (MPT_BAD(flags, tile < c_binom.v[L][kh] && T < (1u << L) && __popc(T) == kh)) return;
 
   for (int c = threadIdx.x; c < (1 << (kB - 2)); c += kRowsThreads) {
     const int row = c >> (kB2 - 2), k = c & ((1 << (kB2 - 2)) - 1);
@@ -630,9 +725,11 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
 
   for (int u = threadIdx.x; u < (1 << kB); u += kRowsThreads) {
     const uint32_t gp = cur[row_pos((uint32_t)u >> kB2) * kRowStride + (u & (kRow - 1))];
+    const uint32_t A = bsplit[best_word((uint32_t)u)];
+    if (MPT_BAD(flags, valid_split(T | ((uint32_t)u << L), A))) continue;
     Gp[tbase | (uint32_t)u] = gp;
     Gc[tbase | (uint32_t)u] = gp | (~(uint32_t)u & kMask);
-    split_rot[tbase | (uint32_t)u] = bsplit[best_word((uint32_t)u)];
+    split_rot[tbase | (uint32_t)u] = A;
   }
 }
 
@@ -715,7 +812,7 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
       if (e != cudaSuccess) return e;
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches], stream);
       k_dp_pairs<<<(unsigned)(tiles * items), kPairThreads, kPairSmemBytes, stream>>>(
-          ws.Gp, ws.Gc, ws.partial, L, kh, P, (uint32_t)items, ppi);
+          ws.Gp, ws.Gc, ws.partial, L, kh, P, (uint32_t)items, ppi, ws.counters + 1);
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches + 1], stream);
       if (timing) {
         timing->pair_launches++;
@@ -728,17 +825,19 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches], stream);
     if (kh == 0) {
       if (s.lean)
-        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.fw_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot);
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.fw_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot,
+                                                  ws.counters + 1);
       else
-        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot);
+        k_dp_tile<<<1, kTileThreads, 0, stream>>>(L, b, 0, ws.wI_rot, nullptr, ws.Gp, ws.Gc, ws.split_rot,
+                                                  ws.counters + 1);
     } else {
       const unsigned long long* part = kh >= 2 ? ws.partial : nullptr;
       if (s.lean)
         k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.fw_rot, part, ws.Gp,
-                                                                                  ws.Gc, ws.split_rot);
+                                                                                  ws.Gc, ws.split_rot, ws.counters + 1);
       else
         k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.wI_rot, part, ws.Gp,
-                                                                                  ws.Gc, ws.split_rot);
+                                                                                  ws.Gc, ws.split_rot, ws.counters + 1);
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;

@@ -56,15 +56,18 @@ __device__ __forceinline__ void scan_splits(uint32_t S, uint32_t low, uint32_t f
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads)
-k_dp_layer_thread(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split) {
+k_dp_layer_thread(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split,
+                  int32_t* __restrict__ flags) {
   const unsigned long long idx = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= count) return;
   const uint32_t S = colex_unrank(idx, k, m);
+  if (MPT_BAD(flags, (unsigned long long)S < (1ull << m) && __popc(S) == k)) return;
   const uint32_t low = S & (~S + 1u);
   const uint32_t rest = S ^ low;
   int64_t best = LLONG_MAX;
   uint32_t arg = 0;
   scan_splits(S, low, 0u, rest, rest, F, best, arg);
+  if (MPT_BAD(flags, valid_split(S, arg))) return;
   F[S] = (T)(best - (int64_t)wI[S]);
   split[S] = arg;
 }
@@ -74,12 +77,14 @@ k_dp_layer_thread(int m, int k, unsigned long long count, const T* wI, T* F, uin
 // lexicographically on (value, A).
 template <typename T>
 __global__ void __launch_bounds__(kThreads)
-k_dp_layer_warp(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split) {
+k_dp_layer_warp(int m, int k, unsigned long long count, const T* wI, T* F, uint32_t* __restrict__ split,
+                int32_t* __restrict__ flags) {
   const int lane = threadIdx.x & 31;
   const unsigned long long warps = (unsigned long long)gridDim.x * (blockDim.x >> 5);
   for (unsigned long long w = (unsigned long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); w < count;
        w += warps) {
     const uint32_t S = colex_unrank(w, k, m);
+    if (MPT_BAD(flags, (unsigned long long)S < (1ull << m) && __popc(S) == k)) continue;  // the same in every lane
     const uint32_t low = S & (~S + 1u);
     const uint32_t rest = S ^ low;
     uint32_t hi = 0, r = rest;
@@ -101,7 +106,7 @@ k_dp_layer_warp(int m, int k, unsigned long long count, const T* wI, T* F, uint3
         arg = oa;
       }
     }
-    if (lane == 0) {
+    if (lane == 0 && !MPT_BAD(flags, valid_split(S, arg))) {
       F[S] = (T)(best - (int64_t)wI[S]);
       split[S] = arg;
     }
@@ -109,8 +114,8 @@ k_dp_layer_warp(int m, int k, unsigned long long count, const T* wI, T* F, uint3
 }
 
 template <typename T>
-cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, cudaStream_t stream, int* launches,
-                       int step_begin, int step_end) {
+cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, int32_t* flags, cudaStream_t stream,
+                       int* launches, int step_begin, int step_end) {
   if (step_end < 0 || step_end > s.m) step_end = s.m;
   cudaError_t err = cudaSuccess;
   if (step_begin <= 0 && step_end > 0) {
@@ -125,11 +130,11 @@ cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, cudaS
     const unsigned long long count = h_binom.v[s.m][k];
     if (k <= kThreadMaxLayer) {
       const unsigned long long blocks = (count + kThreads - 1) / kThreads;
-      k_dp_layer_thread<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split);
+      k_dp_layer_thread<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split, flags);
     } else {
       unsigned long long blocks = (count + (kThreads / 32) - 1) / (kThreads / 32);
       if (blocks > 152ull * 16) blocks = 152ull * 16;
-      k_dp_layer_warp<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split);
+      k_dp_layer_warp<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split, flags);
     }
     ++*launches;
     err = cudaGetLastError();
@@ -144,8 +149,9 @@ int dp_steps(const Shape& s) { return s.blocked ? s.L + 1 : s.m; }
 
 cudaError_t launch_dp_general(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches,
                               int step_begin, int step_end) {
-  if (s.lean) return dp_general<int32_t>(s, ws.fw, ws.fw, ws.split, stream, launches, step_begin, step_end);
-  return dp_general<int64_t>(s, ws.wI, ws.F, ws.split, stream, launches, step_begin, step_end);
+  if (s.lean)
+    return dp_general<int32_t>(s, ws.fw, ws.fw, ws.split, ws.counters + 1, stream, launches, step_begin, step_end);
+  return dp_general<int64_t>(s, ws.wI, ws.F, ws.split, ws.counters + 1, stream, launches, step_begin, step_end);
 }
 
 }  // namespace mpt

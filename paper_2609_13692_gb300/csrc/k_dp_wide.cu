@@ -215,7 +215,8 @@ __device__ __forceinline__ void conv16(u64 (&acc)[kWRow], const u64 (&x)[kWRow],
 
 __global__ void __launch_bounds__(kWThreads, 1)
 k_dp_pairs_w(const u64* __restrict__ Gp, const u64* __restrict__ Gc, u64* __restrict__ pkey, uint32_t* __restrict__ pta,
-             int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item) {
+             int L, int kh, uint32_t pairs_per_tile, uint32_t items_per_tile, uint32_t pairs_per_item,
+             int32_t* __restrict__ flags) {
   extern __shared__ __align__(16) u64 wsm[];
   u64* pmin = wsm + 4 * kWWin;  // two per-pair minimum arrays of 4096
 
@@ -226,6 +227,20 @@ k_dp_pairs_w(const u64* __restrict__ Gp, const u64* __restrict__ Gc, u64* __rest
   const uint32_t R = T ^ low;
   const uint32_t q0 = item * pairs_per_item;
   const uint32_t q1 = min(q0 + pairs_per_item, pairs_per_tile);
+#ifdef MPT_BOUNDS
+  {
+    // the tile, and every pair's Ta: a proper part of T holding its lowest
+    // request, so both windows lie inside the tables
+    bool good = tile < c_binom.v[L][kh] && T < (1u << L) && __popc(T) == kh && q1 <= pairs_per_tile;
+    uint32_t sb = deposit_bits(q0, R);
+    for (uint32_t q = q0; q < q1 && good; ++q) {
+      const uint32_t Ta = low | sb;
+      good = (Ta & ~T) == 0 && Ta != T;
+      sb = (sb - R) & R;
+    }
+    if (MPT_BAD(flags, good)) return;  // the same decision in every thread
+  }
+#endif
   // this thread's chunks, read from constant memory once (lanes read
   // different entries, which the constant cache serves one at a time)
   const uint32_t c0 = c_wplan.first[threadIdx.x];
@@ -339,7 +354,7 @@ template <typename Tab>
 __global__ void __launch_bounds__(kWTileThreads)
 k_dp_tile_w(int L, int b, int kh, const Tab* __restrict__ wIr, const u64* __restrict__ pkey,
             const uint32_t* __restrict__ pta, uint32_t items, u64* __restrict__ Gp, u64* __restrict__ Gc,
-            uint32_t* __restrict__ split_rot) {
+            uint32_t* __restrict__ split_rot, int32_t* __restrict__ flags) {
   extern __shared__ __align__(16) u64 tsm[];
   u64* cur = tsm;                       // this tile, F << b
   u64* oc = tsm + (1 << kWB);           // complement form: this tile (kh = 0) or tile 0 (kh >= 1)
@@ -440,9 +455,11 @@ k_dp_tile_w(int L, int b, int kh, const Tab* __restrict__ wIr, const u64* __rest
         const u64 gc = gp | (u64)(~U & mask);
         cur[U] = gp;
         if (kh == 0) oc[U] = gc;
-        Gp[idx] = gp;
-        Gc[idx] = gc;
-        split_rot[idx] = A;
+        if (!MPT_BAD(flags, idx < ((size_t)1 << (L + b)) && valid_split(T | (U << L), A))) {
+          Gp[idx] = gp;
+          Gc[idx] = gc;
+          split_rot[idx] = A;
+        }
       }
     }
     start += (uint32_t)cnt;
@@ -486,7 +503,7 @@ cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t str
       choose_items(tiles, P, sms, max_items, &items, &ppi);
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches], stream);
       k_dp_pairs_w<<<(unsigned)(tiles * items), kWThreads, kWSmemBytes, stream>>>(
-          ws.Gp64, ws.Gc64, ws.partial, ws.partial_ta, L, kh, P, (uint32_t)items, ppi);
+          ws.Gp64, ws.Gc64, ws.partial, ws.partial_ta, L, kh, P, (uint32_t)items, ppi, ws.counters + 1);
       if (timing && timing->pair_ev) cudaEventRecord(timing->pair_ev[2 * timing->pair_launches + 1], stream);
       if (timing) {
         timing->pair_launches++;
@@ -499,10 +516,12 @@ cudaError_t launch_dp_wide(const Shape& s, const Workspace& ws, cudaStream_t str
     const unsigned grid = kh == 0 ? 1u : (unsigned)tiles;
     if (s.lean)
       k_dp_tile_w<<<grid, kWTileThreads, kWTileSmemBytes, stream>>>(L, b, kh, ws.fw_rot, ws.partial, ws.partial_ta,
-                                                                     (uint32_t)items, ws.Gp64, ws.Gc64, ws.split_rot);
+                                                                     (uint32_t)items, ws.Gp64, ws.Gc64, ws.split_rot,
+                                                                     ws.counters + 1);
     else
       k_dp_tile_w<<<grid, kWTileThreads, kWTileSmemBytes, stream>>>(L, b, kh, ws.wI_rot, ws.partial, ws.partial_ta,
-                                                                     (uint32_t)items, ws.Gp64, ws.Gc64, ws.split_rot);
+                                                                     (uint32_t)items, ws.Gp64, ws.Gc64, ws.split_rot,
+                                                                     ws.counters + 1);
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;
     ++*launches;

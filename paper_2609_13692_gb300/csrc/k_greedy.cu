@@ -463,7 +463,7 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
                o_perm = take((size_t)std::max<int64_t>(occ, 1) * 8), o_dfs = take(M * 4), o_comp = take(M * 4),
                o_bpar = take(M * 4), o_cbest = take(M * 8), o_mst = take(8);
   char* d = nullptr;
-  if (cudaMalloc(&d, off) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  if (device_alloc(reinterpret_cast<void**>(&d), off) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
   mpt_status st = MPT_OK;
   cudaError_t e = cudaSuccess;
   auto h2d = [&](size_t o, const void* h, size_t bytes) {

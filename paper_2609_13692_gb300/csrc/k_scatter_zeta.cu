@@ -56,7 +56,7 @@ k_scatter(const int64_t* __restrict__ w, const uint64_t* __restrict__ bits, int6
         atomicAdd(&priv[__ffs(N) - 1], (unsigned long long)w[x]);
       else if (priv && N == full)  // m >= 2 here: for m = 1 the full set is a singleton
         atomicAdd(&priv[kUniversalSlot], (unsigned long long)w[x]);
-      else
+      else if (!MPT_BAD(&counters[1], (rotated ? rot_index(N, L, b) : (size_t)N) < ((size_t)1 << m)))
         atomicAdd(&g[rotated ? rot_index(N, L, b) : (size_t)N], (G)w[x]);
       const int k = atomicAdd(&counters[0], 1);
       if (k < slots) {
@@ -74,10 +74,12 @@ constexpr int kZetaLowBits = 12;
 constexpr int kZetaThreads = 512;
 
 template <typename G>
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_low(G* __restrict__ g, int tb) {
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_low(G* __restrict__ g, int tb, size_t n,
+                                                           int32_t* __restrict__ flags) {
   __shared__ G t[1 << kZetaLowBits];
   const int size = 1 << tb;
   G* tile = g + ((size_t)blockIdx.x << tb);
+  if (MPT_BAD(flags, ((size_t)blockIdx.x + 1) << tb <= n)) return;
   for (int i = threadIdx.x; i < size; i += blockDim.x) t[i] = tile[i];
   const int half = size >> 1;
   for (int j = 0; j < tb; ++j) {
@@ -92,88 +94,98 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_low(G* __restrict__ g, in
   for (int i = threadIdx.x; i < size; i += blockDim.x) tile[i] = t[i];
 }
 
-// The same for tb = 12 with fewer barriers: thread t holds 8 consecutive
-// entries (bits 0-2 in registers), bits 3-7 are the lane bits (warp shuffles),
-// then one shared-memory pass regroups the tile so that each thread holds 8
-// entries 256 apart (bits 8-10 in registers) and bit 11 is one shared-memory
+// The same for tb = 12 with fewer barriers.  Thread t loads entries
+// t + 512 k (k < 8), so every warp load is one contiguous 256-byte run: index
+// bits 9-11 are in registers and bits 0-4 are the lane bits (warp shuffles).
+// One shared-memory pass regroups the tile so that each thread holds 8
+// entries 32 apart (bits 5-7 in registers), and bit 8 is one shared-memory
 // stage.  Sums are order-independent, so every stage is the same add.
 template <typename G>
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_low12(G* __restrict__ g) {
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_low12(G* __restrict__ g, size_t n, int32_t* __restrict__ flags) {
   static_assert(kZetaThreads * 8 == (1 << kZetaLowBits), "8 entries per thread");
   __shared__ G t[1 << kZetaLowBits];
   G* tile = g + ((size_t)blockIdx.x << kZetaLowBits);
+  if (MPT_BAD(flags, ((size_t)blockIdx.x + 1) << kZetaLowBits <= n)) return;
   const int tid = threadIdx.x, lane = tid & 31;
   G v[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) v[i] = tile[tid * 8 + i];
-#pragma unroll
-  for (int j = 0; j < 3; ++j)
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if (!(i & (1 << j))) v[i] += v[i | (1 << j)];
-#pragma unroll
-  for (int j = 0; j < 5; ++j) {
-    const bool low = !(lane & (1 << j));  // this lane's entries have bit 3 + j clear
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const G o = __shfl_xor_sync(0xFFFFFFFFu, v[i], 1 << j);
-      if (low) v[i] += o;
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) t[tid * 8 + i] = v[i];
-  __syncthreads();
-  // regroup: thread t takes entries base + 256 k, k < 8 (bits 8-10)
-  const int base = (tid & 255) | ((tid >> 8) << 11);
-#pragma unroll
-  for (int k = 0; k < 8; ++k) v[k] = t[base + 256 * k];
+  for (int k = 0; k < 8; ++k) v[k] = tile[tid + kZetaThreads * k];
 #pragma unroll
   for (int j = 0; j < 3; ++j)
 #pragma unroll
     for (int k = 0; k < 8; ++k)
       if (!(k & (1 << j))) v[k] += v[k | (1 << j)];
-  __syncthreads();
 #pragma unroll
-  for (int k = 0; k < 8; ++k) t[base + 256 * k] = v[k];
+  for (int j = 0; j < 5; ++j) {
+    const bool low = !(lane & (1 << j));  // this lane's entries have bit j clear
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const G o = __shfl_xor_sync(0xFFFFFFFFu, v[k], 1 << j);
+      if (low) v[k] += o;
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) t[tid + kZetaThreads * k] = v[k];
   __syncthreads();
-  // bit 11, then write back
-  for (int i = tid; i < (1 << (kZetaLowBits - 1)); i += kZetaThreads) t[i] += t[i | (1 << 11)];
+  // regroup: thread t takes entries base + 32 k, k < 8 (bits 5-7), with bits
+  // 0-4 = t & 31, bit 8 = (t >> 5) & 1 and bits 9-11 = t >> 6
+  const int base = lane | (((tid >> 5) & 1) << 8) | ((tid >> 6) << 9);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) v[k] = t[base + 32 * k];
+#pragma unroll
+  for (int j = 0; j < 3; ++j)
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (!(k & (1 << j))) v[k] += v[k | (1 << j)];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) t[base + 32 * k] = v[k];
+  __syncthreads();
+  // bit 8, then write back
+  for (int i = tid; i < (1 << (kZetaLowBits - 1)); i += kZetaThreads) {
+    const int e = ((i >> 8) << 9) | (i & 255);  // bit 8 of e clear
+    t[e] += t[e | 256];
+  }
   __syncthreads();
   for (int i = tid; i < (1 << kZetaLowBits); i += kZetaThreads) tile[i] = t[i];
 }
 
-// Superset sums over index bits [lo, lo + tb): each block owns 16 adjacent
-// columns (bits below lo) and all 2^tb values of those bits, for one value of
-// the bits above; rows of 16 entries are contiguous 128-byte segments.
+// Superset sums over index bits [lo, lo + tb), tb <= 8: each block owns
+// 4096 >> tb adjacent columns (bits below lo, lo >= 12) and all 2^tb values
+// of those bits, for one value of the bits above -- 4096 entries, rows of
+// contiguous columns.
 constexpr int kZetaCols = 16;
 constexpr int kZetaHighBits = 8;
+constexpr int kZetaBlockEntries = 1 << kZetaLowBits;
 
 template <typename G>
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_high(G* __restrict__ g, int lo, int tb) {
-  __shared__ G t[(1 << kZetaHighBits) * kZetaCols];
-  const size_t col_groups = ((size_t)1 << lo) / kZetaCols;
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_high(G* __restrict__ g, int lo, int tb, size_t n,
+                                                            int32_t* __restrict__ flags) {
+  __shared__ G t[kZetaBlockEntries];
+  const int cshift = kZetaLowBits - tb;  // log2 of the columns per block
+  const int cols = 1 << cshift;
+  const size_t col_groups = ((size_t)1 << lo) >> cshift;
   const size_t cg = blockIdx.x % col_groups;
   const size_t top = blockIdx.x / col_groups;
-  G* base = g + (top << (lo + tb)) + cg * kZetaCols;
-  const int rows = 1 << tb;
-  const int elems = rows * kZetaCols;
-  for (int e = threadIdx.x; e < elems; e += blockDim.x) {
-    const int r = e / kZetaCols, c = e % kZetaCols;
+  G* base = g + (top << (lo + tb)) + (cg << cshift);
+  // the block's last entry: row 2^tb - 1, its last column
+  if (MPT_BAD(flags, (top << (lo + tb)) + ((((size_t)1 << tb) - 1) << lo) + ((cg + 1) << cshift) <= n)) return;
+  for (int e = threadIdx.x; e < kZetaBlockEntries; e += blockDim.x) {
+    const int r = e >> cshift, c = e & (cols - 1);
     t[e] = base[((size_t)r << lo) + c];
   }
-  const int half = elems >> 1;
+  constexpr int kHalf = kZetaBlockEntries / 2;
   for (int j = 0; j < tb; ++j) {
     __syncthreads();
     const int lowmask = (1 << j) - 1;
-    for (int p = threadIdx.x; p < half; p += blockDim.x) {
-      const int c = p % kZetaCols, q = p / kZetaCols;
+    for (int p = threadIdx.x; p < kHalf; p += blockDim.x) {
+      const int c = p & (cols - 1), q = p >> cshift;
       const int r = ((q >> j) << (j + 1)) | (q & lowmask);  // bit j of r is 0
-      t[r * kZetaCols + c] += t[(r | (1 << j)) * kZetaCols + c];
+      t[(r << cshift) + c] += t[((r | (1 << j)) << cshift) + c];
     }
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < elems; e += blockDim.x) {
-    const int r = e / kZetaCols, c = e % kZetaCols;
+  for (int e = threadIdx.x; e < kZetaBlockEntries; e += blockDim.x) {
+    const int r = e >> cshift, c = e & (cols - 1);
     base[((size_t)r << lo) + c] = t[e];
   }
 }
@@ -184,13 +196,17 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_high(G* __restrict__ g, i
 // rows 16 apart (row bits 4-6 in registers), and row bit 7 is one
 // shared-memory stage.
 template <typename G>
-__global__ void __launch_bounds__(kZetaThreads) k_zeta_high8(G* __restrict__ g, int lo) {
+__global__ void __launch_bounds__(kZetaThreads) k_zeta_high8(G* __restrict__ g, int lo, size_t n,
+                                                             int32_t* __restrict__ flags) {
   static_assert(kZetaThreads * 8 == (1 << kZetaHighBits) * kZetaCols, "8 entries per thread");
   __shared__ G t[(1 << kZetaHighBits) * kZetaCols];
   const size_t col_groups = ((size_t)1 << lo) / kZetaCols;
   const size_t cg = blockIdx.x % col_groups;
   const size_t top = blockIdx.x / col_groups;
   G* base = g + (top << (lo + kZetaHighBits)) + cg * kZetaCols;
+  if (MPT_BAD(flags, (top << (lo + kZetaHighBits)) + ((((size_t)1 << kZetaHighBits) - 1) << lo) +
+                         (cg + 1) * kZetaCols <= n))
+    return;
   const int tid = threadIdx.x, c = tid & (kZetaCols - 1), rg = tid >> 4;
   G v[8];
 #pragma unroll
@@ -253,23 +269,25 @@ cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t str
 }
 
 template <typename G>
-static cudaError_t zeta(const Shape& s, G* g, cudaStream_t stream, int* launches) {
+static cudaError_t zeta(const Shape& s, G* g, int32_t* flags, cudaStream_t stream, int* launches) {
   const int tb = s.m < kZetaLowBits ? s.m : kZetaLowBits;
   const size_t low_blocks = (size_t)1 << (s.m - tb);
+  const size_t n = (size_t)1 << s.m;
   if (tb == kZetaLowBits)
-    k_zeta_low12<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g);
+    k_zeta_low12<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, n, flags);
   else
-    k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb);
+    k_zeta_low<<<(unsigned)low_blocks, kZetaThreads, 0, stream>>>(g, tb, n, flags);
   ++*launches;
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   for (int lo = tb; lo < s.m; lo += kZetaHighBits) {
     const int hb = (s.m - lo) < kZetaHighBits ? (s.m - lo) : kZetaHighBits;
-    const size_t blocks = ((size_t)1 << s.m) / (((size_t)1 << hb) * kZetaCols);
+    const size_t blocks = ((size_t)1 << s.m) / (hb == kZetaHighBits ? ((size_t)1 << hb) * kZetaCols
+                                                                      : (size_t)kZetaBlockEntries);
     if (hb == kZetaHighBits)
-      k_zeta_high8<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo);
+      k_zeta_high8<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, n, flags);
     else
-      k_zeta_high<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, hb);
+      k_zeta_high<<<(unsigned)blocks, kZetaThreads, 0, stream>>>(g, lo, hb, n, flags);
     ++*launches;
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
@@ -278,8 +296,8 @@ static cudaError_t zeta(const Shape& s, G* g, cudaStream_t stream, int* launches
 }
 
 cudaError_t launch_zeta(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
-  if (s.lean) return zeta(s, static_cast<unsigned int*>(g_table(s, ws)), stream, launches);
-  return zeta(s, static_cast<unsigned long long*>(g_table(s, ws)), stream, launches);
+  if (s.lean) return zeta(s, static_cast<unsigned int*>(g_table(s, ws)), ws.counters + 1, stream, launches);
+  return zeta(s, static_cast<unsigned long long*>(g_table(s, ws)), ws.counters + 1, stream, launches);
 }
 
 }  // namespace mpt

@@ -647,7 +647,7 @@ mpt_status trie_cost_lex(const int64_t* weights, int64_t n_chunks, int64_t m, co
   LexBuffers b{};
   carve_lex(a, s, n_chunks, 1, true, &b);
   char* mem = nullptr;
-  cudaError_t e = cudaMalloc(&mem, a.off);
+  cudaError_t e = device_alloc(reinterpret_cast<void**>(&mem), a.off);
   if (e != cudaSuccess) return cuda_status(e);
   Arena a2{mem, 0};
   carve_lex(a2, s, n_chunks, 1, true, &b);
@@ -685,7 +685,7 @@ mpt_status mpt_serve_order(int64_t n_chunks, int32_t m, const int64_t* seq_offse
   int32_t* d_arrival = a.take<int32_t>(m);
   int32_t* d_order = a.take<int32_t>(m);
   char* mem = nullptr;
-  cudaError_t e = cudaMalloc(&mem, a.off);
+  cudaError_t e = device_alloc(reinterpret_cast<void**>(&mem), a.off);
   if (e != cudaSuccess) return cuda_status(e);
   Arena a2{mem, 0};
   carve_lex(a2, s, n_chunks, 1, false, &b);
@@ -797,7 +797,7 @@ mpt_status mpt_cache_costs(const int64_t* weights, int64_t n_chunks, int32_t m, 
   carve(a, &b, &d_order, &d_aoff, &node_base, &node, &acc_id, &as, &aw, &asuf, &aowner, &prev_t, &next_t, &dist,
         &d_caps, &limit, &d_costs, &compulsory);
   char* mem = nullptr;
-  cudaError_t e = cudaMalloc(&mem, a.off);
+  cudaError_t e = device_alloc(reinterpret_cast<void**>(&mem), a.off);
   if (e != cudaSuccess) return cuda_status(e);
   Arena a2{mem, 0};
   carve(a2, &b, &d_order, &d_aoff, &node_base, &node, &acc_id, &as, &aw, &asuf, &aowner, &prev_t, &next_t, &dist,

@@ -183,6 +183,12 @@ const char* mpt_status_string(mpt_status s) {
 
 const char* mpt_last_error(const mpt_ctx* ctx) { return ctx ? ctx->err.c_str() : ""; }
 
+mpt_status mpt_build_info(int32_t* flags) {
+  if (!flags) return MPT_ERR_INVALID_ARG;
+  *flags = mpt::kBoundsChecked ? 1 : 0;
+  return MPT_OK;
+}
+
 mpt_status mpt_create(const int64_t* weights, int64_t n_chunks, const uint64_t* req_bits, int32_t m, mpt_ctx** out) {
   if (!weights || !req_bits || !out || n_chunks < 1 || n_chunks > INT32_MAX || m < 1) return MPT_ERR_INVALID_ARG;
   if (m > kMaxRequests) return MPT_ERR_TOO_LARGE;
@@ -306,7 +312,7 @@ mpt_status bind_workspace(mpt_ctx* c, void* d_workspace, size_t workspace_bytes,
       c->own_ws = nullptr;
       c->own_bytes = 0;
       c->resident = nullptr;
-      MPT_CK(cudaMalloc(&c->own_ws, need), "cudaMalloc(workspace)");
+      MPT_CK(mpt::device_alloc(&c->own_ws, need), "cudaMalloc(workspace)");
       c->own_bytes = need;
     }
     *base = static_cast<char*>(c->own_ws);
@@ -387,7 +393,7 @@ mpt_status run_back(mpt_ctx* c, const mpt::Workspace& ws, cudaStream_t stream, i
     char buf[128];
     std::snprintf(buf, sizeof(buf), "device consistency flags 0x%x", counters[1]);
     c->err = buf;
-    return MPT_ERR_INTERNAL;
+    return (counters[1] & mpt::kErrTimeout) ? MPT_ERR_TIMEOUT : MPT_ERR_INTERNAL;
   }
   *opt_out = opt;
   return MPT_OK;
@@ -653,7 +659,7 @@ mpt_status mpt_trie_cost(const int64_t* weights, int64_t n_chunks, int32_t m, co
     if (weights[x] <= 0) return MPT_ERR_INVALID_ARG;
   const size_t bw = (size_t)n_chunks * 8, bo = (size_t)(m + 1) * 8, bc = (size_t)(total > 0 ? total : 1) * 8;
   char* d = nullptr;
-  if (cudaMalloc(&d, bw + bo + bc + 8) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  if (mpt::device_alloc(reinterpret_cast<void**>(&d), bw + bo + bc + 8) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
   int64_t* dw = reinterpret_cast<int64_t*>(d);
   int64_t* doff = reinterpret_cast<int64_t*>(d + bw);
   int64_t* dch = reinterpret_cast<int64_t*>(d + bw + bo);

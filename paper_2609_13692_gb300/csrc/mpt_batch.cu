@@ -223,7 +223,7 @@ mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_byt
       if (b->own_ws) cudaFree(b->own_ws);
       b->own_ws = nullptr;
       b->own_bytes = 0;
-      if (cudaMalloc(&b->own_ws, need) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+      if (mpt::device_alloc(&b->own_ws, need) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
       b->own_bytes = need;
     }
     base = static_cast<char*>(b->own_ws);

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cstdlib>
 
 #include <cuda_runtime.h>
 
@@ -77,7 +78,99 @@ enum DeviceError : int {
   kErrBadSplit = 1,      // a split entry on the hierarchy is not a proper non-empty subset
   kErrLayoutCount = 2,   // the layout walk did not place every chunk occurrence
   kErrWorkspace = 4,     // a kernel saw a size outside what the workspace was carved for
+  kErrTimeout = 8,       // a bounded wait on a shared-memory barrier gave up
+  kErrBounds = 16,       // bounds-checked build: an index, window offset or split failed its check
 };
+
+// Bounds-checked build (-DMPT_BOUNDS; build(bounds=True)), the stand-in for a
+// memory checker: kernels test table indices, window offsets and split
+// entries, record kErrBounds in the device flags (mpt_solve then returns
+// MPT_ERR_INTERNAL) and skip the access.  In the default build MPT_BAD is
+// the constant false and every check compiles away.
+#ifdef MPT_BOUNDS
+#define MPT_BAD(flags, ok) (!(ok) && (atomicOr((flags), ::mpt::kErrBounds), true))
+constexpr bool kBoundsChecked = true;
+#else
+#define MPT_BAD(flags, ok) false
+constexpr bool kBoundsChecked = false;
+#endif
+
+// A split entry A of subset S (natural order) is well formed when S has at
+// most one request and A = 0, or A is a proper non-empty part of S that
+// holds S's lowest request (the Sec. 3.1 recurrence under the tie reading).
+__host__ __device__ __forceinline__ bool valid_split(uint32_t S, uint32_t A) {
+  if ((S & (S - 1u)) == 0) return A == 0;
+  return (A & ~S) == 0 && (A & S & (~S + 1u)) != 0 && A != S;
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory barriers (mbarrier) and bulk global -> shared copies.  Every
+// wait is bounded: after kWaitTries polls it gives up and reports false, and
+// the caller flags kErrTimeout instead of spinning on.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kWaitTries = 1u << 24;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+// Make the initialised barriers visible to the copy engine (the async proxy).
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(unsigned long long* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(unsigned long long* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Wait until the barrier's phase with this parity has completed; false if it
+// did not within kWaitTries polls.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kWaitTries; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+// One contiguous global -> shared copy by the copy engine; its bytes count
+// against the barrier's expected transaction bytes.  Both addresses 16-byte
+// aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_copy_g2s(void* smem_dst, const void* gmem_src, uint32_t bytes,
+                                              unsigned long long* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(smem_dst)), "l"(gmem_src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Device allocation of the library's own buffers.  Setting
+// MPT_FAIL_DEVICE_ALLOC=1 in the environment makes it fail as an exhausted
+// device would (cudaErrorMemoryAllocation), before any CUDA call, so that the
+// out-of-memory path of every entry point can be tested on any machine.
+// ---------------------------------------------------------------------------
+inline cudaError_t device_alloc(void** p, size_t bytes) {
+  const char* f = std::getenv("MPT_FAIL_DEVICE_ALLOC");
+  if (f && f[0] == '1') return cudaErrorMemoryAllocation;
+  return cudaMalloc(p, bytes);
+}
 
 // ---------------------------------------------------------------------------
 // Workspace carve-up (all offsets 256-byte aligned).

@@ -12,8 +12,10 @@ there is no fallback: loading fails loudly if it is missing.
 from __future__ import annotations
 
 import ctypes
+import os
 import itertools
 from dataclasses import dataclass
+from pathlib import Path
 from typing import Optional
 
 import numpy as np
@@ -44,7 +46,7 @@ EXPORTED = [
     "mpt_batch_results", "mpt_batch_tables", "mpt_batch_destroy", "mpt_greedy", "mpt_serve_order",
     "mpt_cache_costs", "mpt_layout_pinned", "mpt_solve_steps", "mpt_solve_begin", "mpt_solve_layers",
     "mpt_solve_end", "mpt_solve_resume", "mpt_set_tables", "mpt_tables32", "mpt_gather_bandwidth",
-    "mpt_alu_addmin_peak",
+    "mpt_alu_addmin_peak", "mpt_build_info",
 ]
 
 
@@ -81,7 +83,9 @@ _LIB = None
 
 
 def library_path() -> str:
-    return str(_build.LIB)
+    """The in-tree libmpt.so, or the build named by MPT_LIBRARY (for instance
+    the bounds-checked one from build(bounds=True))."""
+    return os.environ.get("MPT_LIBRARY") or str(_build.LIB)
 
 
 def load() -> ctypes.CDLL:
@@ -89,7 +93,7 @@ def load() -> ctypes.CDLL:
     global _LIB
     if _LIB is not None:
         return _LIB
-    path = _build.LIB
+    path = Path(library_path())
     if not path.exists():
         raise RuntimeError(f"{path} is missing: build the CUDA library first "
                            "(python -c 'import __graft_entry__ as g; g.build()')")
@@ -132,6 +136,7 @@ def load() -> ctypes.CDLL:
         "mpt_tables32": ([vp, ctypes.POINTER(vp), ctypes.POINTER(vp)], ctypes.c_int),
         "mpt_gather_bandwidth": ([i32, i64, vp, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
         "mpt_alu_addmin_peak": ([i64, vp, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+        "mpt_build_info": ([i32p], ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -689,3 +694,10 @@ def mpt_alu_addmin_peak(ops: int = 1 << 42, stream: Optional[int] = None) -> flo
     s = 0 if stream is None else int(stream)
     _check(load().mpt_alu_addmin_peak(int(ops), ctypes.c_void_p(s), ctypes.byref(out)), "mpt_alu_addmin_peak")
     return float(out.value)
+
+
+def mpt_build_info() -> dict:
+    """How the loaded library was built: {"bounds_checked": bool}."""
+    flags = ctypes.c_int32()
+    _check(load().mpt_build_info(ctypes.byref(flags)), "mpt_build_info")
+    return {"bounds_checked": bool(flags.value & 1)}
