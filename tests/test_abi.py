@@ -399,3 +399,43 @@ def test_binding_fails_loudly_without_the_library(tmp_path):
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True, timeout=120)
     assert r.returncode == 0, r.stdout + r.stderr
     assert "is missing" in r.stdout
+
+
+def test_device_allocation_failure(mpt, monkeypatch):
+    """With MPT_FAIL_DEVICE_ALLOC=1 every allocation the library makes for
+    itself fails as an exhausted device would: each entry point returns
+    MPT_ERR_OUT_OF_MEMORY before any CUDA call and writes no output, and the
+    context stays unsolved (no GPU needed)."""
+    import ctypes
+
+    lib = mpt.load()
+    inst = I.config(1)
+    ctx = mpt.mpt_create(inst.weights, inst.bits)
+    monkeypatch.setenv("MPT_FAIL_DEVICE_ALLOC", "1")
+    opt = ctypes.c_int64(-7)
+    assert lib.mpt_solve(ctx.handle, None, 0, None, ctypes.byref(opt)) == 4
+    assert opt.value == -7
+    offs = np.full(inst.m + 1, -7, dtype=np.int64)
+    chunks = np.full(64, -7, dtype=np.int64)
+    dfs = np.full(inst.m, -7, dtype=np.int32)
+    assert lib.mpt_layout(ctx.handle, offs.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                          chunks.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                          dfs.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))) == 7
+    assert (offs == -7).all() and (chunks == -7).all() and (dfs == -7).all()
+    assert lib.mpt_solve_begin(ctx.handle, None, 0, None) == 4
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_trie_cost(inst.weights, np.array([0, 1, 2], dtype=np.int64), np.array([0, 1], dtype=np.int64))
+    assert e.value.status == 4
+    reqs = [[0, 1, 2], [1, 2, 3], [2, 3, 4]]
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_greedy(np.arange(1, 6, dtype=np.int64), reqs)
+    assert e.value.status == 4
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_serve_order(5, reqs)
+    assert e.value.status == 4
+    with pytest.raises(mpt.MPTError) as e:
+        mpt.mpt_cache_costs(np.arange(1, 6, dtype=np.int64), reqs, [3, 10])
+    assert e.value.status == 4
+    b = mpt.mpt_batch_create(np.arange(1, 6, dtype=np.int64), *mpt.pack_batch([reqs, reqs[:2]]))
+    assert lib.mpt_batch_solve(b.handle, None, 0, None) == 4
+    monkeypatch.delenv("MPT_FAIL_DEVICE_ALLOC")
