@@ -189,7 +189,17 @@ def oracle_sample(inst, m_sub: int, threads: int = 0):
     return splits_per_solve(m_sub), dt, P
 
 
-RUNS_PER_LAYER = 16
+RUNS_PER_LAYER = 4
+_TABLES: dict = {}
+
+
+def stand_in_table(m: int) -> np.ndarray:
+    """A 2^m int64 table of ones, kept for the next sample of the same size
+    (the sampled work does not depend on the values, only on the table's size)."""
+    if m not in _TABLES:
+        _TABLES.clear()
+        _TABLES[m] = np.ones(1 << m, dtype=np.int64)
+    return _TABLES[m]
 
 
 def next_same_size(S: int) -> int:
@@ -220,7 +230,7 @@ def oracle_extrapolated(m: int, threads: int = 0, seed: int = 0, layer_splits: f
     import oracle
 
     P = threads or host_cores()
-    table = np.ones(1 << m, dtype=np.int64)  # stands in for F and w(I)
+    table = stand_in_table(m)  # stands in for F and w(I)
     rng = np.random.default_rng(seed)
     total, measured, modelled, tau = 0.0, [], [], None
     for k in range(2, m + 1):
@@ -263,7 +273,6 @@ def oracle_extrapolated(m: int, threads: int = 0, seed: int = 0, layer_splits: f
         oracle.intersection_weights(inst.weights, bits)
         wi = (time.perf_counter() - t0) * 2.0 ** (m - sub)
         total += wi
-    del table
     return {"m": m, "extrapolated_solve_s": total, "splits_per_s": splits_per_solve(m) / total, "threads": P,
             "layers_sampled": measured, "layers_priced_from_largest_sampled": modelled,
             "wI_walk_s": wi,
