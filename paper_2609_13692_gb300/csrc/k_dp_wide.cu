@@ -420,23 +420,31 @@ k_dp_tile_w(int L, int b, int kh, const Tab* __restrict__ wIr, const u64* __rest
           } while (s != 0);
         }
       }
-      for (int off = G >> 1; off > 0; off >>= 1) {
-        const u64 o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
-        best = o < best ? o : best;
-      }
-      if (active && r == 0) {
-        uint32_t ta = kh == 0 ? 0u : T;
-        if (kh >= 2) {
-          for (uint32_t it = 0; it < items; ++it) {
-            const size_t w = ((size_t)(tile * items + it) << b) | U;
-            const u64 k2 = pkey[w];
-            const uint32_t t2 = pta[w];
-            if (k2 < best || (k2 == best && t2 < ta)) {
-              best = k2;
-              ta = t2;
-            }
+      // the self pair's candidates carry Ta = T (kh = 0: none); the pair
+      // kernel's slots of this tile, one per block, are spread over the G
+      // lanes of the output; then the lexicographic (key, Ta) minimum of the
+      // group, in which the self pair wins ties only against larger Ta
+      uint32_t ta = kh == 0 ? 0u : T;
+      if (active && kh >= 2) {
+        for (uint32_t it = r; it < items; it += (uint32_t)G) {
+          const size_t w = ((size_t)(tile * items + it) << b) | U;
+          const u64 k2 = pkey[w];
+          const uint32_t t2 = pta[w];
+          if (k2 < best || (k2 == best && t2 < ta)) {
+            best = k2;
+            ta = t2;
           }
         }
+      }
+      for (int off = G >> 1; off > 0; off >>= 1) {
+        const u64 o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
+        const uint32_t ot = __shfl_xor_sync(0xFFFFFFFFu, ta, off);
+        if (o < best || (o == best && ot < ta)) {
+          best = o;
+          ta = ot;
+        }
+      }
+      if (active && r == 0) {
         const size_t idx = ((size_t)T << b) | U;
         int64_t f;
         uint32_t A;
