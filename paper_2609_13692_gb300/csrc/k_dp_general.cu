@@ -117,6 +117,7 @@ template <typename T>
 cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, int32_t* flags, cudaStream_t stream,
                        int* launches, int step_begin, int step_end) {
   if (step_end < 0 || step_end > s.m) step_end = s.m;
+  const int64_t sms = sm_count();
   cudaError_t err = cudaSuccess;
   if (step_begin <= 0 && step_end > 0) {
     k_dp_init<<<1, 32, 0, stream>>>(s.m, wI, F, split);
@@ -133,7 +134,7 @@ cudaError_t dp_general(const Shape& s, const T* wI, T* F, uint32_t* split, int32
       k_dp_layer_thread<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split, flags);
     } else {
       unsigned long long blocks = (count + (kThreads / 32) - 1) / (kThreads / 32);
-      if (blocks > 152ull * 16) blocks = 152ull * 16;
+      if (blocks > (unsigned long long)sms * 16) blocks = (unsigned long long)sms * 16;
       k_dp_layer_warp<<<(unsigned)blocks, kThreads, 0, stream>>>(s.m, k, count, wI, F, split, flags);
     }
     ++*launches;

@@ -464,6 +464,7 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
                o_bpar = take(M * 4), o_cbest = take(M * 8), o_mst = take(8);
   char* d = nullptr;
   if (device_alloc(reinterpret_cast<void**>(&d), off) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  const int64_t sms = sm_count();
   mpt_status st = MPT_OK;
   cudaError_t e = cudaSuccess;
   auto h2d = [&](size_t o, const void* h, size_t bytes) {
@@ -488,8 +489,8 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
     k_pair_weights<<<grid, 256, 0, stream>>>(m, I32(o_sig), I32(o_len), I64(o_w), U32(o_W));
     {
       // maximum spanning tree by Borůvka rounds (each at least halves the components)
-      const unsigned vb = (unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, 152 * 32);
-      const unsigned eb = (unsigned)std::min<int64_t>((m + 255) / 256, 152 * 8);
+      const unsigned vb = (unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, sms * 32);
+      const unsigned eb = (unsigned)std::min<int64_t>((m + 255) / 256, sms * 8);
       k_iota32<<<eb, 256, 0, stream>>>(m, I32(o_comp));
       k_bv_reset<<<eb, 256, 0, stream>>>(m, U64(o_cbest));
       int rounds = 1;
@@ -511,10 +512,10 @@ extern "C" mpt_status mpt_greedy(const int64_t* weights, int64_t n_chunks, int32
                                                            I32(o_nlen), I32(o_re));
     }
     k_greedy_tree<<<1, 1, 0, stream>>>(m, I32(o_ch), I32(o_par), I32(o_dep), I32(o_stk), I32(o_dfs));
-    const int64_t eblocks = std::min<int64_t>((std::max<int64_t>(occ, 1) + 255) / 256, 152 * 16);
+    const int64_t eblocks = std::min<int64_t>((std::max<int64_t>(occ, 1) + 255) / 256, sms * 16);
     k_greedy_emit<<<(unsigned)eblocks, 256, 0, stream>>>(m, I32(o_nsig), I32(o_nlen), I64(o_roff), I64(o_chunks),
                                                          I32(o_par), I32(o_dep), U64(o_keys));
-    k_greedy_rank<<<(unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, 152 * 16), 256, 0, stream>>>(
+    k_greedy_rank<<<(unsigned)std::min<int64_t>(((int64_t)m * 32 + 255) / 256, sms * 16), 256, 0, stream>>>(
         m, I64(o_roff), U64(o_keys), I64(o_perm));
     e = cudaGetLastError();
   }

@@ -253,7 +253,8 @@ __global__ void __launch_bounds__(kZetaThreads) k_zeta_high8(G* __restrict__ g, 
 
 cudaError_t launch_scatter(const Shape& s, const Workspace& ws, cudaStream_t stream, int* launches) {
   int64_t blocks = (s.n + kScatterThreads - 1) / kScatterThreads;
-  if (blocks > 152 * 16) blocks = 152 * 16;
+  const int64_t cap = sm_count() * 16;
+  if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   void* g = g_table(s, ws);
   if (s.lean)

@@ -247,8 +247,10 @@ int bits_for(uint64_t max_value) {
 // ---------------------------------------------------------------------------
 constexpr int kThreads = 256;
 
-unsigned grid_for(int64_t n, int64_t cap = 152 * 32) {
+// blocks of kThreads for n items, at most per_sm per SM (grid-stride loops)
+unsigned grid_for(int64_t n, int64_t per_sm = 32) {
   int64_t b = (n + kThreads - 1) / kThreads;
+  const int64_t cap = sm_count() * per_sm;
   if (b > cap) b = cap;
   return (unsigned)(b < 1 ? 1 : b);
 }
@@ -829,9 +831,9 @@ mpt_status mpt_cache_costs(const int64_t* weights, int64_t n_chunks, int32_t m, 
       if (e == cudaSuccess) {
         k_prev_next<<<grid_for(N), kThreads, 0, st>>>(keys, vals, N, aowner, prev_t, next_t);
         k_scan_limit<<<1, 32, 0, st>>>(d_caps, n_caps, b.trie, limit);
-        k_distance<<<grid_for(m * 32, 152 * 64), kDistThreads, 0, st>>>(m, d_aoff, prev_t, next_t, aw, asuf, limit,
+        k_distance<<<grid_for(m * 32, 64), kDistThreads, 0, st>>>(m, d_aoff, prev_t, next_t, aw, asuf, limit,
                                                                          dist);
-        k_cache_costs<<<grid_for(N, 152 * 8), kThreads, 0, st>>>(dist, aw, N, d_caps, n_caps, d_costs, compulsory);
+        k_cache_costs<<<grid_for(N, 8), kThreads, 0, st>>>(dist, aw, N, d_caps, n_caps, d_costs, compulsory);
         launches += 4;
         e = cudaGetLastError();
       }

@@ -161,6 +161,20 @@ __device__ __forceinline__ void bulk_copy_g2s(void* smem_dst, const void* gmem_s
 }
 
 // ---------------------------------------------------------------------------
+// Streaming multiprocessors of the current device, for the grid caps of
+// grid-stride loops (a host query of a few microseconds; 152 on a GB300,
+// also returned if the query fails, in which case the launch that follows
+// reports the error).
+// ---------------------------------------------------------------------------
+inline int64_t sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      sms < 1)
+    return 152;
+  return sms;
+}
+
+// ---------------------------------------------------------------------------
 // Device allocation of the library's own buffers.  Setting
 // MPT_FAIL_DEVICE_ALLOC=1 in the environment makes it fail as an exhausted
 // device would (cudaErrorMemoryAllocation), before any CUDA call, so that the
