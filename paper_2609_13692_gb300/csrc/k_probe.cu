@@ -103,7 +103,8 @@ extern "C" mpt_status mpt_alu_addmin_peak(int64_t ops, void* stream_ptr, double*
   const int64_t steps = (ops + threads * kAluPerStep - 1) / (threads * kAluPerStep);
   if (steps >= ((int64_t)1 << 28)) return MPT_ERR_INVALID_ARG;
   unsigned long long* sink = nullptr;
-  if (cudaMalloc(&sink, sizeof(unsigned long long)) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  if (device_alloc(reinterpret_cast<void**>(&sink), sizeof(unsigned long long)) != cudaSuccess)
+    return MPT_ERR_OUT_OF_MEMORY;
   cudaEvent_t a = nullptr, b = nullptr;
   mpt_status status = MPT_OK;
   float ms = 0.f;
@@ -141,7 +142,7 @@ extern "C" mpt_status mpt_gather_bandwidth(int32_t log2_entries, int64_t loads, 
   int64_t per_thread = (loads + threads - 1) / threads;
   per_thread = (per_thread + kProbeUnroll - 1) / kProbeUnroll * kProbeUnroll;
   char* mem = nullptr;
-  if (cudaMalloc(&mem, n * 8 + 256) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
+  if (device_alloc(reinterpret_cast<void**>(&mem), n * 8 + 256) != cudaSuccess) return MPT_ERR_OUT_OF_MEMORY;
   int64_t* table = reinterpret_cast<int64_t*>(mem);
   unsigned long long* sink = reinterpret_cast<unsigned long long*>(mem + n * 8);
   cudaEvent_t a = nullptr, b = nullptr;
