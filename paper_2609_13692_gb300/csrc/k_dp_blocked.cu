@@ -591,22 +591,50 @@ k_dp_tile(int L, int b, int kh, const Tab* __restrict__ wIr, const unsigned long
 // Rows are finished level by level in |s1|, so every row read is final.
 constexpr int kRowsThreads = 96;
 constexpr int kBestWords = (1 << kB) + kRows;  // per-output arrays, rows 33 words apart
-constexpr int kRowsSmemBytes = (2 * kWin + 2 * kBestWords) * (int)sizeof(uint32_t);
+// With kZcGlobal, tile 0's complement rows are read from global memory (the
+// same 16 KB for every block, so they stay in L1) instead of a shared copy:
+// 52 KB of shared memory per block instead of 70, four blocks per SM instead
+// of three.  That pays on long layers (m >= 26: 7.95 vs 8.37 ms of tile
+// stage at m = 28) but not on short ones (m = 24: 1.22 vs 1.19 ms).
+constexpr int rows_smem_bytes(bool zc_global) {
+  return ((zc_global ? 1 : 2) * kWin + 2 * kBestWords) * (int)sizeof(uint32_t);
+}
+constexpr int kZcGlobalMinL = 14;
 
 // Word of output U = (s1, s2) in a per-output array: rows are 33 words apart,
 // so threads that hold different rows and the same s2 hit different banks.
 __device__ __forceinline__ uint32_t best_word(uint32_t U) { return U + (U >> kB2); }
 
-template <typename Tab>
+// Row r of tile 0's complement form (Gc[0 .. 4095] is written by the tile-0
+// launch and only read here): from the shared copy, or from global memory.
+template <bool kZcGlobal>
+__device__ __forceinline__ void load_zrow(uint32_t (&v)[kRow], const uint32_t* zc, const uint32_t* __restrict__ Gc,
+                                          uint32_t r) {
+  if constexpr (kZcGlobal) {
+    const uint4* q = reinterpret_cast<const uint4*>(Gc + r * kRow);
+#pragma unroll
+    for (int c = 0; c < kRow / 4; ++c) {
+      const uint4 t = __ldg(q + c);
+      v[4 * c] = t.x;
+      v[4 * c + 1] = t.y;
+      v[4 * c + 2] = t.z;
+      v[4 * c + 3] = t.w;
+    }
+  } else {
+    load_row(v, zc + row_pos(r) * kRowStride);
+  }
+}
+
+template <typename Tab, bool kZcGlobal>
 __global__ void __launch_bounds__(kRowsThreads)
 k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long long* __restrict__ partial,
                uint32_t* __restrict__ Gp, uint32_t* __restrict__ Gc, uint32_t* __restrict__ split_rot,
                int32_t* __restrict__ flags) {
   extern __shared__ __align__(16) uint32_t smem[];
-  uint32_t* cur = smem;               // this tile, F << kB, padded rows
-  uint32_t* zc = smem + kWin;         // tile 0, complement form, padded rows
-  uint32_t* bkey = smem + 2 * kWin;   // best key per output so far
-  uint32_t* bsplit = bkey + kBestWords;  // its Ta; after finishing, the split A
+  uint32_t* cur = smem;                                   // this tile, F << kB, padded rows
+  uint32_t* zc = smem + kWin;                             // tile 0, complement form, padded rows (shared copy)
+  uint32_t* bkey = smem + (kZcGlobal ? 1 : 2) * kWin;     // best key per output so far
+  uint32_t* bsplit = bkey + kBestWords;                   // its Ta; after finishing, the split A
   constexpr uint32_t kMask = (1u << kB) - 1u;
 
   const uint32_t tile = blockIdx.x;
@@ -614,10 +642,12 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
   const size_t tbase = (size_t)T << kB;
   if (MPT_BAD(flags, tile < c_binom.v[L][kh] && T < (1u << L) && __popc(T) == kh)) return;
 
-  for (int c = threadIdx.x; c < (1 << (kB - 2)); c += kRowsThreads) {
-    const int row = c >> (kB2 - 2), k = c & ((1 << (kB2 - 2)) - 1);
-    *reinterpret_cast<uint4*>(zc + row_pos((uint32_t)row) * kRowStride + 4 * k) =
-        *reinterpret_cast<const uint4*>(Gc + 4 * c);
+  if constexpr (!kZcGlobal) {
+    for (int c = threadIdx.x; c < (1 << (kB - 2)); c += kRowsThreads) {
+      const int row = c >> (kB2 - 2), k = c & ((1 << (kB2 - 2)) - 1);
+      *reinterpret_cast<uint4*>(zc + row_pos((uint32_t)row) * kRowStride + 4 * k) =
+          *reinterpret_cast<const uint4*>(Gc + 4 * c);
+    }
   }
   for (int u = threadIdx.x; u < (1 << kB); u += kRowsThreads) {
     const unsigned long long pv = kh >= 2 ? partial[((size_t)tile << kB) | (uint32_t)u] : ~0ull;
@@ -665,7 +695,7 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
           if (a1 != s1) {
             uint32_t x[kRow], y[kRow];
             load_row(x, cur + row_pos(a1) * kRowStride);
-            load_row(y, zc + row_pos(s1 ^ a1) * kRowStride);
+            load_zrow<kZcGlobal>(y, zc, Gc, s1 ^ a1);
             conv_rows(acc, x, y);
           }
           sub = (sub - freem) & freem;
@@ -690,7 +720,7 @@ k_dp_tile_rows(int L, int kh, const Tab* __restrict__ wIr, const unsigned long l
     if (finisher) {
       const uint32_t s1 = s1f;
       uint32_t z[kRow], c[kRow];
-      load_row(z, zc + row_pos(0) * kRowStride);
+      load_zrow<kZcGlobal>(z, zc, Gc, 0);
 #pragma unroll
       for (int s2 = 0; s2 < kRow; ++s2) {
         uint32_t key = 0xFFFFFFFFu;
@@ -787,9 +817,17 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
     // host-side call, negligible against a solve), so that any device works
     cudaError_t e = cudaFuncSetAttribute(k_dp_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmemBytes);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_dp_tile_rows<int64_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int64_t, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             rows_smem_bytes(false));
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_dp_tile_rows<int32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRowsSmemBytes);
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int32_t, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             rows_smem_bytes(false));
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int64_t, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             rows_smem_bytes(true));
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_dp_tile_rows<int32_t, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             rows_smem_bytes(true));
     if (e != cudaSuccess) return e;
   }
   const int b = s.b, L = s.L;
@@ -832,12 +870,17 @@ cudaError_t launch_dp_blocked(const Shape& s, const Workspace& ws, cudaStream_t 
                                                   ws.counters + 1);
     } else {
       const unsigned long long* part = kh >= 2 ? ws.partial : nullptr;
-      if (s.lean)
-        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.fw_rot, part, ws.Gp,
-                                                                                  ws.Gc, ws.split_rot, ws.counters + 1);
-      else
-        k_dp_tile_rows<<<(unsigned)tiles, kRowsThreads, kRowsSmemBytes, stream>>>(L, kh, ws.wI_rot, part, ws.Gp,
-                                                                                  ws.Gc, ws.split_rot, ws.counters + 1);
+      const bool zg = L >= kZcGlobalMinL;
+      const int sm_bytes = rows_smem_bytes(zg);
+      if (s.lean) {
+        auto k = zg ? k_dp_tile_rows<int32_t, true> : k_dp_tile_rows<int32_t, false>;
+        k<<<(unsigned)tiles, kRowsThreads, sm_bytes, stream>>>(L, kh, ws.fw_rot, part, ws.Gp, ws.Gc, ws.split_rot,
+                                                               ws.counters + 1);
+      } else {
+        auto k = zg ? k_dp_tile_rows<int64_t, true> : k_dp_tile_rows<int64_t, false>;
+        k<<<(unsigned)tiles, kRowsThreads, sm_bytes, stream>>>(L, kh, ws.wI_rot, part, ws.Gp, ws.Gc, ws.split_rot,
+                                                               ws.counters + 1);
+      }
     }
     if (timing && timing->tile_ev) cudaEventRecord(timing->tile_ev[2 * timing->tile_launches + 1], stream);
     if (timing) timing->tile_launches++;
