@@ -79,8 +79,9 @@ static_assert((kRowStride * 4) % 16 == 0, "padded rows start on 16-byte boundari
 // in registers across all pairs (running best key and Ta), merged with the
 // other tasks of the row once, at the end.
 // Shared rows: the 29 rows with <= 2 bits and those five -- 34 rows, 139
-// units per pair.  They run as whole-warp "slots" of 32 units (lane l takes
-// unit 32 i + l of slot i): 4 full slots and one of 11 lanes per pair.  The
+// units per pair.  They run as whole-warp "slots" of 32 units: 4 full slots
+// and one of 11 lanes per pair, the units of one row spread over the slots
+// (at most two lanes of a slot flush into one bank; see make_plan).  The
 // slots of pair q go to warps (5 (q mod 8) + i) mod 8, so over 8 pairs every
 // warp runs exactly 5 slots, and each sub-partition 128 register units plus
 // 10 slots against 136.7 units of work (not 144, as one extra unit per warp
@@ -143,12 +144,34 @@ constexpr PairPlan make_plan() {
     for (uint32_t v = 0; v < (1u << q); ++v) pl.task[n++] = s1 | (deposit_c(v, lowbits) << 8) | (freem << 16);
   }
   for (int i = 0; i < kExtraSlots * 32; ++i) pl.extra[i] = 0xFFFFFFFFu;
-  for (int ri = 0; ri < nr; ++ri) {
-    const uint32_t s1 = pl.srow[ri];
-    for (uint32_t k = 0; k < (1u << popc_c(s1)); ++k) {
-      const uint32_t a1 = deposit_c(k, s1);
-      pl.extra[ne] = s1 | (a1 << 8) | ((uint32_t)ri << 16);
-      ++ne;
+  // Shared-row units are placed so that few lanes of one slot flush into the
+  // same bank: rows in decreasing unit count, each unit into the slot that
+  // holds the fewest units of rows congruent to its own mod 32 (the bank of
+  // word i of shared row r is (r + i) mod 32), then the emptiest slot.
+  int fill[kExtraSlots] = {};
+  for (int p = kB1; p >= 0; --p) {
+    for (int ri = 0; ri < nr; ++ri) {
+      const uint32_t s1 = pl.srow[ri];
+      if (popc_c(s1) != p) continue;
+      for (uint32_t k = 0; k < (1u << p); ++k) {
+        int best = -1, best_same = 0, best_room = 0;
+        for (int sl = 0; sl < kExtraSlots; ++sl) {
+          const int cap = kExtraUnits - 32 * sl < 32 ? kExtraUnits - 32 * sl : 32;
+          const int room = cap - fill[sl];
+          if (room <= 0) continue;
+          int same = 0;
+          for (int l = 0; l < fill[sl]; ++l)
+            if ((int)((pl.extra[32 * sl + l] >> 16) & 0xFFu) % 32 == ri % 32) ++same;
+          if (best < 0 || same < best_same || (same == best_same && room > best_room)) {
+            best = sl;
+            best_same = same;
+            best_room = room;
+          }
+        }
+        const uint32_t a1 = deposit_c(k, s1);
+        pl.extra[32 * best + fill[best]++] = s1 | (a1 << 8) | ((uint32_t)ri << 16);
+        ++ne;
+      }
     }
   }
   pl.ntask = n;
@@ -157,7 +180,24 @@ constexpr PairPlan make_plan() {
   return pl;
 }
 
+// Largest number of lanes of one slot whose rows share a bank class (rows
+// congruent mod 32 put word i in the same bank).
+constexpr int max_slot_bank_share(const PairPlan& pl) {
+  int worst = 0;
+  for (int sl = 0; sl < kExtraSlots; ++sl)
+    for (int cls = 0; cls < 32; ++cls) {
+      int n = 0;
+      for (int l = 0; l < 32; ++l) {
+        const uint32_t e = pl.extra[32 * sl + l];
+        if (e != 0xFFFFFFFFu && (int)((e >> 16) & 0xFFu) % 32 == cls) ++n;
+      }
+      worst = n > worst ? n : worst;
+    }
+  return worst;
+}
+
 constexpr PairPlan kPlanHost = make_plan();
+static_assert(max_slot_bank_share(kPlanHost) <= 2, "shared-row units spread over the slots");
 static_assert(kPlanHost.ntask == kPairThreads, "register tasks must fill the block");
 static_assert(kPlanHost.nsrow == kSharedRows, "shared row count");
 static_assert(kPlanHost.nextra == kExtraUnits, "extra units");
