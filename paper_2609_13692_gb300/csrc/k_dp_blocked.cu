@@ -54,7 +54,7 @@ constexpr int kSharedWords = kSharedRows * kSharedStride;
 constexpr int kSharedOwned = (kSharedOut + kPairThreads - 1) / kPairThreads;
 constexpr int kExtraUnits = 139;           // shared-row units of one pair
 constexpr int kExtraSlots = (kExtraUnits + 31) / 32;  // whole-warp slots per pair: 4 full, 1 of 11 lanes
-constexpr int kSlotCycle = 8;              // pairs after which the slot-to-warp rotation repeats
+constexpr int kPartial = kExtraUnits - 32 * (kExtraSlots - 1);  // lanes of the partial slot
 constexpr int kPairSmemWords = kRing * 2 * kWin + kRing * kSharedWords + kRow * kPairThreads;
 constexpr int kPairSmemBytes = kPairSmemWords * (int)sizeof(uint32_t) + 3 * kRing * 8;
 constexpr int kMinPairsPerItem = 16;
@@ -63,7 +63,8 @@ constexpr int kMaxTileBits = 12;
 
 static_assert(kRing * 2 * kWin * (int)sizeof(uint32_t) >= (1 << kB) * 8, "merge buffer must fit in the windows");
 static_assert((kRing * 2 * kWin + kRing * kSharedWords + kRow * kPairThreads) % 2 == 0, "8-byte aligned barriers");
-static_assert(kExtraSlots * 32 >= kExtraUnits && kExtraSlots <= kSlotCycle, "extra slots per pair");
+static_assert(kExtraSlots == 5 && 2 * kPartial <= 32, "4 full slots per pair; two partial slots fill one warp");
+static_assert(kPairThreads == 256, "the slot rotation (9 slots per two pairs over 8 warps) assumes 8 warps");
 static_assert((kRowStride * 4) % 16 == 0, "padded rows start on 16-byte boundaries");
 
 // ---------------------------------------------------------------------------
@@ -82,11 +83,13 @@ static_assert((kRowStride * 4) % 16 == 0, "padded rows start on 16-byte boundari
 // units per pair.  They run as whole-warp "slots" of 32 units: 4 full slots
 // and one of 11 lanes per pair, the units of one row spread over the slots
 // (at most two lanes of a slot flush into one bank; see make_plan).  The
-// slots of pair q go to warps (5 (q mod 8) + i) mod 8, so over 8 pairs every
-// warp runs exactly 5 slots, and each sub-partition 128 register units plus
-// 10 slots against 136.7 units of work (not 144, as one extra unit per warp
-// and pair would take).  A slot's 32 minima go to the pair's shared array
-// with atomicMin; owner threads fold that array into registers one pair later.
+// partial slots of pairs 2h and 2h + 1 run as one slot of 22 lanes, so two
+// pairs have 9 slots, numbered 9h .. 9h + 8 and run by warp (number mod 8):
+// over 16 pairs every warp runs exactly 9 slots, and each sub-partition 256
+// register unit-times plus 18 slots against 273.4 units of work (0.2 % idle
+// lanes; 1 % with a partial slot per pair).  A slot's 32 minima go to the
+// pair's shared array with atomicMin; owner threads fold that array into
+// registers one pair later.
 // ---------------------------------------------------------------------------
 __host__ __device__ constexpr int popc_c(uint32_t v) {
   int c = 0;
@@ -315,9 +318,13 @@ __device__ __forceinline__ bool fold_pair(uint32_t jj, uint32_t Ta_jj, uint32_t*
 // block-wide barrier.  Pair q lives in slot q mod kRing.  At the start of
 // step q every warp waits until all threads have folded pair q + 1 - kRing
 // ("folded"), and its threads start their copies of pair q + 1 into that
-// slot; then they wait for pair q's copies ("full"), run their units, arrive
-// on "consumed", fold the previous pair's shared-row minima into their
-// running bests (in pair order) and arrive on "folded".  Every wait is
+// slot; then they wait for pair q's copies ("full"), run their slot and
+// units, arrive on "consumed", fold the previous pair's shared-row minima
+// into their running bests (in pair order) and arrive on "folded".  The warp
+// that runs the merged partial slot of pairs q - 1 and q arrives on
+// "consumed" of pair q - 1 only after that slot, at step q (before it, no
+// thread can fold pair q - 1, whose fold follows the units of step q, and no
+// slot of pair q - 1 is refilled).  Every wait is
 // bounded; one that gives up sets kErrTimeout in *flags and the thread stops
 // (after waiting, bounded again, for the copies it started), so the launch
 // ends with its results marked invalid.
@@ -368,10 +375,14 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
   const uint32_t b2 = freem ^ b0 ^ b1;
   const uint32_t pos_fixed = (uint32_t)row_pos(fixed), pos_s1 = (uint32_t)row_pos(s1);
   const uint32_t pb0 = (uint32_t)row_pos(b0), pb1 = (uint32_t)row_pos(b1), pb2 = (uint32_t)row_pos(b2);
-  // this lane's unit in each of the kExtraSlots slots of a pair
+  // this lane's unit in each of the kExtraSlots slots of a pair, and in the
+  // merged partial slot (lanes 0..kPartial-1: the earlier pair's partial
+  // slot, the next kPartial lanes the later pair's)
   uint32_t ext[kExtraSlots];
 #pragma unroll
   for (int i = 0; i < kExtraSlots; ++i) ext[i] = c_plan.extra[32 * i + (int)lane];
+  const uint32_t ext_part = __shfl_sync(0xFFFFFFFFu, ext[kExtraSlots - 1], lane < (uint32_t)kPartial ? lane : lane - kPartial);
+  const uint32_t ext_merged = lane < 2u * kPartial ? ext_part : 0xFFFFFFFFu;
 
   if (threadIdx.x == 0) {
     for (int c = 0; c < kRing; ++c) {
@@ -422,10 +433,46 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
     const uint32_t* X = smem + 2 * c * kWin;
     const uint32_t* Y = X + kWin;
     {
+      uint32_t acc[kRow];
+      // This warp's shared-row slot of the step, if the rotation gives it
+      // one.  Pairs 2h and 2h + 1 have 9 slots between them, numbered 9h ..
+      // 9h + 8 and run by warps (number mod 8): the full slots of pair 2h at
+      // step 2h, then those of pair 2h + 1 and the merged partial slot of
+      // both at step 2h + 1.  A last pair without a partner runs its own
+      // partial slot.  The warp of the merged slot holds back its "consumed"
+      // arrival for pair 2h until that slot has flushed.
+      const uint32_t h = j >> 1;
+      const bool odd = (j & 1u) != 0;
+      const uint32_t base = odd ? 9u * h + 4u : 9u * h;
+      const uint32_t nslots = odd || j + 1 == npairs ? (uint32_t)kExtraSlots : (uint32_t)kExtraSlots - 1u;
+      const uint32_t si = (warp + 8u - base % 8u) % 8u;
+      if (si < nslots) {
+        uint32_t e = ext[0];
+#pragma unroll
+        for (int i = 1; i < kExtraSlots; ++i)
+          if (si == (uint32_t)i) e = ext[i];
+        const bool merged = odd && si == (uint32_t)kExtraSlots - 1u;
+        uint32_t cs = c;
+        if (merged) {
+          e = ext_merged;
+          if (lane < (uint32_t)kPartial) cs = (j - 1) % kRing;
+        }
+        if (e != 0xFFFFFFFFu) {
+          const uint32_t es1 = e & 0xFFu, ea1 = (e >> 8) & 0xFFu, erow = (e >> 16) & 0xFFu;
+          const uint32_t* Xs = smem + 2 * cs * kWin;
+          uint32_t x[kRow], y[kRow];
+          load_row(x, Xs + row_pos(ea1) * kRowStride);
+          load_row(y, Xs + kWin + row_pos(es1 ^ ea1) * kRowStride);
+          conv_rows<true>(acc, x, y);
+          uint32_t* row = smin + cs * kSharedWords + erow * kSharedStride;
+#pragma unroll
+          for (int i = 0; i < kRow; ++i) atomicMin(&row[i], acc[i]);
+        }
+        if (merged) mbar_arrive(&consumed[(j - 1) % kRing]);
+      }
       // The 8 units of the task visit a1 = fixed | sub with sub running over the
       // subsets of its 3 free bits in Gray-code order; row_pos is linear over
       // GF(2), so each step changes the row position by one XOR.
-      uint32_t acc[kRow];
       uint32_t pa = pos_fixed;
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
@@ -444,26 +491,9 @@ k_dp_pairs(const uint32_t* __restrict__ Gp, const uint32_t* __restrict__ Gc, uns
         bk[i] = __vibmin_u32(bk[i], acc[i], &keep);
         if (!keep) sbest_t[i * kPairThreads + threadIdx.x] = Ta;
       }
-      // this warp's shared-row slot of the pair, if the rotation gives it one
-      const uint32_t slot = (warp + (uint32_t)kSlotCycle - (5u * (j % kSlotCycle)) % kSlotCycle) % kSlotCycle;
-      if (slot < (uint32_t)kExtraSlots) {
-        uint32_t e = ext[0];
-#pragma unroll
-        for (int i = 1; i < kExtraSlots; ++i)
-          if (slot == (uint32_t)i) e = ext[i];
-        if (e != 0xFFFFFFFFu) {
-          const uint32_t es1 = e & 0xFFu, ea1 = (e >> 8) & 0xFFu, erow = (e >> 16) & 0xFFu;
-          uint32_t x[kRow], y[kRow];
-          load_row(x, X + row_pos(ea1) * kRowStride);
-          load_row(y, Y + row_pos(es1 ^ ea1) * kRowStride);
-          conv_rows<true>(acc, x, y);
-          uint32_t* row = smin + c * kSharedWords + erow * kSharedStride;
-#pragma unroll
-          for (int i = 0; i < kRow; ++i) atomicMin(&row[i], acc[i]);
-        }
-      }
     }
-    mbar_arrive(&consumed[c]);
+    // pair j's arrival, unless this warp runs the merged slot of j and j + 1
+    if (!((j & 1u) == 0 && j + 1 < npairs && warp == (j >> 1) % 8u)) mbar_arrive(&consumed[c]);
     if (j >= 1 && !fold_pair(j - 1, prev_Ta, smin, consumed, folded, sbk, sbt)) {
       ok = false;
       break;
