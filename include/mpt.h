@@ -247,9 +247,14 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
 mpt_status mpt_batch_workspace_bytes(const mpt_batch* b, size_t* bytes);
 
 /* Solve every instance (Sec. 3.1 recurrence and Thm 1 layout per instance).
- * d_workspace as in mpt_solve (NULL: the library allocates and keeps one);
- * all work on `stream`, synchronised before return.  Errors: INVALID_ARG,
- * WORKSPACE_TOO_SMALL, OUT_OF_MEMORY, CUDA, INTERNAL. */
+ * d_workspace as in mpt_solve (NULL: the library allocates and keeps one).
+ * Uploads and downloads run on `stream`; the per-size grids run on four
+ * side streams of the batch object (created on the first solve, on the
+ * device current then, and released by mpt_batch_destroy), forked from
+ * `stream` after the uploads and joined back to it before the downloads;
+ * `stream` is synchronised before return, so no work of the call outlives
+ * it.  If the side streams cannot be created the grids run on `stream`.
+ * Errors: INVALID_ARG, WORKSPACE_TOO_SMALL, OUT_OF_MEMORY, CUDA, INTERNAL. */
 mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_bytes, void* stream);
 
 /* Results of the last solve, host outputs (any may be NULL):

@@ -1,6 +1,6 @@
 // C ABI of the batched small-instance solver (include/mpt.h, mpt_batch_*):
-// argument checks, workspace carve-up and one k_batch_solve launch per
-// instance size m.
+// argument checks, workspace carve-up and one grid per instance size m, the
+// grids on side streams forked from the caller's stream.
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
@@ -46,11 +46,60 @@ struct mpt_batch {
   const uint32_t* d_split = nullptr;
   void* own_ws = nullptr;
   size_t own_bytes = 0;
+  // side streams for the per-size launches (created on first use, on the
+  // device current then), with the events that fork them from and join them
+  // to the caller's stream
+  int side_device = -1;
+  std::vector<cudaStream_t> side;
+  std::vector<cudaEvent_t> join;
+  cudaEvent_t fork = nullptr;
 };
 
 namespace {
 
 constexpr int kBatchMaxM = 13;
+constexpr int kBatchSideStreams = 4;
+
+void release_side_streams(mpt_batch* b) {
+  for (cudaStream_t st : b->side) cudaStreamDestroy(st);
+  for (cudaEvent_t ev : b->join) cudaEventDestroy(ev);
+  if (b->fork) cudaEventDestroy(b->fork);
+  b->side.clear();
+  b->join.clear();
+  b->fork = nullptr;
+  b->side_device = -1;
+}
+
+// The side streams of the current device, created on first use; false when
+// they cannot be made (the launches then stay on the caller's stream).
+bool side_streams(mpt_batch* b) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (b->side_device == dev) return true;
+  release_side_streams(b);
+  if (cudaEventCreateWithFlags(&b->fork, cudaEventDisableTiming) != cudaSuccess) {
+    b->fork = nullptr;
+    return false;
+  }
+  for (int i = 0; i < kBatchSideStreams; ++i) {
+    cudaStream_t st = nullptr;
+    cudaEvent_t ev = nullptr;
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) break;
+    if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) {
+      cudaStreamDestroy(st);
+      break;
+    }
+    b->side.push_back(st);
+    b->join.push_back(ev);
+  }
+  if ((int)b->side.size() < kBatchSideStreams) {
+    release_side_streams(b);
+    cudaGetLastError();
+    return false;
+  }
+  b->side_device = dev;
+  return true;
+}
 constexpr int kBatchMaxOcc = 2048;
 constexpr int64_t kBatchSumLimit = (int64_t)1 << 62;
 
@@ -252,16 +301,40 @@ mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_byt
   h2d(c.tab_off, b->tab_off.data(), (B + 1) * 8);
   h2d(c.inst_list, b->inst_list.data(), B * 4);
   h2d(c.flags, b->flags.data(), B);
-  for (int m = 1; m <= kBatchMaxM && e == cudaSuccess; ++m) {
+  // One grid per instance size, largest first.  The grids write disjoint
+  // instances, so they run on side streams forked from the caller's stream
+  // after the uploads and joined back before the downloads: the short grids
+  // of small sizes then fill the SMs that the long ones leave idle.
+  const bool forked = e == cudaSuccess && side_streams(b);
+  if (forked) {
+    e = cudaEventRecord(b->fork, stream);
+    for (int i = 0; i < kBatchSideStreams && e == cudaSuccess; ++i) e = cudaStreamWaitEvent(b->side[(size_t)i], b->fork, 0);
+  }
+  int next_side = 0;
+  for (int m = kBatchMaxM; m >= 1 && e == cudaSuccess; --m) {
     const int64_t g0 = b->group_start[(size_t)m], gr = b->group_rows_end[(size_t)m],
                   g1 = b->group_start[(size_t)m + 1];
+    if (g1 == g0) continue;
     const int cap = b->group_occ_cap[(size_t)m];
+    cudaStream_t st = forked ? b->side[(size_t)(next_side++ % kBatchSideStreams)] : stream;
     if (gr > g0)
       e = mpt::launch_batch_rows((int)(gr - g0), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                                 c.inst_list + g0, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+                                 c.inst_list + g0, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, st);
     if (e == cudaSuccess && g1 > gr)
       e = mpt::launch_batch((int)(g1 - gr), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                            c.inst_list + gr, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, stream);
+                            c.inst_list + gr, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, st);
+  }
+  if (forked) {
+    // join every side stream, also after a failed launch, so that no work
+    // of this call runs on after it returns
+    for (int i = 0; i < kBatchSideStreams; ++i) {
+      cudaError_t ej = cudaEventRecord(b->join[(size_t)i], b->side[(size_t)i]);
+      if (ej == cudaSuccess) ej = cudaStreamWaitEvent(stream, b->join[(size_t)i], 0);
+      if (ej != cudaSuccess) {
+        cudaStreamSynchronize(b->side[(size_t)i]);
+        if (e == cudaSuccess) e = ej;
+      }
+    }
   }
   d2h(b->opt.data(), c.opt, B * 8);
   d2h(b->status.data(), c.status, B * 4);
@@ -299,6 +372,7 @@ mpt_status mpt_batch_tables(const mpt_batch* b, const int64_t** d_F, const uint3
 void mpt_batch_destroy(mpt_batch* b) {
   if (!b) return;
   if (b->own_ws) cudaFree(b->own_ws);
+  release_side_streams(b);
   delete b;
 }
 
