@@ -60,10 +60,16 @@ namespace {
 constexpr int kBatchMaxM = 13;
 constexpr int kBatchSideStreams = 4;
 
+// Destroys the side streams and events on the device they were made on,
+// restoring the caller's current device.
 void release_side_streams(mpt_batch* b) {
+  int cur = -1;
+  const bool switch_dev = b->side_device >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != b->side_device &&
+                          cudaSetDevice(b->side_device) == cudaSuccess;
   for (cudaStream_t st : b->side) cudaStreamDestroy(st);
   for (cudaEvent_t ev : b->join) cudaEventDestroy(ev);
   if (b->fork) cudaEventDestroy(b->fork);
+  if (switch_dev) cudaSetDevice(cur);
   b->side.clear();
   b->join.clear();
   b->fork = nullptr;
