@@ -628,7 +628,8 @@ def run_batch(args):
     torch.cuda.set_device(0)
     if not B.LIB.exists():
         B.build()
-    weights, groups = batch_groups(args.batch_size, seed=0)
+    m_lo, m_hi = (int(v) for v in args.batch_sizes.split("-"))
+    weights, groups = batch_groups(args.batch_size, seed=0, m_lo=m_lo, m_hi=m_hi)
     ir, ro, ch = mpt.pack_batch(groups)
     ms = np.diff(ir)
     splits = int(sum((3 ** int(m) + 1) // 2 - 2 ** int(m) for m in ms))
@@ -646,7 +647,7 @@ def run_batch(args):
     e1.record(stream)
     torch.cuda.synchronize()
     ms_step = e0.elapsed_time(e1) / args.steps
-    line = {"mode": "batch", "metric": "exact solves of request groups (m = 8..13, k = 8) per second",
+    line = {"mode": "batch", "metric": f"exact solves of request groups (m = {m_lo}..{m_hi}, k = 8) per second",
             "value": len(groups) / (ms_step / 1000.0), "unit": "instances/s", "splits_per_s": splits / (ms_step / 1000.0),
             "ms_per_step": ms_step, "steps": args.steps, "warmup": args.warmup, "batch": len(groups),
             "splits_per_step": splits, "note": "timed region includes the per-step input upload and result download"}
@@ -797,6 +798,7 @@ def main():
                          "greedy: agglomerative hierarchy on a trace-sized request set; "
                          "cache: serving order and radix-cache simulator timings on a request stream")
     ap.add_argument("--batch-size", type=int, default=20000)
+    ap.add_argument("--batch-sizes", default="8-13", help="request-count range of the batched groups, e.g. 14-15")
     ap.add_argument("--greedy-m", type=int, default=3000)
     ap.add_argument("--cache-m", type=int, default=0,
                     help="cache mode: requests in a scaled stream (default: the 2,921-request stream)")

@@ -1,5 +1,6 @@
-// Batched exact solve of many small instances (m <= 13 requests each), one
-// block per instance with every table in shared memory.
+// Batched exact solve of many small instances (m <= 15 requests each), one
+// block per instance with every table in shared memory: the row-blocked
+// kernel for packed keys up to m = 13, the per-subset kernel otherwise.
 //
 // This is the paper's own use of the exact recurrence (Sec. 6.2: 72 synthetic
 // groups of 10-15 requests; Sec. 7: real request groups of at most 13): many
@@ -40,7 +41,7 @@ namespace mpt {
 namespace {
 
 constexpr int kBatchThreads = 256;
-constexpr int kBatchOffsets = 17;  // pi_i in slots 0..12, u in slot kBatchUniv
+constexpr int kBatchOffsets = 17;  // pi_i in slots 0..m-1 (m <= 15), u in slot kBatchUniv
 constexpr int kBatchUniv = 16;
 
 // Step 2's scatter: chunk u of the instance goes to pi_i (N_x = {i}), to u
@@ -355,8 +356,9 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   // outputs: tables and OPT
   const int64_t tb = tab_off[inst];
   if (use_off) {
-    __shared__ long long hi_off[32];
-    if (t < 32) hi_off[t] = batch_pi((uint32_t)t * kBatchThreads, off) + (long long)off[kBatchUniv];
+    __shared__ long long hi_off[(1 << 15) / kBatchThreads];
+    for (int i = t; i < (N + kBatchThreads - 1) / kBatchThreads; i += kBatchThreads)
+      hi_off[i] = batch_pi((uint32_t)i * kBatchThreads, off) + (long long)off[kBatchUniv];
     __syncthreads();
     const int64_t lo = batch_pi((uint32_t)t & (kBatchThreads - 1), off);
     for (int S = t; S < N; S += kBatchThreads) {

@@ -57,7 +57,9 @@ struct mpt_batch {
 
 namespace {
 
-constexpr int kBatchMaxM = 13;
+constexpr int kBatchMaxM = 15;
+constexpr int kBatchRowsMaxM = 13;           // the row-blocked kernel; m = 14, 15 run the per-subset kernel
+constexpr size_t kBatchMaxSmem = 227 * 1024;  // shared memory of one block
 constexpr int kBatchSideStreams = 4;
 
 // Destroys the side streams and events on the device they were made on,
@@ -211,6 +213,15 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
         }
         j = k;
       }
+      // the per-subset kernel keeps the 2^m tables and the occurrence
+      // arrays in shared memory: at m = 15 that leaves room for 1024
+      // occurrences (the rows kernel needs less)
+      int cap = 1;
+      while (cap < occ) cap <<= 1;
+      if (mpt::batch_smem_bytes(m, cap) > kBatchMaxSmem) {
+        delete c;
+        return MPT_ERR_TOO_LARGE;
+      }
       c->tab_off[(size_t)b] = tab;
       tab += (int64_t)1 << m;
       c->max_m = std::max(c->max_m, m);
@@ -230,7 +241,7 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
     for (int pass = 0; pass < 2; ++pass) {
       for (int32_t b = 0; b < batch; ++b) {
         const int m = (int)(inst_requests[b + 1] - inst_requests[b]);
-        const bool rows = m >= 6 && (c->flags[(size_t)b] & mpt::kFlagPacked);
+        const bool rows = m >= 6 && m <= kBatchRowsMaxM && (c->flags[(size_t)b] & mpt::kFlagPacked);
         if (rows != (pass == 0)) continue;
         c->inst_list[(size_t)fill[(size_t)m]++] = b;
         int& cap = c->group_occ_cap[(size_t)m];

@@ -128,7 +128,8 @@ def _batch_status(mpt, weights, instances):
 def test_batch_create_validation(mpt):
     w = np.ones(50, dtype=np.int64)
     assert _batch_status(mpt, w, [[[1, 2], [3]], [[4]]]) == 0
-    assert _batch_status(mpt, w, [[[i] for i in range(14)]]) == 2           # m > 13
+    assert _batch_status(mpt, w, [[[i] for i in range(14)]]) == 0           # m = 14
+    assert _batch_status(mpt, w, [[[i] for i in range(16)]]) == 2           # m > 15
     assert _batch_status(mpt, w, [[[1, 1]]]) == 1                           # repeated chunk in a request
     assert _batch_status(mpt, w, [[[50]]]) == 1                             # chunk id >= n
     assert _batch_status(mpt, w, [[]]) == 1                                 # an instance with no request
@@ -139,6 +140,12 @@ def test_batch_create_validation(mpt):
     assert _batch_status(mpt, huge, [[[0, 1], [0, 1]]]) == 3                # sum of w(R_i) >= 2^62
     big = [[list(range(0, 2049))]]
     assert _batch_status(mpt, np.ones(3000, dtype=np.int64), big) == 2      # > 2048 occurrences
+    m14 = [[list(range(146 * i, 146 * i + 146)) for i in range(14)]]
+    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m14) == 0      # m = 14, 2044 occurrences
+    m15 = [[list(range(70 * i, 70 * i + 70)) for i in range(15)]]
+    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m15) == 2      # m = 15, > 1024 occurrences
+    m15 = [[list(range(68 * i, 68 * i + 68)) for i in range(15)]]
+    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m15) == 0      # m = 15, 1020 occurrences
 
 
 def test_schedule_and_cache_validation(mpt):

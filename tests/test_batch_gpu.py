@@ -2,7 +2,7 @@
 
 Every instance of a batch must match the oracle bit for bit: OPT, every F(S)
 and split(S) of its own 2^m table, every request's chunk order and the DFS
-order.  The batch mixes sizes m = 1..13, empty and repeated requests, and
+order.  The batches mix sizes m = 1..15, empty and repeated requests, and
 RAG-like groups drawn from topical pools (the shape of the paper's request
 groups, Sec. 7).
 """
@@ -91,6 +91,32 @@ def test_batch_edge_cases(mpt):
 def test_batch_large_requests(mpt):
     """Requests of up to 150 chunks (near the 2048-occurrence limit at m = 13)."""
     weights, batch = rag_batch(40, 20000, seed=2, m_range=(10, 13), k_range=(100, 150), pool_size=400)
+    check_batch(mpt, weights, batch)
+
+
+def test_batch_fourteen_and_fifteen_requests(mpt):
+    """Groups of 14 and 15 requests (the per-subset kernel, tables in shared
+    memory): RAG-shaped groups on the packed keys, heavy groups on the 64-bit
+    keys, groups with private suffixes and a common prefix, and a 15-request
+    group at the 1024-occurrence limit, mixed with smaller sizes."""
+    weights, batch = rag_batch(24, 3000, seed=14, m_range=(14, 15), k_range=(0, 10))
+    rng = np.random.default_rng(15)
+    n = int(weights.shape[0])
+    heavy_ids = n
+    weights = np.concatenate([weights, rng.integers(1 << 18, 1 << 20, size=40, dtype=np.int64)])
+    for _ in range(4):
+        m = int(rng.integers(14, 16))
+        batch.append([sorted(set(int(x) for x in heavy_ids + rng.choice(40, size=int(rng.integers(1, 8)),
+                                                                        replace=False))) for _ in range(m)])
+    prefix = len(weights)
+    weights = np.concatenate([weights, [1 << 35], rng.integers(1 << 30, 1 << 40, size=15, dtype=np.int64)])
+    grp = [sorted(set(int(x) for x in rng.choice(300, size=6, replace=False))) + [prefix, prefix + 1 + i]
+           for i in range(15)]
+    batch.append(grp)
+    batch.append([list(range(68 * i, 68 * i + 68)) for i in range(15)])
+    batch += rag_batch(20, 3000, seed=16, m_range=(1, 13))[1]
+    shared = [_shared_weight(weights, reqs) for reqs in batch if len(reqs) >= 14]
+    assert any(s >= 1 << 17 for s in shared) and any(s < 1 << 17 for s in shared)
     check_batch(mpt, weights, batch)
 
 
