@@ -1,6 +1,6 @@
 // Batched exact solve of many small instances (m <= 15 requests each), one
-// block per instance with every table in shared memory: the row-blocked
-// kernel for packed keys up to m = 13, the per-subset kernel otherwise.
+// block per instance with its tables in shared memory: the row-blocked
+// kernel for packed keys (m >= 6), the per-subset kernel otherwise.
 //
 // This is the paper's own use of the exact recurrence (Sec. 6.2: 72 synthetic
 // groups of 10-15 requests; Sec. 7: real request groups of at most 13): many
@@ -406,7 +406,9 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 // ---------------------------------------------------------------------------
 constexpr int kBRow = 32;
 constexpr int kBRowStride = 36;
-constexpr int kBMaxLevelRows = 70;  // C(8, 4): the most rows of one level (m = 13)
+constexpr int kBMaxLevelRows = 252;  // C(10, 5): the most rows of one level (m = 15)
+constexpr int kBMaxRowsM = 15;
+constexpr int kBGlobalSplitM = 14;   // from here the split table goes straight to global memory
 constexpr int kBkStride = kBRow + 1; // phase A minima: 33 words a row, so rows read by one warp use different banks
 
 // rows of the largest level C(nb, nb / 2), rounded up to even so that the
@@ -416,28 +418,37 @@ __host__ __device__ constexpr int batch_level_rows(int nb) {
   for (int i = 0; i < nb / 2; ++i) c = c * (nb - i) / (i + 1);
   return (c + 1) & ~1;
 }
-static_assert(batch_level_rows(8) == kBMaxLevelRows, "the most rows of one level (m = 13)");
+static_assert(batch_level_rows(kBMaxRowsM - 5) == kBMaxLevelRows, "the most rows of one level (m = 15)");
 
 // threads per block of the row-blocked kernel for m requests: enough lanes for
 // the busiest level (rows x lanes per row) -- 30 up to m = 11, 84 at m = 12,
-// 224 at m = 13
+// 224 at m = 13; from m = 14 the 256 threads take a level's lanes in passes
 constexpr int batch_rows_threads(int m) { return m <= 11 ? 64 : (m == 12 ? 128 : 256); }
 
-// lanes the busiest level needs: rows C(nb, p1) times 2^(p1 - 3) lanes per row
-// in phase A, C(nb, p1) threads in phase B
+// lanes per row in phase A at row level p1: enough that each lane runs at
+// most 8 row pairs, but no more than a warp (the lanes of a row reduce with
+// shuffles)
+__host__ __device__ constexpr int batch_rows_g(int p1) { return p1 <= 3 ? 0 : (p1 - 3 < 5 ? p1 - 3 : 5); }
+
+// lanes the busiest level needs: rows C(nb, p1) times 2^g lanes per row in
+// phase A, C(nb, p1) threads in phase B
 constexpr int batch_rows_lanes(int nb) {
   int most = 0;
   for (int p1 = 1; p1 <= nb; ++p1) {
     int c = 1;
     for (int i = 0; i < p1; ++i) c = c * (nb - i) / (i + 1);
-    const int lanes = c * (p1 > 3 ? 1 << (p1 - 3) : 1);
+    const int lanes = c * (1 << batch_rows_g(p1));
     most = lanes > most ? lanes : most;
   }
   return most;
 }
+// Up to m = 13 every level's lanes fit the block in one pass; beyond, phase
+// A runs in passes, and phase B still has one thread per row.
 constexpr bool batch_rows_fit() {
-  for (int m = 6; m <= 13; ++m)
-    if (batch_rows_lanes(m - 5) > batch_rows_threads(m) || batch_level_rows(m - 5) > batch_rows_threads(m)) return false;
+  for (int m = 6; m <= kBMaxRowsM; ++m) {
+    if (batch_level_rows(m - 5) > batch_rows_threads(m)) return false;
+    if (m <= 13 && batch_rows_lanes(m - 5) > batch_rows_threads(m)) return false;
+  }
   return true;
 }
 static_assert(batch_rows_fit(), "every level of the row-blocked kernel fits its block");
@@ -504,7 +515,17 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   int32_t* cx = reinterpret_cast<int32_t*>(keys + occ_cap);                        // [occ_cap]
   uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                        // [occ_cap]
   uint32_t* tmask = cN + occ_cap;                                                  // [2 * occ_cap] hash-table masks
-  uint16_t* split = reinterpret_cast<uint16_t*>(tmask + 2 * occ_cap);              // [2^m] for the walk
+  uint16_t* split = reinterpret_cast<uint16_t*>(tmask + 2 * occ_cap);              // [2^m] for the walk (m < 14)
+  // from m = 14 the split table is written to its output slots directly and
+  // the walk reads it there
+  const bool gsplit = mm >= kBGlobalSplitM;
+  uint32_t* gsp = split_out + tab_off[inst];
+  auto put_split = [&](uint32_t U, uint32_t A) {
+    if (gsplit)
+      gsp[U] = A;
+    else
+      split[U] = (uint16_t)A;
+  };
   __shared__ int ndistinct;
   const int t = threadIdx.x;
 
@@ -570,7 +591,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       }
       zp[s2] = (f << m) + (uint32_t)s2;
       zc[s2] = f << m;
-      split[s2] = (uint16_t)A;
+      put_split((uint32_t)s2, A);
     }
 #pragma unroll
     for (int s2 = 0; s2 < kBRow; ++s2) Gp[s2] = zp[s2];
@@ -580,48 +601,51 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   for (int p1 = 1; p1 <= nb; ++p1) {
     const int rows = (int)c_binom.v[nb][p1];
     if (p1 >= 2) {
-      // phase A: row pairs (a1, s1 ^ a1), a1 not in {0, s1}; G lanes per row
-      const int g = p1 > 3 ? p1 - 3 : 0;
+      // phase A: row pairs (a1, s1 ^ a1), a1 not in {0, s1}; G lanes per row,
+      // the level's rows x G lanes in passes of TPI (one pass up to m = 13)
+      const int g = batch_rows_g(p1);
       const int G = 1 << g;
-      const int ri = t >> g;
-      const uint32_t r = (uint32_t)t & (uint32_t)(G - 1);
-      uint32_t acc[kBRow];
+      for (int pass = 0; pass < (rows << g); pass += TPI) {
+        const int ri = (pass + t) >> g;
+        const uint32_t r = (uint32_t)t & (uint32_t)(G - 1);
+        uint32_t acc[kBRow];
 #pragma unroll
-      for (int i = 0; i < kBRow; ++i) acc[i] = 0xFFFFFFFFu;
-      if (ri < rows) {
-        const uint32_t s1 = colex_unrank((unsigned long long)ri, p1, nb);
-        const uint32_t lowb = s1 & (~s1 + 1u);
-        uint32_t hi = 0, rr = s1;
-        for (int q = 0; q < g; ++q) {
-          const uint32_t top = 1u << (31 - __clz(rr));
-          hi |= top;
-          rr ^= top;
-        }
-        const uint32_t freem = s1 ^ hi;
-        const uint32_t fixed = deposit_bits(r, hi);
-        uint32_t sub = 0;
-        do {
-          const uint32_t a1 = fixed | sub;
-          if (a1 != 0 && a1 != s1) {
-            uint32_t x[kBRow], y[kBRow];
-            bload_row(x, Gp + brow_pos(a1) * kBRowStride);
-            bload_row(y, Gp + brow_pos(s1 ^ a1) * kBRowStride);
-            const uint32_t yb = (s1 ^ a1) << 5;
-#pragma unroll
-            for (int i = 0; i < kBRow; ++i) y[i] -= yb | (uint32_t)i;  // Gc = Gp - X
-            bconv_restricted(acc, x, y);
-            if (a1 & lowb) acc[0] = min(acc[0], x[0] + y[0]);
+        for (int i = 0; i < kBRow; ++i) acc[i] = 0xFFFFFFFFu;
+        if (ri < rows) {
+          const uint32_t s1 = colex_unrank((unsigned long long)ri, p1, nb);
+          const uint32_t lowb = s1 & (~s1 + 1u);
+          uint32_t hi = 0, rr = s1;
+          for (int q = 0; q < g; ++q) {
+            const uint32_t top = 1u << (31 - __clz(rr));
+            hi |= top;
+            rr ^= top;
           }
-          sub = (sub - freem) & freem;
-        } while (sub != 0);
-      }
-      for (int off = G >> 1; off > 0; off >>= 1) {
+          const uint32_t freem = s1 ^ hi;
+          const uint32_t fixed = deposit_bits(r, hi);
+          uint32_t sub = 0;
+          do {
+            const uint32_t a1 = fixed | sub;
+            if (a1 != 0 && a1 != s1) {
+              uint32_t x[kBRow], y[kBRow];
+              bload_row(x, Gp + brow_pos(a1) * kBRowStride);
+              bload_row(y, Gp + brow_pos(s1 ^ a1) * kBRowStride);
+              const uint32_t yb = (s1 ^ a1) << 5;
 #pragma unroll
-        for (int i = 0; i < kBRow; ++i) acc[i] = min(acc[i], __shfl_xor_sync(0xFFFFFFFFu, acc[i], off));
-      }
-      if (ri < rows && r == 0) {
+              for (int i = 0; i < kBRow; ++i) y[i] -= yb | (uint32_t)i;  // Gc = Gp - X
+              bconv_restricted(acc, x, y);
+              if (a1 & lowb) acc[0] = min(acc[0], x[0] + y[0]);
+            }
+            sub = (sub - freem) & freem;
+          } while (sub != 0);
+        }
+        for (int off = G >> 1; off > 0; off >>= 1) {
 #pragma unroll
-        for (int i = 0; i < kBRow; ++i) bk[ri * kBkStride + i] = acc[i];
+          for (int i = 0; i < kBRow; ++i) acc[i] = min(acc[i], __shfl_xor_sync(0xFFFFFFFFu, acc[i], off));
+        }
+        if (ri < rows && r == 0) {
+#pragma unroll
+          for (int i = 0; i < kBRow; ++i) bk[ri * kBkStride + i] = acc[i];
+        }
       }
       __syncthreads();
     }
@@ -667,7 +691,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
             A = key & mask;
           }
           cc[s2] = f << m;
-          split[S1 | (uint32_t)s2] = (uint16_t)A;
+          put_split(S1 | (uint32_t)s2, A);
         }
       }
       uint32_t gp[kBRow];
@@ -680,24 +704,30 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 
   // outputs: tables and OPT
   if (use_off) {
-    __shared__ long long hi_off[32];
-    if (t < 32) hi_off[t] = batch_pi((uint32_t)t * TPI, off) + (long long)off[kBatchUniv];
+    // N / TPI entries: m <= 12 on the 64- and 128-thread variants, m <= 15 on 256
+    __shared__ long long hi_off[TPI == 256 ? (1 << kBMaxRowsM) / 256 : 32];
+    for (int i = t; i < (N + TPI - 1) / TPI; i += TPI)
+      hi_off[i] = batch_pi((uint32_t)i * TPI, off) + (long long)off[kBatchUniv];
     __syncthreads();
     const int64_t lo = batch_pi((uint32_t)t & (TPI - 1), off);
     for (int U = t; U < N; U += TPI) {
       F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m) + batch_offset<TPI>((uint32_t)U, lo, hi_off);
-      split_out[tb + U] = split[U];
+      if (!gsplit) split_out[tb + U] = split[U];
     }
     if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m) + batch_pi(mask, off) + (int64_t)off[kBatchUniv];
   } else {
     for (int U = t; U < N; U += TPI) {
       F_out[tb + U] = (int64_t)(Gp[bidx((uint32_t)U)] >> m);
-      split_out[tb + U] = split[U];
+      if (!gsplit) split_out[tb + U] = split[U];
     }
     if (t == 0) opt_out[inst] = (int64_t)(Gp[bidx(mask)] >> m);
   }
   __syncthreads();
-  batch_walk<TPI>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  if (gsplit)
+    batch_walk<TPI>(inst, m, r0, o0, roff, static_cast<const uint32_t*>(gsp), keys, cx, cN, nd, perm_out, dfs_out,
+                    status);
+  else
+    batch_walk<TPI>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
 }
 
 }  // namespace
@@ -724,7 +754,7 @@ cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, 
 size_t batch_rows_smem_bytes(int m, int occ_cap) {
   const size_t R = (size_t)1 << (m - 5);
   return R * kBRowStride * 4 + (size_t)batch_level_rows(m - 5) * kBkStride * 4 + (size_t)occ_cap * 16 +
-         (size_t)occ_cap * 8 + ((size_t)2 << m) + 64;
+         (size_t)occ_cap * 8 + (m >= kBGlobalSplitM ? 0 : ((size_t)2 << m)) + 64;
 }
 
 // One grid of the row-blocked kernel over `count` instances of size m >= 6
@@ -733,7 +763,7 @@ cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weig
                               const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
                               const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
                               uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream) {
-  if (m < 6 || m > 13) return cudaErrorInvalidValue;
+  if (m < 6 || m > kBMaxRowsM) return cudaErrorInvalidValue;
   const size_t smem = batch_rows_smem_bytes(m, occ_cap);
   const int tpi = batch_rows_threads(m);
   cudaError_t e = cudaSuccess;

@@ -58,7 +58,7 @@ struct mpt_batch {
 namespace {
 
 constexpr int kBatchMaxM = 15;
-constexpr int kBatchRowsMaxM = 13;           // the row-blocked kernel; m = 14, 15 run the per-subset kernel
+constexpr int kBatchRowsMaxM = 15;           // the row-blocked kernel (packed keys, m >= 6)
 constexpr size_t kBatchMaxSmem = 227 * 1024;  // shared memory of one block
 constexpr int kBatchSideStreams = 4;
 
@@ -215,7 +215,7 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
       }
       // the per-subset kernel keeps the 2^m tables and the occurrence
       // arrays in shared memory: at m = 15 that leaves room for 1024
-      // occurrences (the rows kernel needs less)
+      // occurrences (the row-blocked kernel needs less at every m)
       int cap = 1;
       while (cap < occ) cap <<= 1;
       if (mpt::batch_smem_bytes(m, cap) > kBatchMaxSmem) {

@@ -95,10 +95,11 @@ def test_batch_large_requests(mpt):
 
 
 def test_batch_fourteen_and_fifteen_requests(mpt):
-    """Groups of 14 and 15 requests (the per-subset kernel, tables in shared
-    memory): RAG-shaped groups on the packed keys, heavy groups on the 64-bit
-    keys, groups with private suffixes and a common prefix, and a 15-request
-    group at the 1024-occurrence limit, mixed with smaller sizes."""
+    """Groups of 14 and 15 requests: RAG-shaped groups on the packed keys
+    (row-blocked kernel, split table in global memory, phase A in passes),
+    heavy groups on the 64-bit keys (per-subset kernel), groups with private
+    suffixes and a common prefix, and a 15-request group at the
+    1024-occurrence limit, mixed with smaller sizes."""
     weights, batch = rag_batch(24, 3000, seed=14, m_range=(14, 15), k_range=(0, 10))
     rng = np.random.default_rng(15)
     n = int(weights.shape[0])
