@@ -453,6 +453,15 @@ constexpr bool batch_rows_fit() {
 }
 static_assert(batch_rows_fit(), "every level of the row-blocked kernel fits its block");
 
+// entries of the per-block offset table (one per TPI subsets) of each variant
+__host__ __device__ constexpr int batch_rows_hi_entries(int tpi) { return tpi == 256 ? (1 << kBMaxRowsM) / 256 : 32; }
+constexpr bool batch_rows_hi_fit() {
+  for (int m = 6; m <= kBMaxRowsM; ++m)
+    if ((1 << m) / batch_rows_threads(m) > batch_rows_hi_entries(batch_rows_threads(m))) return false;
+  return true;
+}
+static_assert(batch_rows_hi_fit(), "the offset table covers every size of each block width");
+
 __device__ __forceinline__ int brow_pos(uint32_t r) { return (int)(r ^ (((r >> 3) ^ (r >> 6)) & 7u)); }
 __device__ __forceinline__ int bidx(uint32_t U) { return brow_pos(U >> 5) * kBRowStride + (int)(U & 31u); }
 
@@ -704,8 +713,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 
   // outputs: tables and OPT
   if (use_off) {
-    // N / TPI entries: m <= 12 on the 64- and 128-thread variants, m <= 15 on 256
-    __shared__ long long hi_off[TPI == 256 ? (1 << kBMaxRowsM) / 256 : 32];
+    __shared__ long long hi_off[batch_rows_hi_entries(TPI)];
     for (int i = t; i < (N + TPI - 1) / TPI; i += TPI)
       hi_off[i] = batch_pi((uint32_t)i * TPI, off) + (long long)off[kBatchUniv];
     __syncthreads();
