@@ -219,7 +219,7 @@ mpt_status mpt_get_profile(const mpt_ctx* ctx, mpt_profile* out);
 /* ---------------------------------------------------------------------------
  * Batched exact solves of many small instances (the paper's own use of the
  * recurrence: synthetic groups of 10-15 requests, Sec. 6.2, and real request
- * groups of at most 13, Sec. 7); instances of up to 15 requests.
+ * groups of at most 13, Sec. 7); instances of up to 16 requests.
  * Every instance shares one chunk universe and weight array; instance b owns
  * requests inst_requests[b] .. inst_requests[b+1]-1, request r the chunk ids
  * chunk_ids[req_offsets[r] .. req_offsets[r+1]).  One CUDA block solves one
@@ -234,8 +234,9 @@ typedef struct mpt_batch mpt_batch;
  *   0; req_offsets: int64[inst_requests[batch]+1], starting at 0;
  *   chunk_ids: int64[req_offsets[last]] in [0, n_chunks), no repeat inside a
  *   request.
- * Limits per instance: 1 <= m <= 15 and at most 2048 chunk occurrences
- * (1024 at m = 15; MPT_ERR_TOO_LARGE beyond); sum_i w(R_i) < 2^62 and a shared weight
+ * Limits per instance: 1 <= m <= 16 and at most 2048 chunk occurrences
+ * (1024 at m = 15 unless the keys pack, see below; at m = 16 the keys must
+ * pack: shared weight below 2^16; MPT_ERR_TOO_LARGE beyond); sum_i w(R_i) < 2^62 and a shared weight
  * (sum_i w(R_i) less the chunks that one request alone or all m >= 2
  * requests hold, see MPT_DP_AUTO) below 2^31 (MPT_ERR_OVERFLOW).
  * Errors: INVALID_ARG, TOO_LARGE, OVERFLOW, OUT_OF_MEMORY.  No CUDA call. */

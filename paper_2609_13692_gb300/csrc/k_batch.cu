@@ -233,7 +233,7 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   uint32_t* cN = reinterpret_cast<uint32_t*>(cx + occ_cap);                    // [occ_cap] their request sets
   uint32_t* tmask = cN + occ_cap;                                                // [2 * occ_cap] hash-table masks
   __shared__ int ndistinct;
-  __shared__ int roff[16];  // request offsets relative to o0
+  __shared__ int roff[17];  // request offsets relative to o0 (m + 1 <= 17)
   __shared__ unsigned long long off[kBatchOffsets];
   const int t = threadIdx.x;
   const int nd = batch_gather<kBatchThreads>(m, r0, o0, occ, occ_cap, req_off, chunks,
@@ -406,8 +406,9 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
 // ---------------------------------------------------------------------------
 constexpr int kBRow = 32;
 constexpr int kBRowStride = 36;
-constexpr int kBMaxLevelRows = 252;  // C(10, 5): the most rows of one level (m = 15)
-constexpr int kBMaxRowsM = 15;
+constexpr int kBMaxLevelRows = 462;  // C(11, 5): the most rows of one level (m = 16)
+constexpr int kBMaxRowsM = 16;
+constexpr int kBGlobalRowsM = 16;    // from here the rows live in a global scratch slot per block
 constexpr int kBGlobalSplitM = 14;   // from here the split table goes straight to global memory
 constexpr int kBkStride = kBRow + 1; // phase A minima: 33 words a row, so rows read by one warp use different banks
 
@@ -418,7 +419,7 @@ __host__ __device__ constexpr int batch_level_rows(int nb) {
   for (int i = 0; i < nb / 2; ++i) c = c * (nb - i) / (i + 1);
   return (c + 1) & ~1;
 }
-static_assert(batch_level_rows(kBMaxRowsM - 5) == kBMaxLevelRows, "the most rows of one level (m = 15)");
+static_assert(batch_level_rows(kBMaxRowsM - 5) == kBMaxLevelRows, "the most rows of one level (m = 16)");
 
 // threads per block of the row-blocked kernel for m requests: enough lanes for
 // the busiest level (rows x lanes per row) -- 30 up to m = 11, 84 at m = 12,
@@ -442,22 +443,26 @@ constexpr int batch_rows_lanes(int nb) {
   }
   return most;
 }
-// Up to m = 13 every level's lanes fit the block in one pass; beyond, phase
-// A runs in passes, and phase B still has one thread per row.
+// Up to m = 13 every level's lanes and rows fit the block in one pass;
+// beyond, phase A and phase B run in passes.
 constexpr bool batch_rows_fit() {
-  for (int m = 6; m <= kBMaxRowsM; ++m) {
-    if (batch_level_rows(m - 5) > batch_rows_threads(m)) return false;
-    if (m <= 13 && batch_rows_lanes(m - 5) > batch_rows_threads(m)) return false;
-  }
+  for (int m = 6; m <= 13; ++m)
+    if (batch_level_rows(m - 5) > batch_rows_threads(m) || batch_rows_lanes(m - 5) > batch_rows_threads(m))
+      return false;
   return true;
 }
 static_assert(batch_rows_fit(), "every level of the row-blocked kernel fits its block");
 
-// entries of the per-block offset table (one per TPI subsets) of each variant
-__host__ __device__ constexpr int batch_rows_hi_entries(int tpi) { return tpi == 256 ? (1 << kBMaxRowsM) / 256 : 32; }
+// entries of the per-block offset table (one per TPI subsets) of each
+// variant: m <= 12 on 64 and 128 threads, m <= 15 on 256, m = 16 with the
+// rows in global memory
+__host__ __device__ constexpr int batch_rows_hi_entries(int tpi, bool grows) {
+  return grows ? (1 << kBGlobalRowsM) / 256 : (tpi == 256 ? (1 << (kBGlobalRowsM - 1)) / 256 : 32);
+}
 constexpr bool batch_rows_hi_fit() {
   for (int m = 6; m <= kBMaxRowsM; ++m)
-    if ((1 << m) / batch_rows_threads(m) > batch_rows_hi_entries(batch_rows_threads(m))) return false;
+    if ((1 << m) / batch_rows_threads(m) > batch_rows_hi_entries(batch_rows_threads(m), m >= kBGlobalRowsM))
+      return false;
   return true;
 }
 static_assert(batch_rows_hi_fit(), "the offset table covers every size of each block width");
@@ -495,14 +500,14 @@ __device__ __forceinline__ void bconv_restricted(uint32_t (&acc)[kBRow], const u
   }
 }
 
-template <int TPI>
+template <int TPI, bool kGRows = false>
 __global__ void __launch_bounds__(TPI, TPI >= 256 ? 3 : (TPI == 128 ? 6 : 12))  // 12 warps or more per SM
 k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ inst_req,
              const int64_t* __restrict__ req_off, const int64_t* __restrict__ chunks,
              const int64_t* __restrict__ tab_off, const int32_t* __restrict__ inst_list,
              const uint8_t* __restrict__ flags, int occ_cap, int mm, int64_t* __restrict__ opt_out,
              int64_t* __restrict__ F_out, uint32_t* __restrict__ split_out, int64_t* __restrict__ perm_out,
-             int32_t* __restrict__ dfs_out, int32_t* __restrict__ status) {
+             int32_t* __restrict__ dfs_out, int32_t* __restrict__ status, uint32_t* __restrict__ rows_scratch) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int inst = inst_list[blockIdx.x];
   const int64_t r0 = inst_req[inst], r1 = inst_req[inst + 1];
@@ -517,8 +522,12 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 
   // Gp(X) = (F(X) << m) + X only: the complement form Gc(X) = Gp(X) - X is
   // formed from it when a row is loaded
-  uint32_t* Gp = reinterpret_cast<uint32_t*>(smem_raw);                          // [R * 36]
-  uint32_t* bk = Gp + (1 << (mm - 5)) * kBRowStride;                               // [level rows * 33] phase A minima
+  // (kGRows: the rows, 295 KB at m = 16, live in this block's slot of a
+  // global scratch array instead, L1/L2-resident while the block runs)
+  const size_t row_words = (size_t)(1 << (mm - 5)) * kBRowStride;
+  uint32_t* Gp = kGRows ? rows_scratch + (size_t)blockIdx.x * row_words
+                        : reinterpret_cast<uint32_t*>(smem_raw);                 // [R * 36]
+  uint32_t* bk = kGRows ? reinterpret_cast<uint32_t*>(smem_raw) : Gp + row_words;  // [level rows * 33] phase A minima
   unsigned long long* keys =
       reinterpret_cast<unsigned long long*>(bk + batch_level_rows(mm - 5) * kBkStride);  // [occ_cap]
   int32_t* cx = reinterpret_cast<int32_t*>(keys + occ_cap);                        // [occ_cap]
@@ -538,7 +547,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   __shared__ int ndistinct;
   const int t = threadIdx.x;
 
-  __shared__ int roff[16];  // request offsets relative to o0
+  __shared__ int roff[17];  // request offsets relative to o0 (m + 1 <= 17)
   __shared__ unsigned long long off[kBatchOffsets];
   const int nd = batch_gather<TPI>(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask,
                                    cx, cN, roff, &ndistinct);
@@ -658,62 +667,66 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       }
       __syncthreads();
     }
-    // phase B: one thread finishes each row of the level
-    if (t < rows) {
-      const uint32_t s1 = colex_unrank((unsigned long long)t, p1, nb);
-      const uint32_t S1 = s1 << 5;
-      uint32_t* prow = Gp + brow_pos(s1) * kBRowStride;
-      uint32_t zp[kBRow], zcs[kBRow], cc[kBRow];
-      bload_row(zp, Gp);   // row 0 is at position 0
-      bload_row(zcs, Gp);
+    // phase B: one thread finishes each row of the level (in passes of TPI
+    // rows from m = 14)
+    for (int rb = 0; rb < rows; rb += TPI) {
+    const int tr = rb + t;
+      if (tr < rows) {
+        const uint32_t s1 = colex_unrank((unsigned long long)tr, p1, nb);
+        const uint32_t S1 = s1 << 5;
+        uint32_t* prow = Gp + brow_pos(s1) * kBRowStride;
+        uint32_t zp[kBRow], zcs[kBRow], cc[kBRow];
+        bload_row(zp, Gp);   // row 0 is at position 0
+        bload_row(zcs, Gp);
 #pragma unroll
-      for (int i = 0; i < kBRow; ++i) zcs[i] += S1 - (uint32_t)i;  // Gc(0, x) + (s1 << 5): the A-part of a1 = s1 splits
+        for (int i = 0; i < kBRow; ++i) zcs[i] += S1 - (uint32_t)i;  // Gc(0, x) + (s1 << 5): the A-part of a1 = s1 splits
 #pragma unroll
-      for (int blk = 0; blk < kBRow / 8; ++blk) {
-        uint32_t wv[8], bkv[8];
+        for (int blk = 0; blk < kBRow / 8; ++blk) {
+          uint32_t wv[8], bkv[8];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          wv[q] = prow[blk * 8 + q];
-          bkv[q] = p1 >= 2 ? bk[t * kBkStride + blk * 8 + q] : 0xFFFFFFFFu;
-        }
+          for (int q = 0; q < 8; ++q) {
+            wv[q] = prow[blk * 8 + q];
+            bkv[q] = p1 >= 2 ? bk[tr * kBkStride + blk * 8 + q] : 0xFFFFFFFFu;
+          }
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const int s2 = blk * 8 + q;
-          uint32_t f, A;
-          if (s2 == 0 && p1 == 1) {  // U = (s1, 0) is a single request
-            f = wv[q];
-            A = 0;
-          } else {
-            // two independent minima (a1 = 0 and a1 = s1) shorten the chains
-            uint32_t k0 = bkv[q], k1 = 0xFFFFFFFFu;
-            if (s2 != 0) {
+          for (int q = 0; q < 8; ++q) {
+            const int s2 = blk * 8 + q;
+            uint32_t f, A;
+            if (s2 == 0 && p1 == 1) {  // U = (s1, 0) is a single request
+              f = wv[q];
+              A = 0;
+            } else {
+              // two independent minima (a1 = 0 and a1 = s1) shorten the chains
+              uint32_t k0 = bkv[q], k1 = 0xFFFFFFFFu;
+              if (s2 != 0) {
 #pragma unroll
-              for (int a2 = 1; a2 < kBRow; ++a2) {
-                if ((a2 & s2) == a2 && (a2 & (s2 & -s2)) != 0) {
-                  k0 = min(k0, zp[a2] + cc[s2 ^ a2]);                             // a1 = 0
-                  if (a2 != s2) k1 = min(k1, cc[a2] + zcs[s2 ^ a2] + (uint32_t)a2);  // a1 = s1
+                for (int a2 = 1; a2 < kBRow; ++a2) {
+                  if ((a2 & s2) == a2 && (a2 & (s2 & -s2)) != 0) {
+                    k0 = min(k0, zp[a2] + cc[s2 ^ a2]);                             // a1 = 0
+                    if (a2 != s2) k1 = min(k1, cc[a2] + zcs[s2 ^ a2] + (uint32_t)a2);  // a1 = s1
+                  }
                 }
               }
+              const uint32_t key = min(k0, k1);
+              f = (key >> m) - wv[q];
+              A = key & mask;
             }
-            const uint32_t key = min(k0, k1);
-            f = (key >> m) - wv[q];
-            A = key & mask;
+            cc[s2] = f << m;
+            put_split(S1 | (uint32_t)s2, A);
           }
-          cc[s2] = f << m;
-          put_split(S1 | (uint32_t)s2, A);
         }
-      }
-      uint32_t gp[kBRow];
+        uint32_t gp[kBRow];
 #pragma unroll
-      for (int i = 0; i < kBRow; ++i) gp[i] = cc[i] + (S1 | (uint32_t)i);
-      bstore_row(prow, gp);
+        for (int i = 0; i < kBRow; ++i) gp[i] = cc[i] + (S1 | (uint32_t)i);
+        bstore_row(prow, gp);
+      }
     }
     __syncthreads();
   }
 
   // outputs: tables and OPT
   if (use_off) {
-    __shared__ long long hi_off[batch_rows_hi_entries(TPI)];
+    __shared__ long long hi_off[batch_rows_hi_entries(TPI, kGRows)];
     for (int i = t; i < (N + TPI - 1) / TPI; i += TPI)
       hi_off[i] = batch_pi((uint32_t)i * TPI, off) + (long long)off[kBatchUniv];
     __syncthreads();
@@ -761,8 +774,14 @@ cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, 
 
 size_t batch_rows_smem_bytes(int m, int occ_cap) {
   const size_t R = (size_t)1 << (m - 5);
-  return R * kBRowStride * 4 + (size_t)batch_level_rows(m - 5) * kBkStride * 4 + (size_t)occ_cap * 16 +
-         (size_t)occ_cap * 8 + (m >= kBGlobalSplitM ? 0 : ((size_t)2 << m)) + 64;
+  return (m >= kBGlobalRowsM ? 0 : R * kBRowStride * 4) + (size_t)batch_level_rows(m - 5) * kBkStride * 4 +
+         (size_t)occ_cap * 16 + (size_t)occ_cap * 8 + (m >= kBGlobalSplitM ? 0 : ((size_t)2 << m)) + 64;
+}
+
+// 4-byte words of global row scratch one instance of size m needs (0 while
+// its rows fit shared memory)
+size_t batch_rows_scratch_words(int m) {
+  return m >= kBGlobalRowsM ? ((size_t)1 << (m - 5)) * kBRowStride : 0;
 }
 
 // One grid of the row-blocked kernel over `count` instances of size m >= 6
@@ -770,8 +789,9 @@ size_t batch_rows_smem_bytes(int m, int occ_cap) {
 cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                               const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
                               const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
-                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream) {
-  if (m < 6 || m > kBMaxRowsM) return cudaErrorInvalidValue;
+                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, uint32_t* rows_scratch,
+                              cudaStream_t stream) {
+  if (m < 6 || m > kBMaxRowsM || (m >= kBGlobalRowsM && !rows_scratch)) return cudaErrorInvalidValue;
   const size_t smem = batch_rows_smem_bytes(m, occ_cap);
   const int tpi = batch_rows_threads(m);
   cudaError_t e = cudaSuccess;
@@ -779,9 +799,11 @@ cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weig
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e == cudaSuccess)
       kernel<<<(unsigned)count, tpi, smem, stream>>>(weights, inst_req, req_off, chunks, tab_off, inst_list, flags,
-                                                      occ_cap, m, opt, F, split, perm, dfs, status);
+                                                      occ_cap, m, opt, F, split, perm, dfs, status, rows_scratch);
   };
-  if (tpi == 64)
+  if (m >= kBGlobalRowsM)
+    go(k_batch_rows<256, true>);
+  else if (tpi == 64)
     go(k_batch_rows<64>);
   else if (tpi == 128)
     go(k_batch_rows<128>);

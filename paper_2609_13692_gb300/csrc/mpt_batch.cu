@@ -13,6 +13,8 @@
 
 namespace mpt {
 size_t batch_smem_bytes(int max_m, int occ_cap);
+size_t batch_rows_smem_bytes(int m, int occ_cap);
+size_t batch_rows_scratch_words(int m);
 cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                          const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
                          const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
@@ -20,7 +22,8 @@ cudaError_t launch_batch(int count, int m, int occ_cap, const int64_t* weights, 
 cudaError_t launch_batch_rows(int count, int m, int occ_cap, const int64_t* weights, const int64_t* inst_req,
                               const int64_t* req_off, const int64_t* chunks, const int64_t* tab_off,
                               const int32_t* inst_list, const uint8_t* flags, int64_t* opt, int64_t* F,
-                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, cudaStream_t stream);
+                              uint32_t* split, int64_t* perm, int32_t* dfs, int32_t* status, uint32_t* rows_scratch,
+                              cudaStream_t stream);
 }  // namespace mpt
 
 struct mpt_batch {
@@ -30,10 +33,10 @@ struct mpt_batch {
   std::vector<int64_t> w, inst_req, req_off, chunks, tab_off;
   // instances grouped by size m: inst_list[group_start[m] .. group_start[m+1]),
   // those for the row-blocked kernel (m >= 6, packed keys) first, up to
-  // group_rows_end[m]
+  // group_rows_end[m]; each part with its own occurrence cap
   std::vector<int32_t> inst_list;
   std::vector<int64_t> group_start, group_rows_end;
-  std::vector<int> group_occ_cap;
+  std::vector<int> group_occ_cap_rows, group_occ_cap;
   // per instance: kFlagPacked when the shared weight is below 2^(32 - m)
   // (32-bit keys), kFlagOffsets when sum_i w(R_i) is not (private and
   // universal chunks kept out of the kernels' values, k_batch.cu)
@@ -57,8 +60,7 @@ struct mpt_batch {
 
 namespace {
 
-constexpr int kBatchMaxM = 15;
-constexpr int kBatchRowsMaxM = 15;           // the row-blocked kernel (packed keys, m >= 6)
+constexpr int kBatchMaxM = 16;  // m = 16: packed keys only (the row-blocked kernel)
 constexpr size_t kBatchMaxSmem = 227 * 1024;  // shared memory of one block
 constexpr int kBatchSideStreams = 4;
 
@@ -113,7 +115,7 @@ constexpr int64_t kBatchSumLimit = (int64_t)1 << 62;
 
 struct BatchCarve {
   int64_t *weights, *inst_req, *req_off, *chunks, *tab_off, *opt, *F, *perm;
-  uint32_t* split;
+  uint32_t *split, *rows_scratch;
   int32_t *dfs, *status, *inst_list;
   uint8_t* flags;
 };
@@ -138,6 +140,14 @@ size_t carve(const mpt_batch* b, char* base, BatchCarve* c) {
   c->status = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
   c->inst_list = reinterpret_cast<int32_t*>(take((size_t)b->batch * 4));
   c->flags = reinterpret_cast<uint8_t*>(take((size_t)b->batch));
+  // rows of the row-blocked instances too large for shared memory, one slot
+  // per block of their size's launch
+  size_t scratch_words = 0;
+  if (!b->group_rows_end.empty())
+    for (int m = 1; m <= kBatchMaxM; ++m)
+      scratch_words = std::max(scratch_words, (size_t)(b->group_rows_end[(size_t)m] - b->group_start[(size_t)m]) *
+                                                  mpt::batch_rows_scratch_words(m));
+  c->rows_scratch = scratch_words ? reinterpret_cast<uint32_t*>(take(scratch_words * 4)) : nullptr;
   return off;
 }
 
@@ -213,12 +223,16 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
         }
         j = k;
       }
-      // the per-subset kernel keeps the 2^m tables and the occurrence
-      // arrays in shared memory: at m = 15 that leaves room for 1024
-      // occurrences (the row-blocked kernel needs less at every m)
+      c->flags[(size_t)b] = (uint8_t)((shared < ((int64_t)1 << (32 - m)) ? mpt::kFlagPacked : 0) |
+                                      (sum >= ((int64_t)1 << (32 - m)) ? mpt::kFlagOffsets : 0));
+      // the instance's kernel must hold its shared-memory arrays: the
+      // per-subset kernel keeps the 2^m tables there (m = 15: room for 1024
+      // occurrences; m = 16 does not fit, so 16 requests need packed keys),
+      // the row-blocked kernel its rows up to m = 15
       int cap = 1;
       while (cap < occ) cap <<= 1;
-      if (mpt::batch_smem_bytes(m, cap) > kBatchMaxSmem) {
+      const bool rows = m >= 6 && (c->flags[(size_t)b] & mpt::kFlagPacked);
+      if ((rows ? mpt::batch_rows_smem_bytes(m, cap) : mpt::batch_smem_bytes(m, cap)) > kBatchMaxSmem) {
         delete c;
         return MPT_ERR_TOO_LARGE;
       }
@@ -226,8 +240,6 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
       tab += (int64_t)1 << m;
       c->max_m = std::max(c->max_m, m);
       while (c->occ_cap < occ) c->occ_cap <<= 1;
-      c->flags[(size_t)b] = (uint8_t)((shared < ((int64_t)1 << (32 - m)) ? mpt::kFlagPacked : 0) |
-                                      (sum >= ((int64_t)1 << (32 - m)) ? mpt::kFlagOffsets : 0));
       inst_occ[(size_t)b] = (int)occ;
     }
     c->tab_off[(size_t)batch] = tab;
@@ -236,15 +248,16 @@ mpt_status mpt_batch_create(const int64_t* weights, int64_t n_chunks, int32_t ba
     for (int32_t b = 0; b < batch; ++b) ++c->group_start[(size_t)(inst_requests[b + 1] - inst_requests[b]) + 1];
     for (int m = 1; m <= kBatchMaxM + 1; ++m) c->group_start[(size_t)m] += c->group_start[(size_t)m - 1];
     c->inst_list.resize((size_t)batch);
+    c->group_occ_cap_rows.assign(kBatchMaxM + 1, 1);
     c->group_occ_cap.assign(kBatchMaxM + 1, 1);
     std::vector<int64_t> fill(c->group_start.begin(), c->group_start.end());
     for (int pass = 0; pass < 2; ++pass) {
       for (int32_t b = 0; b < batch; ++b) {
         const int m = (int)(inst_requests[b + 1] - inst_requests[b]);
-        const bool rows = m >= 6 && m <= kBatchRowsMaxM && (c->flags[(size_t)b] & mpt::kFlagPacked);
+        const bool rows = m >= 6 && (c->flags[(size_t)b] & mpt::kFlagPacked);
         if (rows != (pass == 0)) continue;
         c->inst_list[(size_t)fill[(size_t)m]++] = b;
-        int& cap = c->group_occ_cap[(size_t)m];
+        int& cap = rows ? c->group_occ_cap_rows[(size_t)m] : c->group_occ_cap[(size_t)m];
         while (cap < inst_occ[(size_t)b]) cap <<= 1;
       }
       if (pass == 0) c->group_rows_end.assign(fill.begin(), fill.end());
@@ -332,14 +345,15 @@ mpt_status mpt_batch_solve(mpt_batch* b, void* d_workspace, size_t workspace_byt
     const int64_t g0 = b->group_start[(size_t)m], gr = b->group_rows_end[(size_t)m],
                   g1 = b->group_start[(size_t)m + 1];
     if (g1 == g0) continue;
-    const int cap = b->group_occ_cap[(size_t)m];
     cudaStream_t st = forked ? b->side[(size_t)(next_side++ % kBatchSideStreams)] : stream;
     if (gr > g0)
-      e = mpt::launch_batch_rows((int)(gr - g0), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                                 c.inst_list + g0, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, st);
+      e = mpt::launch_batch_rows((int)(gr - g0), m, b->group_occ_cap_rows[(size_t)m], c.weights, c.inst_req, c.req_off,
+                                 c.chunks, c.tab_off, c.inst_list + g0, c.flags, c.opt, c.F, c.split, c.perm, c.dfs,
+                                 c.status, c.rows_scratch, st);
     if (e == cudaSuccess && g1 > gr)
-      e = mpt::launch_batch((int)(g1 - gr), m, cap, c.weights, c.inst_req, c.req_off, c.chunks, c.tab_off,
-                            c.inst_list + gr, c.flags, c.opt, c.F, c.split, c.perm, c.dfs, c.status, st);
+      e = mpt::launch_batch((int)(g1 - gr), m, b->group_occ_cap[(size_t)m], c.weights, c.inst_req, c.req_off,
+                            c.chunks, c.tab_off, c.inst_list + gr, c.flags, c.opt, c.F, c.split, c.perm, c.dfs,
+                            c.status, st);
   }
   if (forked) {
     // join every side stream, also after a failed launch, so that no work

@@ -426,7 +426,7 @@ def solve(weights, bits, mode: str = "auto", workspace=None, stream: Optional[in
 # ---------------------------------------------------------------------------
 
 class Batch:
-    """Owns one ``mpt_batch`` (many instances of at most 15 requests)."""
+    """Owns one ``mpt_batch`` (many instances of at most 16 requests)."""
 
     def __init__(self, handle: int, batch: int, inst_requests: np.ndarray, req_offsets: np.ndarray):
         self.handle = ctypes.c_void_p(handle)

@@ -129,7 +129,10 @@ def test_batch_create_validation(mpt):
     w = np.ones(50, dtype=np.int64)
     assert _batch_status(mpt, w, [[[1, 2], [3]], [[4]]]) == 0
     assert _batch_status(mpt, w, [[[i] for i in range(14)]]) == 0           # m = 14
-    assert _batch_status(mpt, w, [[[i] for i in range(16)]]) == 2           # m > 15
+    assert _batch_status(mpt, w, [[[i] for i in range(16)]]) == 0           # m = 16 (packed keys)
+    assert _batch_status(mpt, w, [[[i] for i in range(17)]]) == 2           # m > 16
+    heavy16 = np.full(50, 1 << 12, dtype=np.int64)
+    assert _batch_status(mpt, heavy16, [[[0, 1]] * 8 + [[2]] * 8]) == 2    # m = 16, shared weight >= 2^16
     assert _batch_status(mpt, w, [[[1, 1]]]) == 1                           # repeated chunk in a request
     assert _batch_status(mpt, w, [[[50]]]) == 1                             # chunk id >= n
     assert _batch_status(mpt, w, [[]]) == 1                                 # an instance with no request
@@ -142,10 +145,15 @@ def test_batch_create_validation(mpt):
     assert _batch_status(mpt, np.ones(3000, dtype=np.int64), big) == 2      # > 2048 occurrences
     m14 = [[list(range(146 * i, 146 * i + 146)) for i in range(14)]]
     assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m14) == 0      # m = 14, 2044 occurrences
-    m15 = [[list(range(70 * i, 70 * i + 70)) for i in range(15)]]
-    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m15) == 2      # m = 15, > 1024 occurrences
-    m15 = [[list(range(68 * i, 68 * i + 68)) for i in range(15)]]
-    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m15) == 0      # m = 15, 1020 occurrences
+    # m = 15 on 64-bit keys (the per-subset kernel): 1024 occurrences at most
+    w200 = np.full(3000, 200, dtype=np.int64)
+    m15 = [[list(range(35 * i, 35 * i + 70)) for i in range(15)]]
+    assert _batch_status(mpt, w200, m15) == 2                               # 1050 occurrences
+    m15 = [[list(range(34 * i, 34 * i + 68)) for i in range(15)]]
+    assert _batch_status(mpt, w200, m15) == 0                               # 1020 occurrences
+    # m = 15 on packed keys (the row-blocked kernel): up to 2048
+    m15 = [[list(range(136 * i, 136 * i + 136)) for i in range(15)]]
+    assert _batch_status(mpt, np.ones(3000, dtype=np.int64), m15) == 0      # 2040 occurrences
 
 
 def test_schedule_and_cache_validation(mpt):

@@ -2,7 +2,7 @@
 
 Every instance of a batch must match the oracle bit for bit: OPT, every F(S)
 and split(S) of its own 2^m table, every request's chunk order and the DFS
-order.  The batches mix sizes m = 1..15, empty and repeated requests, and
+order.  The batches mix sizes m = 1..16, empty and repeated requests, and
 RAG-like groups drawn from topical pools (the shape of the paper's request
 groups, Sec. 7).
 """
@@ -118,6 +118,25 @@ def test_batch_fourteen_and_fifteen_requests(mpt):
     batch += rag_batch(20, 3000, seed=16, m_range=(1, 13))[1]
     shared = [_shared_weight(weights, reqs) for reqs in batch if len(reqs) >= 14]
     assert any(s >= 1 << 17 for s in shared) and any(s < 1 << 17 for s in shared)
+    check_batch(mpt, weights, batch)
+
+
+def test_batch_sixteen_requests(mpt):
+    """Groups of 16 requests (packed keys only; the row-blocked kernel with
+    its rows in a global scratch slot per block), RAG-shaped with light
+    passages, one with private suffixes and a common prefix, and the
+    leave-one-out family L_16 (its optimum has a closed form), mixed with
+    smaller sizes."""
+    weights, batch = rag_batch(12, 3000, seed=161, m_range=(16, 16), k_range=(0, 8))
+    weights = (weights % 97) + 1
+    rng = np.random.default_rng(162)
+    prefix = len(weights)
+    weights = np.concatenate([weights, [1 << 33], rng.integers(1 << 30, 1 << 38, size=16, dtype=np.int64)])
+    batch.append([sorted(set(int(x) for x in rng.choice(300, size=5, replace=False))) + [prefix, prefix + 1 + i]
+                  for i in range(16)])
+    batch.append([[x for x in range(16) if x != i] for i in range(16)])
+    batch += rag_batch(10, 3000, seed=163, m_range=(12, 15))[1]
+    assert all(_shared_weight(weights, reqs) < 1 << 16 for reqs in batch if len(reqs) == 16)
     check_batch(mpt, weights, batch)
 
 
