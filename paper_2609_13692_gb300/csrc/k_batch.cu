@@ -443,12 +443,14 @@ constexpr int batch_rows_lanes(int nb) {
   }
   return most;
 }
-// Up to m = 13 every level's lanes and rows fit the block in one pass;
-// beyond, phase A and phase B run in passes.
+// Up to m = 13 every level's lanes fit the block in one pass, beyond it
+// phase A runs in passes; phase B has one thread per row in one pass up to
+// m = 15 and runs in passes at m = 16.
 constexpr bool batch_rows_fit() {
   for (int m = 6; m <= 13; ++m)
-    if (batch_level_rows(m - 5) > batch_rows_threads(m) || batch_rows_lanes(m - 5) > batch_rows_threads(m))
-      return false;
+    if (batch_rows_lanes(m - 5) > batch_rows_threads(m)) return false;
+  for (int m = 6; m < kBGlobalRowsM; ++m)
+    if (batch_level_rows(m - 5) > batch_rows_threads(m)) return false;
   return true;
 }
 static_assert(batch_rows_fit(), "every level of the row-blocked kernel fits its block");
@@ -667,9 +669,9 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       }
       __syncthreads();
     }
-    // phase B: one thread finishes each row of the level (in passes of TPI
-    // rows from m = 14)
-    for (int rb = 0; rb < rows; rb += TPI) {
+    // phase B: one thread finishes each row of the level (one pass up to
+    // m = 15, passes of TPI rows at m = 16)
+    for (int rb = 0; rb < (kGRows ? rows : 1); rb += TPI) {
     const int tr = rb + t;
       if (tr < rows) {
         const uint32_t s1 = colex_unrank((unsigned long long)tr, p1, nb);
