@@ -85,7 +85,7 @@ __device__ __forceinline__ int64_t batch_offset(uint32_t S, int64_t lo, const lo
 template <int TPI>
 __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap, const int64_t* __restrict__ req_off,
                             const int64_t* __restrict__ chunks, int32_t* tkey, uint32_t* tmask, int32_t* cx,
-                            uint32_t* cN, int* roff, int* ndistinct_s) {
+                            uint32_t* cN, int* roff, int* ndistinct_s, int32_t* bflags) {
   int& ndistinct = *ndistinct_s;
   const int t = threadIdx.x;
   const int size = 2 * occ_cap;  // a power of two
@@ -116,6 +116,7 @@ __device__ int batch_gather(int m, int64_t r0, int64_t o0, int occ, int occ_cap,
     const int32_t x = tkey[h];
     if (x >= 0) {
       const int u = atomicAdd(&ndistinct, 1);
+      if (MPT_BAD(bflags, u < occ_cap)) continue;
       cx[u] = x;
       cN[u] = tmask[h];
     }
@@ -235,9 +236,18 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   __shared__ int ndistinct;
   __shared__ int roff[17];  // request offsets relative to o0 (m + 1 <= 17)
   __shared__ unsigned long long off[kBatchOffsets];
+  __shared__ int32_t bflags;  // bounds-checked build: failed checks of this block
   const int t = threadIdx.x;
+  // the shared arrays were sized for max_m and occ_cap (the same decision in
+  // every thread)
+  if (MPT_BAD(&bflags, m >= 1 && m <= max_m && occ <= occ_cap)) {
+    if (t == 0) status[inst] = kErrBounds;
+    return;
+  }
+  if (t == 0) bflags = 0;
   const int nd = batch_gather<kBatchThreads>(m, r0, o0, occ, occ_cap, req_off, chunks,
-                                             reinterpret_cast<int32_t*>(keys), tmask, cx, cN, roff, &ndistinct);
+                                             reinterpret_cast<int32_t*>(keys), tmask, cx, cN, roff, &ndistinct,
+                                             &bflags);
   for (int S = t; S < N; S += kBatchThreads) wI[S] = 0;
   if (t < kBatchOffsets) off[t] = 0;
   __syncthreads();
@@ -302,6 +312,7 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
       if (idx < count && r == 0) {
         F[S] = ((best >> m) - wI[S]) << m;
         split[S] = (uint16_t)(best & (uint32_t)(N - 1));
+        (void)MPT_BAD(&bflags, valid_split(S, best & (uint32_t)(N - 1)));
       }
     }
     __syncthreads();
@@ -348,6 +359,7 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
       if (idx < count && r == 0) {
         F[S] = (uint32_t)(best >> 16) - wI[S];
         split[S] = (uint16_t)(best & 0xFFFFu);
+        (void)MPT_BAD(&bflags, valid_split(S, (uint32_t)(best & 0xFFFFu)));
       }
     }
     __syncthreads();
@@ -378,6 +390,10 @@ k_batch_solve(const int64_t* __restrict__ weights, const int64_t* __restrict__ i
   // 4. hierarchy walk
   __syncthreads();
   batch_walk<kBatchThreads>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  if (kBoundsChecked) {
+    __syncthreads();
+    if (t == 0 && bflags) status[inst] = bflags;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -540,7 +556,8 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
   // the walk reads it there
   const bool gsplit = mm >= kBGlobalSplitM;
   uint32_t* gsp = split_out + tab_off[inst];
-  auto put_split = [&](uint32_t U, uint32_t A) {
+  auto put_split = [&](uint32_t U, uint32_t A, int32_t* bf) {
+    (void)MPT_BAD(bf, valid_split(U, A));
     if (gsplit)
       gsp[U] = A;
     else
@@ -551,8 +568,16 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
 
   __shared__ int roff[17];  // request offsets relative to o0 (m + 1 <= 17)
   __shared__ unsigned long long off[kBatchOffsets];
+  __shared__ int32_t bflags;  // bounds-checked build: failed checks of this block
+  // the shared arrays and the rows were sized for mm and occ_cap (the same
+  // decision in every thread)
+  if (MPT_BAD(&bflags, m == mm && occ <= occ_cap && (!kGRows || rows_scratch))) {
+    if (t == 0) status[inst] = kErrBounds;
+    return;
+  }
+  if (t == 0) bflags = 0;
   const int nd = batch_gather<TPI>(m, r0, o0, occ, occ_cap, req_off, chunks, reinterpret_cast<int32_t*>(keys), tmask,
-                                   cx, cN, roff, &ndistinct);
+                                   cx, cN, roff, &ndistinct, &bflags);
 
   // g, the offsets and the superset sums, in the padded row layout: the five
   // in-row bits per row in registers, then one row-pair pass per row bit
@@ -611,7 +636,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
       }
       zp[s2] = (f << m) + (uint32_t)s2;
       zc[s2] = f << m;
-      put_split((uint32_t)s2, A);
+      put_split((uint32_t)s2, A, &bflags);
     }
 #pragma unroll
     for (int s2 = 0; s2 < kBRow; ++s2) Gp[s2] = zp[s2];
@@ -714,7 +739,7 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
               A = key & mask;
             }
             cc[s2] = f << m;
-            put_split(S1 | (uint32_t)s2, A);
+            put_split(S1 | (uint32_t)s2, A, &bflags);
           }
         }
         uint32_t gp[kBRow];
@@ -751,6 +776,10 @@ k_batch_rows(const int64_t* __restrict__ weights, const int64_t* __restrict__ in
                     status);
   else
     batch_walk<TPI>(inst, m, r0, o0, roff, split, keys, cx, cN, nd, perm_out, dfs_out, status);
+  if (kBoundsChecked) {
+    __syncthreads();
+    if (t == 0 && bflags) status[inst] = bflags;
+  }
 }
 
 }  // namespace

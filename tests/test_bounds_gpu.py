@@ -3,7 +3,9 @@
 It stands in for a device memory checker: the exact-solve kernels test their
 table indices, window offsets and split entries, skip any access that fails
 and report it through the device flags, which mpt_solve turns into
-MPT_ERR_INTERNAL.  Every solve here must therefore succeed and still match the
+MPT_ERR_INTERNAL; the batched kernels test their block's size and
+occurrence cap, their hash-table slots and every split entry, and report
+through the instance's status (MPT_ERR_INTERNAL from mpt_batch_solve).  Every solve here must therefore succeed and still match the
 oracle, in every DP mode and table layout, one-shot and staged.  The checked
 library runs in a child process (MPT_LIBRARY), so the default build this
 session has loaded is untouched.
@@ -62,6 +64,29 @@ CHILD = textwrap.dedent(r"""
     check(I.rag_pools(18, 4000, 4, 60, 8, 1.1, seed=5), tables="lean")
     check(I.rag_pools(17, 4000, 4, 60, 8, 1.1, seed=6), staged=True)
     check(I.with_query_chunks(I.config(1), 1 << 28, 1 << 36, seed=3))
+    # the batched kernels: every size 1..16 (row-blocked and per-subset
+    # kernels, rows in shared and in global memory), F and split per instance
+    rng = np.random.default_rng(17)
+    n = 400
+    bw = rng.integers(1, 60, size=n, dtype=np.int64)
+    groups = []
+    for m in list(range(1, 17)) * 2:
+        pool = rng.choice(n, size=40, replace=False)
+        groups.append([sorted(set(int(x) for x in rng.choice(pool, size=int(rng.integers(1, 7)), replace=False)))
+                       for _ in range(m)])
+    heavy_w = np.concatenate([bw, rng.integers(1 << 18, 1 << 20, size=20, dtype=np.int64)])
+    for m in (5, 9, 13, 15):  # shared weight >= 2^(32 - m): the per-subset kernel's 64-bit keys
+        groups.append([sorted(set(int(x) for x in n + rng.choice(20, size=4, replace=False))) for _ in range(m)])
+    opt, perms, orders, b = mpt.solve_batch(heavy_w, groups)
+    F_all, S_all, offs = mpt.mpt_batch_tables(b)
+    F_all = F_all.cpu().numpy()
+    S_all = S_all.cpu().numpy().view(np.uint32)
+    for i, reqs in enumerate(groups):
+        bits = I.pack_requests(reqs, heavy_w.shape[0])
+        o_opt, oF, owI, osplit = O.solve(heavy_w, bits)
+        assert opt[i] == o_opt, (i, len(reqs), opt[i], o_opt)
+        lo, hi = int(offs[i]), int(offs[i + 1])
+        assert np.array_equal(F_all[lo:hi], oF) and np.array_equal(S_all[lo:hi], osplit), i
     # the pair kernel at scale: workload 3 (m = 24), OPT against its layout's trie cost
     inst = I.config(3)
     res = mpt.solve(inst.weights, inst.bits)
