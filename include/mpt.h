@@ -274,6 +274,9 @@ mpt_status mpt_batch_results(const mpt_batch* b, int64_t* opt, int64_t* perm_chu
 mpt_status mpt_batch_tables(const mpt_batch* b, const int64_t** d_F, const uint32_t** d_split,
                             int64_t* table_offsets);
 
+/* Releases the batch, its library-owned workspace and its side streams.  A
+ * batch object, like a context, is not thread-safe; distinct batches are
+ * independent. */
 void mpt_batch_destroy(mpt_batch* b);
 
 /* Agglomerative common-intersection hierarchy (Sec. 6.2; H_g of Thm 6) and
